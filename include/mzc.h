@@ -1,0 +1,345 @@
+/*
+ * mzc.h -- C ABI of libmzc: prefill over a partially evicted LLM memory state
+ * on one GB300 (sm_103a).
+ *
+ * The paper (mzCache) splits LLM memory into per-layer weight units and
+ * fixed-size KV chunks per layer (Sec. 4.2), evicts them under memory
+ * pressure with a backward-out order (Sec. 4.4), and on the next request
+ * restores them while prefill already runs on the resident units ("zero-wait",
+ * Sec. 1 and Sec. 4.4, Fig. 8b).  Its interface is evict(size) and
+ * restore_generate(input_tokens) (Sec. 5).  This library keeps that model
+ * with the restore paths a GB300 has: a copy of swapped blocks from pinned
+ * host memory to HBM on a side stream, and recompute of a dropped token tail
+ * against the resident prefix (the paper's balance principle of Sec. 4.3
+ * applied to these two paths).
+ *
+ * Conventions for every call:
+ *   - Status codes only; nothing throws or aborts across the ABI.
+ *     mzc_last_error() returns a text for the last failing call on a ctx.
+ *   - The ctx owns every device buffer, the pinned swap store and its two
+ *     CUDA streams.  Pointers passed in are borrowed for the call only
+ *     (mzc_create copies the weights).  Host pointers are plain host memory
+ *     unless a parameter says "device".
+ *   - One ctx per host thread; calls on one ctx must not overlap.  Different
+ *     ctxs share nothing.
+ *   - Token ranges are in absolute positions of the context; KV blocks are
+ *     block_tokens (16) consecutive positions of one layer.
+ */
+#ifndef MZC_H
+#define MZC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MZC_OK = 0,
+  MZC_ERR_INVALID = 1, /* bad argument: null pointer, unsupported shape, illegal eviction shape */
+  MZC_ERR_RANGE = 2,   /* layer / token / block index outside the context or a capacity */
+  MZC_ERR_STATE = 3,   /* not legal in the current residency state (e.g. double evict) */
+  MZC_ERR_OOM = 4,     /* KV pool, row capacity or pinned store exhausted */
+  MZC_ERR_CUDA = 5,    /* a CUDA runtime call failed; the text names it */
+  MZC_ERR_TIMEOUT = 6, /* a bounded device wait gave up (kernel status word) */
+  MZC_ERR_DEVICE = 7   /* a device-side bounds check failed (kernel status word) */
+} mzc_status;
+
+enum { MZC_KV_BF16 = 0, MZC_KV_FP16 = 1 };
+/* eviction modes: COPY = swap to pinned host (restored by copy); DROP =
+ * discard (restored by recompute); AUTO = split by the ctx's policy. */
+enum { MZC_COPY = 0, MZC_DROP = 1, MZC_AUTO = 2 };
+enum { MZC_POLICY_COPY = 0, MZC_POLICY_RECOMPUTE = 1, MZC_POLICY_HYBRID = 2 };
+/* residency of one (layer, logical block) */
+enum { MZC_RESIDENT = 0, MZC_SWAPPED = 1, MZC_DROPPED = 2, MZC_INFLIGHT = 3, MZC_EMPTY = 4 };
+
+/* Decoder shape (Llama-style: RMSNorm, rotary q/k with half-split pairs,
+ * grouped-query attention, SwiGLU MLP, untied LM head, no biases). */
+typedef struct {
+  int32_t n_layers, d_model, n_q_heads, n_kv_heads, head_dim, ffn_dim, vocab;
+  float rope_theta; /* rotary base; angle(pos, i) = pos * theta^(-2i/head_dim) */
+  float rms_eps;
+  int32_t kv_dtype;     /* MZC_KV_BF16 or MZC_KV_FP16 (storage type of K/V) */
+  int32_t block_tokens; /* positions per KV block; must be 16 */
+  int64_t max_ctx;      /* positions the context may hold */
+} mzc_model_shape;
+
+typedef struct {
+  int64_t pool_blocks;      /* physical KV blocks; 0 = 2 * n_layers * ceil(max_ctx/16) */
+  int64_t max_rows;         /* rows per prefill call (recompute + prompt); 0 = max_ctx */
+  int64_t host_store_bytes; /* pinned swap store; 0 = the whole context's KV bytes */
+  int32_t overlap;          /* 1 = zero-wait overlap of restore and prefill; 0 = restore
+                               completes before prefill starts (ablation) */
+  int32_t device;           /* CUDA device ordinal */
+} mzc_options;
+
+/* Weights, host memory, bf16 bit patterns, row-major [out_features][in_features]
+ * (the layout of torch.nn.Linear.weight).  Norm gains are fp32. */
+typedef struct {
+  const uint16_t *wq;     /* [n_q_heads*head_dim][d_model] */
+  const uint16_t *wk;     /* [n_kv_heads*head_dim][d_model] */
+  const uint16_t *wv;     /* [n_kv_heads*head_dim][d_model] */
+  const uint16_t *wo;     /* [d_model][n_q_heads*head_dim] */
+  const uint16_t *w_gate; /* [ffn_dim][d_model] */
+  const uint16_t *w_up;   /* [ffn_dim][d_model] */
+  const uint16_t *w_down; /* [d_model][ffn_dim] */
+  const float *attn_norm; /* [d_model] */
+  const float *ffn_norm;  /* [d_model] */
+} mzc_layer_weights;
+
+typedef struct {
+  const uint16_t *embed;           /* [vocab][d_model] */
+  const uint16_t *lm_head;         /* [vocab][d_model] */
+  const float *final_norm;         /* [d_model] */
+  const mzc_layer_weights *layers; /* [n_layers] */
+} mzc_weights;
+
+/* Per-unit restore rates (the paper's offline profiling, Sec. 4.3: each
+ * path's time per unit, assumed linear in the number of units). */
+typedef struct {
+  double h2d_gbs;     /* pinned host -> HBM copy rate, GB/s */
+  double hbm_gbs;     /* HBM streaming rate, GB/s (weight-bound small-M GEMMs) */
+  double gemm_tflops; /* BF16 GEMM rate at recompute sizes, TFLOP/s */
+  double attn_tflops; /* prefill attention rate, TFLOP/s */
+  double launch_us;   /* fixed cost per layer of one prefill call, microseconds */
+} mzc_profile;
+
+typedef struct {
+  int64_t context_tokens;   /* positions currently in the context */
+  int64_t blocks_resident;  /* (layer, block) pairs by state */
+  int64_t blocks_swapped;
+  int64_t blocks_dropped;
+  int64_t pool_free_blocks;
+  int64_t bytes_h2d_last;   /* KV + weight bytes copied by the last restore */
+  int64_t copies_last;      /* cudaMemcpyAsync calls of the last restore */
+  int64_t rows_last;        /* rows (recompute + prompt) of the last prefill */
+  int64_t recompute_rows_last;
+  int32_t weights_evicted_layers;
+  int32_t reserved;
+} mzc_stats_t;
+
+typedef struct mzc_ctx mzc_ctx;
+
+/* Builds a ctx on options->device: uploads the weights (copied; the caller
+ * keeps ownership of `weights`), allocates the KV block pool, the per-layer
+ * block tables (logical block -> physical block, Sec. 4.2's chunk-pointer
+ * array), the residency table and scratch.  The context starts empty.
+ * options may be NULL (defaults).  On failure *out is NULL. */
+mzc_status mzc_create(const mzc_model_shape *shape, const mzc_options *options,
+                      const mzc_weights *weights, mzc_ctx **out);
+mzc_status mzc_destroy(mzc_ctx *ctx);
+
+/* Prefill: appends tokens[0..n) at positions context_tokens.. and runs, in one
+ * fused pass, those rows together with any pending recompute rows
+ * (mzc_recompute_tail) through every layer.  Each layer's attention waits only
+ * for that layer's restore copies (zero-wait, Sec. 4.4).  Writes the fp32
+ * logits of the last new token to logits_out[vocab] (host), or nothing when
+ * logits_out is NULL or n == 0.  Returns after the logits are on the host.
+ * Errors: MZC_ERR_STATE if any block the rows attend to is SWAPPED without a
+ * restore in flight, or DROPPED without a pending recompute; MZC_ERR_OOM if
+ * the rows exceed max_rows or the pool is full; MZC_ERR_RANGE past max_ctx. */
+mzc_status mzc_prefill(mzc_ctx *ctx, const int32_t *tokens, int64_t n, float *logits_out);
+
+/* Evicts layers [layer_begin, layer_end) x positions [tok_begin, tok_end).
+ * The token range is rounded outward to whole blocks (Sec. 6.2 evicts
+ * slightly more than asked at chunk granularity).  MZC_COPY swaps the blocks
+ * to the pinned store (D2H, packed per layer) and frees their physical
+ * blocks; MZC_DROP frees them for later recompute and is legal only across
+ * all layers, with the dropped positions forming one contiguous range;
+ * MZC_AUTO splits [tok_begin, context_tokens) into a recomputed front and a
+ * copied back by the ctx's policy (mzc_set_policy).  Every block in range
+ * must be RESIDENT (else MZC_ERR_STATE, nothing changes).  Synchronous. */
+mzc_status mzc_evict(mzc_ctx *ctx, int32_t layer_begin, int32_t layer_end, int64_t tok_begin,
+                     int64_t tok_end, int32_t mode);
+/* Fine-grained COPY eviction of n scattered (layer[i], logical_block[i]). */
+mzc_status mzc_evict_blocks(mzc_ctx *ctx, const int32_t *layer, const int64_t *logical_block,
+                            int64_t n, int32_t mode);
+/* Evicts the weights of layers [layer_begin, layer_end) (Sec. 4.2: one unit per
+ * layer) to a pinned host copy; restored per layer by mzc_restore_async. */
+mzc_status mzc_evict_weights(mzc_ctx *ctx, int32_t layer_begin, int32_t layer_end);
+
+/* Enqueues the restore of every swapped unit on the copy stream, forward-in
+ * (Sec. 4.4: earliest layer first): per layer, the weight unit, then one
+ * host->device copy per packed run of KV blocks into contiguous free physical
+ * blocks; then records that layer's event.  Returns without waiting. */
+mzc_status mzc_restore_async(mzc_ctx *ctx);
+
+/* Declares the recompute of dropped positions [p, p+n): they are re-prefilled
+ * against the resident prefix in the next mzc_prefill (or mzc_sync), fused
+ * with its prompt rows.  [p, p+n) must equal the dropped range (MZC_ERR_RANGE
+ * otherwise). */
+mzc_status mzc_recompute_tail(mzc_ctx *ctx, int64_t p, int64_t n);
+
+/* Sets the policy MZC_AUTO evictions use and the per-unit profile that sizes
+ * the hybrid split (profile may be NULL to keep the current one). */
+mzc_status mzc_set_policy(mzc_ctx *ctx, int32_t policy, const mzc_profile *profile);
+
+/* Hybrid split (pure host arithmetic): for an evicted tail [p, n_ctx) and a
+ * prompt of n_prompt tokens, the block-aligned s in [p, n_ctx] at which the
+ * recompute of [p, s) and the copy of [s, n_ctx) finish together, i.e. that
+ * minimises max(T_recompute(p, s) + T_prompt, T_copy(s, n_ctx)) under the
+ * profile's linear per-unit costs (Sec. 4.3, split in inverse proportion to
+ * per-unit times). */
+mzc_status mzc_plan_split(const mzc_model_shape *shape, const mzc_profile *profile, int64_t p,
+                          int64_t n_ctx, int64_t n_prompt, int64_t *s_out);
+
+/* Measures the per-unit profile on this ctx's device (the paper's one-time
+ * offline profiling, Sec. 4.3): timed host->device copies from the pinned
+ * store, and the ctx's own GEMM and attention kernels on scratch. */
+mzc_status mzc_profile_measure(mzc_ctx *ctx, mzc_profile *out);
+
+/* Shrinks the context to n_ctx positions (frees the blocks past it). */
+mzc_status mzc_truncate(mzc_ctx *ctx, int64_t n_ctx);
+/* Runs any pending recompute, waits for both streams, and surfaces device
+ * status words (MZC_ERR_TIMEOUT / MZC_ERR_DEVICE). */
+mzc_status mzc_sync(mzc_ctx *ctx);
+
+/* Residency of (layer, logical_block) and its physical block (-1 if none). */
+mzc_status mzc_query(mzc_ctx *ctx, int32_t layer, int64_t logical_block, int32_t *state,
+                     int32_t *phys);
+/* Reads one resident block's K and V ([n_kv_heads][16][head_dim], KV dtype
+ * bits) into host buffers of block_bytes/2 each. */
+mzc_status mzc_read_kv(mzc_ctx *ctx, int32_t layer, int64_t logical_block, void *k_host,
+                       void *v_host);
+/* Reads K and V of every position [0, n) of every layer, widened to fp32,
+ * into host arrays [n_layers][n][n_kv_heads][head_dim].  Every block must be
+ * RESIDENT. */
+mzc_status mzc_read_kv_all(mzc_ctx *ctx, int64_t n, float *k_host, float *v_host);
+mzc_status mzc_stats(mzc_ctx *ctx, mzc_stats_t *out);
+/* Device time in ms of the last mzc_prefill: [0] the call on the compute
+ * stream, [1] restore copies on the copy stream, [2] LM head, [3] TTFT on the
+ * device: from the start of the restore copies (or of the prefill when
+ * nothing was restored) to the logits' arrival in host memory.  ms must hold
+ * 4 floats; -1 marks a phase that did not run. */
+mzc_status mzc_last_times(mzc_ctx *ctx, float *ms3);
+const char *mzc_last_error(mzc_ctx *ctx);
+
+/* Kernel classes of the prefill path, for launch counts and timing. */
+enum {
+  MZC_K_GEMM = 0,      /* projections (tcgen05) */
+  MZC_K_ATTENTION = 1, /* block-table attention (+ split-KV combine) */
+  MZC_K_ROPE_KV = 2,   /* rotary + KV-block write */
+  MZC_K_RMSNORM = 3,
+  MZC_K_LM_HEAD = 4,
+  MZC_K_EMBED = 5,
+  MZC_K_NCLASS = 6
+};
+typedef struct {
+  int64_t launches; /* kernels launched (always counted) */
+  double ms;        /* summed CUDA-event duration on the compute stream (timing on) */
+  double flops;     /* algorithmic FLOPs of those launches */
+  double bytes;     /* algorithmic HBM bytes of those launches */
+} mzc_kernel_stat;
+/* on != 0: bracket every kernel of mzc_prefill with CUDA events on the
+ * compute stream.  Either way, resets the per-class counters. */
+mzc_status mzc_set_kernel_timing(mzc_ctx *ctx, int32_t on);
+mzc_status mzc_kernel_stats(mzc_ctx *ctx, int32_t kernel_class, mzc_kernel_stat *out);
+
+/* ---------------------------------------------------------------------------
+ * Host bookkeeping without a device (no CUDA call is made): the residency
+ * table, block tables, physical-block allocator and restore planner the ctx
+ * uses, for planning and for tests.  Same rules and status codes as above.
+ */
+typedef struct mzc_state mzc_state;
+
+/* One planned host->device copy: n_blocks blocks of `layer` from host store
+ * offset host_off to physical blocks [phys_begin, phys_begin + n_blocks). */
+typedef struct {
+  int32_t layer;
+  int32_t n_blocks;
+  int64_t host_off;
+  int64_t phys_begin;
+} mzc_copy_run;
+
+mzc_status mzc_state_create(const mzc_model_shape *shape, int64_t pool_blocks,
+                            int64_t host_store_bytes, mzc_state **out);
+mzc_status mzc_state_destroy(mzc_state *st);
+/* Context grows by n positions (what mzc_prefill does to the state). */
+mzc_status mzc_state_append(mzc_state *st, int64_t n);
+mzc_status mzc_state_evict(mzc_state *st, int32_t layer_begin, int32_t layer_end,
+                           int64_t tok_begin, int64_t tok_end, int32_t mode);
+mzc_status mzc_state_evict_blocks(mzc_state *st, const int32_t *layer,
+                                  const int64_t *logical_block, int64_t n, int32_t mode);
+mzc_status mzc_state_recompute_tail(mzc_state *st, int64_t p, int64_t n);
+/* Plans the restore of every swapped block (forward-in); swapped blocks
+ * become INFLIGHT.  Writes up to cap runs; *n_runs is the number planned
+ * (MZC_ERR_OOM with nothing changed if cap is too small). */
+mzc_status mzc_state_plan_restore(mzc_state *st, mzc_copy_run *runs, int64_t cap,
+                                  int64_t *n_runs);
+/* Completes the restore and any pending recompute: INFLIGHT and recomputed
+ * blocks become RESIDENT. */
+mzc_status mzc_state_complete(mzc_state *st);
+mzc_status mzc_state_truncate(mzc_state *st, int64_t n_ctx);
+mzc_status mzc_state_query(mzc_state *st, int32_t layer, int64_t logical_block, int32_t *state,
+                           int32_t *phys);
+mzc_status mzc_state_counts(mzc_state *st, mzc_stats_t *out);
+
+/* ---------------------------------------------------------------------------
+ * Single kernels of the prefill path, for parity tests and profiling.  All
+ * pointers are DEVICE pointers; `stream` is a cudaStream_t (NULL = default
+ * stream).  Launch errors return MZC_ERR_CUDA; the calls do not synchronize.
+ */
+
+/* y[n][d] (fp16) = x / sqrt(mean(x^2) + eps) * g, x fp32 [n][d] (RMSNorm). */
+mzc_status mzc_k_rmsnorm(const float *x, const float *g, int64_t n, int32_t d, float eps,
+                         uint16_t *y, void *stream);
+
+/* C = A W^T with A fp16 [m][k] and W fp16 [n][k] (IEEE half bits, both
+ * row-major, K-major), fp32 accumulation on tcgen05 tensor cores.  (The ctx
+ * converts the bf16 model weights to fp16 at creation; fp16 activations keep
+ * 3 more mantissa bits than bf16 at the same tensor-core rate.)  epilogue:
+ *   0: out fp16 [m][n] = C
+ *   1: out fp32 [m][n] += C                       (residual add)
+ *   2: out fp16 [m][n/2] = silu(C_gate) * C_up     (SwiGLU; W's rows must be in
+ *      the interleaved order mzc_k_swiglu_pack produces)
+ * k must be a multiple of 8; n a multiple of 16 (epilogue 2: of 128). */
+mzc_status mzc_k_gemm(const uint16_t *a, const uint16_t *w, void *out, int64_t m, int64_t n,
+                      int64_t k, int32_t epilogue, void *stream);
+/* Host helper: interleaves gate [f][d] and up [f][d] into the [2f][d] row
+ * order epilogue 2 reads (per 64 output features: 64 gate rows then the
+ * matching 64 up rows).  f must be a multiple of 64. */
+mzc_status mzc_k_swiglu_pack(const uint16_t *gate, const uint16_t *up, int64_t f, int64_t d,
+                             uint16_t *out_host);
+
+/* Rotary embedding of q and k and the KV-block write.
+ * qkv fp16 [n][(hq + 2*hkv)*hd] (q heads, then k heads, then v heads),
+ * pos int32 [n], cos/sin fp32 [max_pos][hd/2] (angle pos*theta^(-2i/hd)),
+ * block_table int32 [n_logical] -> physical block, pool: block b holds
+ * K [hkv][16][hd] then V [hkv][16][hd] in the KV dtype.
+ * Out: q_out [n][hq][hd] rotated, in the KV dtype (the attention's operand type); K/V stored at pool[table[pos/16]]
+ * slot pos%16.  cos_t/sin_t must cover positions < n_logical*16.  status
+ * (device int32, may be NULL) gets MZC_ERR_DEVICE on a bad index or block. */
+mzc_status mzc_k_rope_kv_write(const uint16_t *qkv, const int32_t *pos, int64_t n, int32_t hq,
+                               int32_t hkv, int32_t hd, const float *cos_t, const float *sin_t,
+                               const int32_t *block_table, int64_t n_logical, void *pool,
+                               int64_t pool_blocks, int32_t kv_dtype, uint16_t *q_out,
+                               int32_t *status, void *stream);
+
+/* Causal grouped-query attention over a block-table KV cache (the paper's
+ * attention over non-contiguous KV chunks with online softmax, Sec. 4.2).
+ * q [n][hq][hd] in the KV dtype at positions pos int32 [n]; row i attends to
+ * every position <= pos[i] through block_table; out fp16 [n][hq][hd].
+ * max_keys: an upper bound of pos[i] + 1 (sizes the split of long key
+ * ranges).  scratch: device buffer of mzc_k_attention_scratch_bytes() bytes
+ * for the split-KV partials, or NULL to run without splitting. */
+mzc_status mzc_k_attention(const uint16_t *q, const int32_t *pos, int64_t n, int32_t hq,
+                           int32_t hkv, int32_t hd, const int32_t *block_table, int64_t n_logical,
+                           const void *pool, int64_t pool_blocks, int32_t kv_dtype,
+                           uint16_t *out, int64_t max_keys, void *scratch, int64_t scratch_bytes,
+                           int32_t *status, void *stream);
+int64_t mzc_k_attention_scratch_bytes(int64_t n, int32_t hq, int32_t hkv, int32_t hd,
+                                      int64_t max_keys);
+
+/* logits fp32 [vocab] = RMSNorm(x_row) * g  W^T, x_row fp32 [d], W bf16 [vocab][d]. */
+mzc_status mzc_k_lm_head(const float *x_row, const float *g, int32_t d, float eps,
+                         const uint16_t *w, int64_t vocab, float *logits, void *stream);
+
+/* x fp32 [n][d] = embed[tokens[i]] widened (bf16 -> fp32). */
+mzc_status mzc_k_embed(const int32_t *tokens, int64_t n, const uint16_t *embed, int32_t d,
+                       int64_t vocab, float *x, int32_t *status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MZC_H */

@@ -1,0 +1,302 @@
+// Memory-bound kernels of the prefill path: embedding gather, RMSNorm,
+// rotary embedding fused with the KV-block write, the LM-head GEMV, and the
+// block gather/poison used by eviction.  All global accesses are 16-byte
+// vectors along the contiguous dimension.
+#include <cstdio>
+
+#include "kernels.hpp"
+#include "ptx.cuh"
+
+namespace mzc {
+
+namespace {
+
+__device__ __forceinline__ float bf16_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+
+__device__ __forceinline__ void unpack8_f16(const uint4& v, float* f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 t = __half22float2(*reinterpret_cast<const __half2*>(&w[i]));
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+
+__device__ __forceinline__ void unpack8_bf16(const uint4& v, float* f) {
+  f[0] = bf16_lo(v.x); f[1] = bf16_hi(v.x);
+  f[2] = bf16_lo(v.y); f[3] = bf16_hi(v.y);
+  f[4] = bf16_lo(v.z); f[5] = bf16_hi(v.z);
+  f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
+}
+
+template <bool F16>
+__device__ __forceinline__ uint4 pack8(const float* f) {
+  return make_uint4(pack2<F16>(f[0], f[1]), pack2<F16>(f[2], f[3]), pack2<F16>(f[4], f[5]),
+                    pack2<F16>(f[6], f[7]));
+}
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  float t = lane < nw ? red[lane] : 0.0f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  __syncthreads();
+  return t;
+}
+
+// x[i][:] = embed[tokens[i]][:] widened to fp32; one CTA per row.
+__global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t* __restrict__ emb,
+                             int d, int64_t vocab, float* __restrict__ x, int32_t* status) {
+  const int64_t i = blockIdx.x;
+  const int32_t t = tokens[i];
+  if (t < 0 || t >= vocab) {
+    if (threadIdx.x == 0) set_status(status, kStatusDevice);
+    return;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(emb + static_cast<int64_t>(t) * d);
+  float4* dst = reinterpret_cast<float4*>(x + i * d);
+  for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+    float f[8];
+    unpack8_bf16(src[c], f);
+    dst[2 * c] = make_float4(f[0], f[1], f[2], f[3]);
+    dst[2 * c + 1] = make_float4(f[4], f[5], f[6], f[7]);
+  }
+}
+
+// y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, fp16 out; one CTA per row.
+__global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g, int d,
+                               float eps, uint16_t* __restrict__ y) {
+  __shared__ float red[32];
+  const int64_t i = blockIdx.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + i * d);
+  float ss = 0.0f;
+  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) {
+    float4 v = xr[c];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / static_cast<float>(d) + eps);
+  const float4* gr = reinterpret_cast<const float4*>(g);
+  uint4* yr = reinterpret_cast<uint4*>(y + i * d);
+  for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
+    float4 a = xr[2 * c], b = xr[2 * c + 1], ga = gr[2 * c], gb = gr[2 * c + 1];
+    float f[8] = {a.x * r * ga.x, a.y * r * ga.y, a.z * r * ga.z, a.w * r * ga.w,
+                  b.x * r * gb.x, b.y * r * gb.y, b.z * r * gb.z, b.w * r * gb.w};
+    yr[c] = pack8<true>(f);
+  }
+}
+
+// Rotary embedding (pairs (i, i + hd/2), angle pos * theta^(-2i/hd) from the
+// fp32 tables) of q and k (fp16 projection output), then K/V stored into
+// their KV block slot:
+// pool[table[pos/16]] = K [hkv][16][hd] then V [hkv][16][hd], slot pos % 16.
+// q goes to q_out [n][hq][hd] in the KV dtype.  One CTA per row.
+template <bool F16>
+__global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* __restrict__ pos,
+                               int hq, int hkv, int hd, const float* __restrict__ cos_t,
+                               const float* __restrict__ sin_t, const int32_t* __restrict__ table,
+                               int64_t n_logical, uint16_t* __restrict__ pool,
+                               int64_t pool_blocks, uint16_t* __restrict__ q_out,
+                               int32_t* status) {
+  const int64_t i = blockIdx.x;
+  const int p = pos[i];
+  const int half = hd / 2;
+  const int64_t blk = p >> 4;
+  if (p < 0 || blk >= n_logical) {  // the rotary tables cover positions < n_logical * 16
+    if (threadIdx.x == 0) set_status(status, kStatusDevice);
+    return;
+  }
+  const int32_t phys = table[blk];
+  const bool kv_ok = phys >= 0 && phys < pool_blocks;
+  if (!kv_ok && threadIdx.x == 0) set_status(status, kStatusDevice);
+  const int64_t blk_elems = 2LL * hkv * 16 * hd;
+  uint16_t* kbase = pool + (kv_ok ? phys : 0) * blk_elems;
+  uint16_t* vbase = kbase + static_cast<int64_t>(hkv) * 16 * hd;
+  const int slot = p & 15;
+  const uint16_t* row = qkv + i * static_cast<int64_t>(hq + 2 * hkv) * hd;
+  const int rot_chunks = half / 8;              // 8-element chunks per half
+  const int n_rot = (hq + hkv) * rot_chunks;    // q and k heads
+  const int n_v = hkv * (hd / 8);
+  const float* cs = cos_t + static_cast<int64_t>(p) * half;
+  const float* sn = sin_t + static_cast<int64_t>(p) * half;
+  for (int w = threadIdx.x; w < n_rot + n_v; w += blockDim.x) {
+    if (w < n_rot) {
+      const int head = w / rot_chunks, c = (w % rot_chunks) * 8;
+      const uint16_t* src = row + static_cast<int64_t>(head) * hd;
+      float x1[8], x2[8], y1[8], y2[8];
+      unpack8_f16(*reinterpret_cast<const uint4*>(src + c), x1);
+      unpack8_f16(*reinterpret_cast<const uint4*>(src + c + half), x2);
+      const float4 c0 = *reinterpret_cast<const float4*>(cs + c);
+      const float4 c1 = *reinterpret_cast<const float4*>(cs + c + 4);
+      const float4 s0 = *reinterpret_cast<const float4*>(sn + c);
+      const float4 s1 = *reinterpret_cast<const float4*>(sn + c + 4);
+      const float cc[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+      const float ss[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        y1[j] = x1[j] * cc[j] - x2[j] * ss[j];
+        y2[j] = x2[j] * cc[j] + x1[j] * ss[j];
+      }
+      uint16_t* dst;
+      if (head < hq) {
+        dst = q_out + (i * hq + head) * hd;
+      } else {
+        if (!kv_ok) continue;
+        dst = kbase + (static_cast<int64_t>(head - hq) * 16 + slot) * hd;
+      }
+      *reinterpret_cast<uint4*>(dst + c) = pack8<F16>(y1);
+      *reinterpret_cast<uint4*>(dst + c + half) = pack8<F16>(y2);
+    } else {
+      if (!kv_ok) continue;
+      const int v = w - n_rot;
+      const int head = v / (hd / 8), c = (v % (hd / 8)) * 8;
+      const uint16_t* src = row + static_cast<int64_t>(hq + hkv + head) * hd + c;
+      uint4 raw = *reinterpret_cast<const uint4*>(src);
+      uint16_t* dst = vbase + (static_cast<int64_t>(head) * 16 + slot) * hd + c;
+      if constexpr (!F16) {  // fp16 projection output -> bf16 KV
+        float f[8];
+        unpack8_f16(raw, f);
+        raw = pack8<false>(f);
+      }
+      *reinterpret_cast<uint4*>(dst) = raw;
+    }
+  }
+}
+
+// logits[v] = sum_k h[k] * W[v][k], h = RMSNorm(x_row) * g kept in fp32.
+// Each CTA normalises the row into shared memory, then every warp streams
+// whole vocabulary rows (16-byte loads, 4 rows in flight per warp).
+__global__ void __launch_bounds__(256) lm_head_kernel(const float* __restrict__ x,
+                                                      const float* __restrict__ g, int d,
+                                                      float eps, const uint16_t* __restrict__ w,
+                                                      int64_t vocab, float* __restrict__ logits) {
+  extern __shared__ float sh[];
+  __shared__ float red[32];
+  float ss = 0.0f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    float v = x[c];
+    ss += v * v;
+  }
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / static_cast<float>(d) + eps);
+  for (int c = threadIdx.x; c < d; c += blockDim.x) sh[c] = x[c] * r * g[c];
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t gw = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
+  const int64_t nw = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  const int chunks = d / 8;
+  constexpr int R = 4;
+  for (int64_t v0 = gw * R; v0 < vocab; v0 += nw * R) {
+    float acc[R] = {0.f, 0.f, 0.f, 0.f};
+    for (int c = lane; c < chunks; c += 32) {
+      float hv[8];
+      const float4 h0 = *reinterpret_cast<const float4*>(sh + c * 8);
+      const float4 h1 = *reinterpret_cast<const float4*>(sh + c * 8 + 4);
+      hv[0] = h0.x; hv[1] = h0.y; hv[2] = h0.z; hv[3] = h0.w;
+      hv[4] = h1.x; hv[5] = h1.y; hv[6] = h1.z; hv[7] = h1.w;
+      uint4 wv[R];
+#pragma unroll
+      for (int j = 0; j < R; ++j)
+        if (v0 + j < vocab)
+          wv[j] = __ldcs(reinterpret_cast<const uint4*>(w + (v0 + j) * d) + c);
+#pragma unroll
+      for (int j = 0; j < R; ++j) {
+        if (v0 + j < vocab) {
+          float f[8];
+          unpack8_bf16(wv[j], f);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[j] += hv[e] * f[e];
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < R; ++j) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], o);
+      if (lane == 0 && v0 + j < vocab) logits[v0 + j] = acc[j];
+    }
+  }
+}
+
+__global__ void gather_blocks_kernel(const uint4* __restrict__ pool, const int32_t* __restrict__ phys,
+                                     int64_t chunks_per_block, uint4* __restrict__ dst) {
+  const int64_t b = blockIdx.x;
+  const uint4* src = pool + static_cast<int64_t>(phys[b]) * chunks_per_block;
+  uint4* d = dst + b * chunks_per_block;
+  for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = src[c];
+}
+
+__global__ void poison_blocks_kernel(uint4* __restrict__ pool, const int32_t* __restrict__ phys,
+                                     int64_t chunks_per_block) {
+  const int64_t b = blockIdx.x;
+  uint4* d = pool + static_cast<int64_t>(phys[b]) * chunks_per_block;
+  const uint4 nan = make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu);
+  for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = nan;
+}
+
+}  // namespace
+
+cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
+                         int64_t vocab, float* x, int32_t* status, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  embed_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(tokens, embed, d, vocab, x, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
+                           uint16_t* y, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  rmsnorm_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(x, g, d, eps, y);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_t n, int32_t hq,
+                                 int32_t hkv, int32_t hd, const float* cos_t, const float* sin_t,
+                                 const int32_t* table, int64_t n_logical, void* pool,
+                                 int64_t pool_blocks, int32_t kv_dtype, uint16_t* q_out,
+                                 int32_t* status, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  if (kv_dtype == 1)
+    rope_kv_kernel<true><<<static_cast<unsigned>(n), 128, 0, st>>>(
+        qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
+        pool_blocks, q_out, status);
+  else
+    rope_kv_kernel<false><<<static_cast<unsigned>(n), 128, 0, st>>>(
+        qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
+        pool_blocks, q_out, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float eps,
+                           const uint16_t* w, int64_t vocab, float* logits, int num_sms,
+                           cudaStream_t st) {
+  const int grid = num_sms * 4;
+  lm_head_kernel<<<grid, 256, static_cast<size_t>(d) * sizeof(float), st>>>(x_row, g, d, eps, w,
+                                                                            vocab, logits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t n,
+                                 int64_t block_bytes, void* dst, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  gather_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(
+      static_cast<const uint4*>(pool), phys, block_bytes / 16, static_cast<uint4*>(dst));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
+                                 cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), phys,
+                                                                  block_bytes / 16);
+  return cudaGetLastError();
+}
+
+}  // namespace mzc

@@ -1,0 +1,64 @@
+// Launchers of the prefill-path kernels (host side).  Each returns the
+// cudaError_t of its launch; none synchronizes.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace mzc {
+
+enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
+
+// Row group of the SwiGLU weight interleave: 64 gate rows, then the matching
+// 64 up rows, repeated.  The fused epilogue needs both halves in one tile.
+constexpr int kSwigluGroup = 64;
+
+// A 2-D fp16 tensor map [rows][cols] (cols contiguous) with a box of
+// 64 columns x box_rows rows and 128-byte swizzle (the UMMA K-major layout).
+bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
+                    uint32_t box_rows);
+
+// A weight operand W [n][k] with one tensor map per tile width the GEMM may
+// pick (box rows 64 and 128).
+struct GemmWeight {
+  CUtensorMap box64, box128;
+};
+bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
+
+// C = A W^T; A map [>= m][k] with box rows 128.  The W map used is the one
+// whose box matches the tile width gemm_box_n(m, n, epilogue) selects.
+uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
+cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
+                        int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st);
+
+cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
+                         int64_t vocab, float* x, int32_t* status, cudaStream_t st);
+cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
+                           uint16_t* y, cudaStream_t st);
+cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_t n, int32_t hq,
+                                 int32_t hkv, int32_t hd, const float* cos_t, const float* sin_t,
+                                 const int32_t* table, int64_t n_logical, void* pool,
+                                 int64_t pool_blocks, int32_t kv_dtype, uint16_t* q_out,
+                                 int32_t* status, cudaStream_t st);
+// Split-KV plan: how many key splits a launch of n rows over at most
+// max_keys keys uses, and the keys per split (a multiple of 64).
+void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int num_sms,
+                     int* n_splits, int* keys_per_split);
+int64_t attention_scratch_bytes(int64_t n, int32_t hq, int32_t hd, int n_splits);
+cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
+                             int32_t hkv, int32_t hd, const int32_t* table, int64_t n_logical,
+                             const void* pool, int64_t pool_blocks, int32_t kv_dtype,
+                             uint16_t* out, void* scratch, int64_t scratch_bytes,
+                             int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st);
+cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float eps,
+                           const uint16_t* w, int64_t vocab, float* logits, int num_sms,
+                           cudaStream_t st);
+// Copies blocks phys[i] (block_bytes each) of the pool to dst + i*block_bytes.
+cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t n,
+                                 int64_t block_bytes, void* dst, cudaStream_t st);
+// Fills blocks phys[i] with 0xFF bytes (NaN in bf16 and fp16).
+cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
+                                 cudaStream_t st);
+
+}  // namespace mzc

@@ -1,0 +1,1121 @@
+// libmzc runtime: the C ABI of include/mzc.h.
+//
+// A ctx owns, on one device:
+//   - the weights, one contiguous slot per layer (QKV rows q|k|v, O, gate/up
+//     interleaved in groups of 64 rows, down padded to a multiple of 64
+//     features), so that evicting or restoring a layer's weights is one copy
+//     (the paper's per-layer weight unit, Sec. 4.2);
+//   - the KV block pool: physical block b holds one layer's K [hkv][16][hd]
+//     then V [hkv][16][hd] for 16 positions; the per-layer block tables map
+//     logical blocks to physical ones (the chunk-pointer array, Sec. 4.2);
+//   - activations for max_rows rows, split-KV scratch, rotary tables;
+//   - a compute stream and a copy stream, with per-layer events recorded by
+//     the restore on the copy stream; each layer's attention waits only on
+//     its own layer's event (zero-wait, Sec. 4.4);
+//   - the pinned swap store (allocated on the first COPY eviction) and the
+//     pinned master copies of evicted layer weights.
+// Host bookkeeping (residency, allocation, restore planning) is state.cpp.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.hpp"
+#include "mzc.h"
+#include "state.hpp"
+
+using mzc::ceil_div;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+struct LayerDev {
+  uint8_t* base = nullptr;  // slot start (device)
+  size_t bytes = 0;
+  uint16_t *wqkv = nullptr, *wo = nullptr, *w13 = nullptr, *w2 = nullptr;
+  float *attn_norm = nullptr, *ffn_norm = nullptr;
+  mzc::GemmWeight tm_qkv, tm_o, tm_13, tm_2;
+  uint8_t* host_master = nullptr;  // pinned, allocated on first eviction
+};
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+mzc_profile default_profile() {
+  mzc_profile p;
+  p.h2d_gbs = 200.0;
+  p.hbm_gbs = 6000.0;
+  p.gemm_tflops = 1000.0;
+  p.attn_tflops = 400.0;
+  p.launch_us = 30.0;
+  return p;
+}
+
+}  // namespace
+
+struct mzc_ctx {
+  mzc::State st;
+  mzc_model_shape shape{};
+  mzc_options opt{};
+  int num_sms = 0;
+  int64_t f_pad = 0, qkv_dim = 0, max_rows = 0, nblk = 0, block_bytes = 0;
+  cudaStream_t cs = nullptr, xs = nullptr;
+  std::vector<LayerDev> layers;
+  uint8_t* d_weights = nullptr;
+  uint16_t *d_embed = nullptr, *d_lm = nullptr;
+  float* d_fnorm = nullptr;
+  uint8_t* d_pool = nullptr;
+  float *d_cos = nullptr, *d_sin = nullptr;
+  float* d_x = nullptr;
+  uint16_t *d_h = nullptr, *d_qkv = nullptr, *d_q = nullptr, *d_attn = nullptr, *d_act = nullptr;
+  CUtensorMap tm_h, tm_attn, tm_act;
+  uint8_t* d_meta = nullptr;  // tokens | pos | block tables
+  uint8_t* h_meta = nullptr;
+  size_t meta_bytes = 0;
+  float* d_logits = nullptr;
+  float* h_logits = nullptr;
+  void* d_scratch = nullptr;
+  int64_t scratch_bytes = 0;
+  int32_t* d_status = nullptr;
+  uint8_t* h_store = nullptr;
+  uint8_t* d_staging = nullptr;
+  int32_t* d_list = nullptr;
+  int32_t* h_list = nullptr;
+  uint8_t* h_staging = nullptr;  // pinned, one layer of blocks (reads)
+  std::vector<cudaEvent_t> ev_kv, ev_w;
+  cudaEvent_t ev_t0 = nullptr, ev_t1 = nullptr, ev_c0 = nullptr, ev_c1 = nullptr,
+              ev_l0 = nullptr, ev_l1 = nullptr;
+  bool restore_issued = false, lm_timed = false, ttft_from_copy = false;
+  // per-class launch counts and optional CUDA-event timing
+  bool ktime = false;
+  mzc_kernel_stat kstat[MZC_K_NCLASS] = {};
+  struct KEv {
+    int cls;
+    cudaEvent_t a, b;
+    double flops, bytes;
+  };
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<KEv> kev;
+  size_t ev_next = 0;
+  std::vector<int32_t> tokens;
+  int32_t policy = MZC_POLICY_COPY;
+  mzc_profile prof = default_profile();
+  mzc_stats_t last{};
+  std::string err;
+
+  mzc_status fail(mzc_status s, const std::string& m) {
+    err = m;
+    return s;
+  }
+  mzc_status from_state(mzc_status s) {
+    if (s != MZC_OK) err = st.error();
+    return s;
+  }
+};
+
+#define CK(call)                                                                          \
+  do {                                                                                    \
+    cudaError_t e_ = (call);                                                              \
+    if (e_ != cudaSuccess)                                                                \
+      return ctx->fail(MZC_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+namespace {
+
+mzc_status destroy_impl(mzc_ctx* ctx) {
+  if (!ctx) return MZC_ERR_INVALID;
+  cudaSetDevice(ctx->opt.device);
+  if (ctx->cs) cudaStreamSynchronize(ctx->cs);
+  if (ctx->xs) cudaStreamSynchronize(ctx->xs);
+  for (auto& L : ctx->layers)
+    if (L.host_master) cudaFreeHost(L.host_master);
+  void* dev[] = {ctx->d_weights, ctx->d_embed, ctx->d_lm,      ctx->d_fnorm,   ctx->d_pool,
+                 ctx->d_cos,     ctx->d_sin,   ctx->d_x,       ctx->d_h,       ctx->d_qkv,
+                 ctx->d_q,       ctx->d_attn,  ctx->d_act,     ctx->d_meta,    ctx->d_logits,
+                 ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list};
+  for (void* p : dev)
+    if (p) cudaFree(p);
+  void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging};
+  for (void* p : host)
+    if (p) cudaFreeHost(p);
+  for (auto e : ctx->ev_pool) cudaEventDestroy(e);
+  for (auto e : ctx->ev_kv) cudaEventDestroy(e);
+  for (auto e : ctx->ev_w) cudaEventDestroy(e);
+  cudaEvent_t evs[] = {ctx->ev_t0, ctx->ev_t1, ctx->ev_c0, ctx->ev_c1, ctx->ev_l0, ctx->ev_l1};
+  for (auto e : evs)
+    if (e) cudaEventDestroy(e);
+  if (ctx->cs) cudaStreamDestroy(ctx->cs);
+  if (ctx->xs) cudaStreamDestroy(ctx->xs);
+  delete ctx;
+  return MZC_OK;
+}
+
+// bf16 weights -> fp16 GEMM operands (round to nearest even).  Exact for
+// every bf16 value in [2^-14, 65504]; smaller magnitudes round to fp16
+// subnormals (absolute error <= 2^-25).  Returns false if a value would
+// overflow fp16.
+bool bf16_to_f16(const uint16_t* src, uint16_t* dst, int64_t n) {
+  bool ok = true;
+  for (int64_t i = 0; i < n; ++i) {
+    uint32_t u = static_cast<uint32_t>(src[i]) << 16;
+    float f;
+    std::memcpy(&f, &u, 4);
+    if (!(std::fabs(f) <= 65504.0f)) ok = false;
+    __half h = __float2half_rn(f);
+    dst[i] = __half_as_ushort(h);
+  }
+  return ok;
+}
+
+// Converts one layer's canonical bf16 weights into its packed fp16 host image.
+bool pack_layer(const mzc_model_shape& s, int64_t f_pad, const mzc_layer_weights& w,
+                std::vector<uint8_t>& img, const LayerDev& L) {
+  const int64_t d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim, f = s.ffn_dim;
+  std::fill(img.begin(), img.end(), 0);
+  auto off = [&](const void* dev) { return static_cast<size_t>(static_cast<const uint8_t*>(dev) - L.base); };
+  bool ok = true;
+  uint16_t* qkv = reinterpret_cast<uint16_t*>(img.data() + off(L.wqkv));
+  ok &= bf16_to_f16(w.wq, qkv, hq * hd * d);
+  ok &= bf16_to_f16(w.wk, qkv + hq * hd * d, hkv * hd * d);
+  ok &= bf16_to_f16(w.wv, qkv + (hq + hkv) * hd * d, hkv * hd * d);
+  ok &= bf16_to_f16(w.wo, reinterpret_cast<uint16_t*>(img.data() + off(L.wo)), d * hq * hd);
+  uint16_t* w13 = reinterpret_cast<uint16_t*>(img.data() + off(L.w13));
+  const int64_t G = mzc::kSwigluGroup;
+  for (int64_t j = 0; j < f; ++j) {
+    const int64_t grp = j / G, r = j % G;
+    ok &= bf16_to_f16(w.w_gate + j * d, w13 + (grp * 2 * G + r) * d, d);
+    ok &= bf16_to_f16(w.w_up + j * d, w13 + (grp * 2 * G + G + r) * d, d);
+  }
+  uint16_t* w2 = reinterpret_cast<uint16_t*>(img.data() + off(L.w2));
+  for (int64_t r = 0; r < d; ++r) ok &= bf16_to_f16(w.w_down + r * f, w2 + r * f_pad, f);
+  std::memcpy(img.data() + off(L.attn_norm), w.attn_norm, sizeof(float) * d);
+  std::memcpy(img.data() + off(L.ffn_norm), w.ffn_norm, sizeof(float) * d);
+  return ok;
+}
+
+mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
+                       const mzc_weights* weights, mzc_ctx* ctx) {
+  const mzc_model_shape& s = *shape;
+  ctx->shape = s;
+  ctx->opt = options ? *options : mzc_options{};
+  if (!options) ctx->opt.overlap = 1;
+  if (s.head_dim != 64 && s.head_dim != 128)
+    return ctx->fail(MZC_ERR_INVALID, "head_dim must be 64 or 128");
+  if (s.d_model % 64 != 0) return ctx->fail(MZC_ERR_INVALID, "d_model must be a multiple of 64");
+  if ((static_cast<int64_t>(s.n_q_heads) * s.head_dim) % 64 != 0)
+    return ctx->fail(MZC_ERR_INVALID, "n_q_heads*head_dim must be a multiple of 64");
+  mzc_status ss = ctx->st.init(s, ctx->opt.pool_blocks, ctx->opt.host_store_bytes);
+  if (ss != MZC_OK) return ctx->fail(ss, ctx->st.error());
+  if (!weights || !weights->embed || !weights->lm_head || !weights->final_norm || !weights->layers)
+    return ctx->fail(MZC_ERR_INVALID, "weights are incomplete");
+  CK(cudaSetDevice(ctx->opt.device));
+  CK(cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, ctx->opt.device));
+  const int64_t d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim;
+  const int64_t L = s.n_layers, V = s.vocab;
+  ctx->f_pad = align_up(s.ffn_dim, mzc::kSwigluGroup);
+  ctx->qkv_dim = (hq + 2 * hkv) * hd;
+  ctx->max_rows = ctx->opt.max_rows > 0 ? ctx->opt.max_rows : s.max_ctx;
+  ctx->nblk = ctx->st.nblk_max();
+  ctx->block_bytes = ctx->st.block_bytes();
+  const int64_t R = ctx->max_rows, F2 = 2 * ctx->f_pad;
+
+  CK(cudaStreamCreateWithFlags(&ctx->cs, cudaStreamNonBlocking));
+  CK(cudaStreamCreateWithFlags(&ctx->xs, cudaStreamNonBlocking));
+  ctx->ev_kv.assign(L, nullptr);
+  ctx->ev_w.assign(L, nullptr);
+  for (int64_t l = 0; l < L; ++l) {
+    CK(cudaEventCreateWithFlags(&ctx->ev_kv[l], cudaEventDisableTiming));
+    CK(cudaEventCreateWithFlags(&ctx->ev_w[l], cudaEventDisableTiming));
+  }
+  cudaEvent_t* timed[] = {&ctx->ev_t0, &ctx->ev_t1, &ctx->ev_c0, &ctx->ev_c1, &ctx->ev_l0, &ctx->ev_l1};
+  for (auto e : timed) CK(cudaEventCreate(e));
+
+  // ---- weights: one slot per layer ----
+  size_t o = 0;
+  const size_t sz_qkv = align_up(ctx->qkv_dim * d * 2, 1024), sz_o = align_up(d * hq * hd * 2, 1024);
+  const size_t sz_13 = align_up(F2 * d * 2, 1024), sz_2 = align_up(d * ctx->f_pad * 2, 1024);
+  const size_t sz_n = align_up(d * 4, 1024);
+  const size_t slot = sz_qkv + sz_o + sz_13 + sz_2 + 2 * sz_n;
+  CK(cudaMalloc(&ctx->d_weights, slot * L));
+  ctx->layers.assign(L, LayerDev{});
+  std::vector<uint8_t> img(slot);
+  for (int64_t l = 0; l < L; ++l) {
+    LayerDev& Ld = ctx->layers[l];
+    Ld.base = ctx->d_weights + slot * l;
+    Ld.bytes = slot;
+    o = 0;
+    Ld.wqkv = reinterpret_cast<uint16_t*>(Ld.base + o); o += sz_qkv;
+    Ld.wo = reinterpret_cast<uint16_t*>(Ld.base + o); o += sz_o;
+    Ld.w13 = reinterpret_cast<uint16_t*>(Ld.base + o); o += sz_13;
+    Ld.w2 = reinterpret_cast<uint16_t*>(Ld.base + o); o += sz_2;
+    Ld.attn_norm = reinterpret_cast<float*>(Ld.base + o); o += sz_n;
+    Ld.ffn_norm = reinterpret_cast<float*>(Ld.base + o); o += sz_n;
+    const mzc_layer_weights& w = weights->layers[l];
+    if (!w.wq || !w.wk || !w.wv || !w.wo || !w.w_gate || !w.w_up || !w.w_down || !w.attn_norm || !w.ffn_norm)
+      return ctx->fail(MZC_ERR_INVALID, "layer weights are incomplete");
+    if (!pack_layer(s, ctx->f_pad, w, img, Ld))
+      return ctx->fail(MZC_ERR_INVALID, "a projection weight is outside the fp16 range");
+    CK(cudaMemcpy(Ld.base, img.data(), slot, cudaMemcpyHostToDevice));
+  }
+  CK(cudaMalloc(&ctx->d_embed, V * d * 2));
+  CK(cudaMalloc(&ctx->d_lm, V * d * 2));
+  CK(cudaMalloc(&ctx->d_fnorm, d * 4));
+  CK(cudaMemcpy(ctx->d_embed, weights->embed, V * d * 2, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(ctx->d_lm, weights->lm_head, V * d * 2, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(ctx->d_fnorm, weights->final_norm, d * 4, cudaMemcpyHostToDevice));
+
+  // ---- KV pool (zeroed: never-written slots hold finite values) ----
+  const size_t pool_bytes = static_cast<size_t>(ctx->st.pool_blocks()) * ctx->block_bytes;
+  CK(cudaMalloc(&ctx->d_pool, pool_bytes));
+  CK(cudaMemset(ctx->d_pool, 0, pool_bytes));
+
+  // ---- rotary tables: angle(pos, i) = pos * theta^(-2i/hd) in double ----
+  {
+    const int64_t P = s.max_ctx, half = hd / 2;
+    std::vector<float> c(P * half), sn(P * half);
+    for (int64_t i = 0; i < half; ++i) {
+      const double inv = std::pow(static_cast<double>(s.rope_theta), -2.0 * static_cast<double>(i) / static_cast<double>(hd));
+      for (int64_t p = 0; p < P; ++p) {
+        const double a = static_cast<double>(p) * inv;
+        c[p * half + i] = static_cast<float>(std::cos(a));
+        sn[p * half + i] = static_cast<float>(std::sin(a));
+      }
+    }
+    CK(cudaMalloc(&ctx->d_cos, P * half * 4));
+    CK(cudaMalloc(&ctx->d_sin, P * half * 4));
+    CK(cudaMemcpy(ctx->d_cos, c.data(), P * half * 4, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(ctx->d_sin, sn.data(), P * half * 4, cudaMemcpyHostToDevice));
+  }
+
+  // ---- activations ----
+  CK(cudaMalloc(&ctx->d_x, R * d * 4));
+  CK(cudaMalloc(&ctx->d_h, R * d * 2));
+  CK(cudaMalloc(&ctx->d_qkv, R * ctx->qkv_dim * 2));
+  CK(cudaMalloc(&ctx->d_q, R * hq * hd * 2));
+  CK(cudaMalloc(&ctx->d_attn, R * hq * hd * 2));
+  CK(cudaMalloc(&ctx->d_act, R * ctx->f_pad * 2));
+  CK(cudaMemset(ctx->d_h, 0, R * d * 2));
+  CK(cudaMemset(ctx->d_attn, 0, R * hq * hd * 2));
+  CK(cudaMemset(ctx->d_act, 0, R * ctx->f_pad * 2));
+  // A operands: box 128 rows of 64 columns
+  bool ok = mzc::make_tmap_f16(&ctx->tm_h, ctx->d_h, R, d, 128) &&
+            mzc::make_tmap_f16(&ctx->tm_attn, ctx->d_attn, R, hq * hd, 128) &&
+            mzc::make_tmap_f16(&ctx->tm_act, ctx->d_act, R, ctx->f_pad, 128);
+  for (int64_t l = 0; l < L && ok; ++l) {
+    LayerDev& Ld = ctx->layers[l];
+    ok = mzc::make_gemm_weight(&Ld.tm_qkv, Ld.wqkv, ctx->qkv_dim, d) &&
+         mzc::make_gemm_weight(&Ld.tm_o, Ld.wo, d, hq * hd) &&
+         mzc::make_gemm_weight(&Ld.tm_13, Ld.w13, F2, d) &&
+         mzc::make_gemm_weight(&Ld.tm_2, Ld.w2, d, ctx->f_pad);
+  }
+  if (!ok) return ctx->fail(MZC_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+
+  // ---- per-call metadata, logits, scratch, status ----
+  ctx->meta_bytes = static_cast<size_t>(R) * 8 + static_cast<size_t>(L) * ctx->nblk * 4;
+  CK(cudaMalloc(&ctx->d_meta, ctx->meta_bytes));
+  CK(cudaHostAlloc(&ctx->h_meta, ctx->meta_bytes, cudaHostAllocDefault));
+  CK(cudaMalloc(&ctx->d_logits, V * 4));
+  CK(cudaHostAlloc(&ctx->h_logits, V * 4, cudaHostAllocDefault));
+  int64_t scratch = 0;
+  for (int64_t n = 1; n <= std::min<int64_t>(R, 8192); ++n) {
+    int sp = 1, per = 0;
+    mzc::attention_split(n, s.n_q_heads, s.n_kv_heads, s.max_ctx, ctx->num_sms, &sp, &per);
+    scratch = std::max(scratch, mzc::attention_scratch_bytes(n, s.n_q_heads, s.head_dim, sp));
+  }
+  ctx->scratch_bytes = scratch;
+  if (scratch > 0) CK(cudaMalloc(&ctx->d_scratch, scratch));
+  CK(cudaMalloc(&ctx->d_status, 4));
+  CK(cudaMemset(ctx->d_status, 0, 4));
+  CK(cudaMalloc(&ctx->d_staging, ctx->nblk * ctx->block_bytes));
+  CK(cudaMalloc(&ctx->d_list, L * ctx->nblk * 4));
+  CK(cudaHostAlloc(&ctx->h_list, L * ctx->nblk * 4, cudaHostAllocDefault));
+  CK(cudaHostAlloc(&ctx->h_staging, ctx->nblk * ctx->block_bytes, cudaHostAllocDefault));
+  CK(cudaDeviceSynchronize());
+  return MZC_OK;
+}
+
+// Moves `moves` (COPY eviction) out to the pinned store, then poisons the
+// freed physical blocks so that a missing wait shows up as NaN.
+mzc_status copy_out(mzc_ctx* ctx, const std::vector<mzc::EvictMove>& moves) {
+  int64_t total = 0;
+  for (auto& mv : moves) {
+    std::memcpy(ctx->h_list + total, mv.phys.data(), mv.phys.size() * 4);
+    total += static_cast<int64_t>(mv.phys.size());
+  }
+  if (total == 0) return MZC_OK;
+  CK(cudaMemcpyAsync(ctx->d_list, ctx->h_list, total * 4, cudaMemcpyHostToDevice, ctx->cs));
+  int64_t at = 0;
+  for (auto& mv : moves) {
+    const int64_t nb = static_cast<int64_t>(mv.phys.size());
+    CK(mzc::launch_gather_blocks(ctx->d_pool, ctx->d_list + at, nb, ctx->block_bytes, ctx->d_staging, ctx->cs));
+    CK(cudaMemcpyAsync(ctx->h_store + mv.host_off, ctx->d_staging, nb * ctx->block_bytes,
+                       cudaMemcpyDeviceToHost, ctx->cs));
+    at += nb;
+  }
+  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, total, ctx->block_bytes, ctx->cs));
+  CK(cudaStreamSynchronize(ctx->cs));
+  return MZC_OK;
+}
+
+mzc_status poison(mzc_ctx* ctx, const std::vector<int32_t>& phys) {
+  if (phys.empty()) return MZC_OK;
+  std::memcpy(ctx->h_list, phys.data(), phys.size() * 4);
+  CK(cudaMemcpyAsync(ctx->d_list, ctx->h_list, phys.size() * 4, cudaMemcpyHostToDevice, ctx->cs));
+  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, static_cast<int64_t>(phys.size()), ctx->block_bytes, ctx->cs));
+  CK(cudaStreamSynchronize(ctx->cs));
+  return MZC_OK;
+}
+
+mzc_status ensure_store(mzc_ctx* ctx) {
+  if (ctx->h_store) return MZC_OK;
+  CK(cudaHostAlloc(&ctx->h_store, ctx->st.host_store_bytes(), cudaHostAllocDefault));
+  return MZC_OK;
+}
+
+mzc_status check_status(mzc_ctx* ctx) {
+  int32_t s = 0;
+  CK(cudaMemcpy(&s, ctx->d_status, 4, cudaMemcpyDeviceToHost));
+  if (s != 0) {
+    CK(cudaMemset(ctx->d_status, 0, 4));
+    return ctx->fail(static_cast<mzc_status>(s), s == MZC_ERR_TIMEOUT
+                                                     ? "a device wait timed out"
+                                                     : "a device bounds check failed");
+  }
+  return MZC_OK;
+}
+
+cudaEvent_t next_event(mzc_ctx* ctx) {
+  if (ctx->ev_next == ctx->ev_pool.size()) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    ctx->ev_pool.push_back(e);
+  }
+  return ctx->ev_pool[ctx->ev_next++];
+}
+
+// Launches one kernel of class `cls` (n_kernels launches, algorithmic work
+// flops / bytes), bracketed by CUDA events on the compute stream when kernel
+// timing is on.
+template <class F>
+cudaError_t klaunch(mzc_ctx* ctx, int cls, double flops, double bytes, int n_kernels, F&& fn) {
+  mzc_kernel_stat& k = ctx->kstat[cls];
+  k.launches += n_kernels;
+  k.flops += flops;
+  k.bytes += bytes;
+  if (!ctx->ktime) return fn();
+  cudaEvent_t a = next_event(ctx), b = next_event(ctx);
+  if (!a || !b) return cudaErrorMemoryAllocation;
+  cudaError_t e = cudaEventRecord(a, ctx->cs);
+  if (e != cudaSuccess) return e;
+  e = fn();
+  if (e != cudaSuccess) return e;
+  e = cudaEventRecord(b, ctx->cs);
+  ctx->kev.push_back(mzc_ctx::KEv{cls, a, b, flops, bytes});
+  return e;
+}
+
+mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* logits_out) {
+  const mzc_model_shape& s = ctx->shape;
+  const int64_t d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim, L = s.n_layers;
+  for (int64_t i = 0; i < n; ++i)
+    if (tokens[i] < 0 || tokens[i] >= s.vocab) return ctx->fail(MZC_ERR_INVALID, "token id outside the vocabulary");
+  mzc::PrefillPlan P;
+  mzc_status ss = ctx->st.prepare_prefill(n, ctx->max_rows, &P);
+  if (ss != MZC_OK) return ctx->from_state(ss);
+  const int64_t nrec = P.rec_end - P.rec_begin, rows = nrec + n;
+  if (rows == 0) {
+    ctx->st.complete(0);
+    return MZC_OK;
+  }
+  // metadata: tokens | positions | block tables
+  int32_t* htok = reinterpret_cast<int32_t*>(ctx->h_meta);
+  int32_t* hpos = htok + rows;
+  int32_t* htab = hpos + rows;
+  for (int64_t i = 0; i < nrec; ++i) {
+    htok[i] = ctx->tokens[P.rec_begin + i];
+    hpos[i] = static_cast<int32_t>(P.rec_begin + i);
+  }
+  for (int64_t i = 0; i < n; ++i) {
+    htok[nrec + i] = tokens[i];
+    hpos[nrec + i] = static_cast<int32_t>(P.prompt_begin + i);
+  }
+  std::vector<int32_t> tab;
+  ctx->st.block_table(&tab);
+  std::memcpy(htab, tab.data(), tab.size() * 4);
+  const size_t mbytes = static_cast<size_t>(rows) * 8 + tab.size() * 4;
+  int32_t* dtok = reinterpret_cast<int32_t*>(ctx->d_meta);
+  int32_t* dpos = dtok + rows;
+  int32_t* dtab = dpos + rows;
+  cudaStream_t cs = ctx->cs;
+  auto bail = [&](mzc_status e) {
+    cudaStreamSynchronize(cs);
+    ctx->st.abort_prefill(P);
+    return e;
+  };
+#define CKP(call)                                                                             \
+  do {                                                                                        \
+    cudaError_t e_ = (call);                                                                  \
+    if (e_ != cudaSuccess)                                                                    \
+      return bail(ctx->fail(MZC_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_))); \
+  } while (0)
+  CKP(cudaEventRecord(ctx->ev_t0, cs));
+  ctx->ttft_from_copy = ctx->restore_issued;
+  CKP(cudaMemcpyAsync(ctx->d_meta, ctx->h_meta, mbytes, cudaMemcpyHostToDevice, cs));
+  if (!ctx->opt.overlap && ctx->restore_issued) CKP(cudaStreamWaitEvent(cs, ctx->ev_c1, 0));
+  ctx->ev_next = 0;
+  ctx->kev.clear();
+  const double kvb = s.kv_dtype == MZC_KV_FP16 ? 2.0 : 2.0;  // bytes per stored K/V element
+  // algorithmic attention work of rows [r0, r0 + nr)
+  auto attn_work = [&](int64_t r0, int64_t nr, double* fl, double* by) {
+    double pairs = 0.0;
+    int64_t mx = 0;
+    for (int64_t i = r0; i < r0 + nr; ++i) {
+      pairs += static_cast<double>(hpos[i]) + 1.0;
+      mx = std::max<int64_t>(mx, hpos[i] + 1);
+    }
+    *fl = 4.0 * hd * hq * pairs;
+    *by = 2.0 * hkv * hd * kvb * mx + 2.0 * nr * hq * hd * 2.0;
+  };
+  const double dd = static_cast<double>(d), R = static_cast<double>(rows);
+  CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
+    return mzc::launch_embed(dtok, rows, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
+  }));
+  const int64_t max_keys = n > 0 ? P.prompt_end : P.rec_end;
+  auto gemm = [&](const CUtensorMap& ta, const mzc::GemmWeight& w, void* out, int64_t N, int64_t K, int epi) {
+    const double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
+    return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
+                   [&] { return mzc::launch_gemm(ta, w, out, rows, N, K, epi, ctx->d_status, cs); });
+  };
+  auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab) {
+    double fl, by;
+    attn_work(r0, nr, &fl, &by);
+    int sp = 1, per = 0;
+    mzc::attention_split(nr, s.n_q_heads, s.n_kv_heads, mk, ctx->num_sms, &sp, &per);
+    const bool fits = sp == 1 || ctx->scratch_bytes >= mzc::attention_scratch_bytes(nr, s.n_q_heads, s.head_dim, sp);
+    return klaunch(ctx, MZC_K_ATTENTION, fl, by, (sp > 1 && fits) ? 2 : 1, [&] {
+      return mzc::launch_attention(ctx->d_q + r0 * hq * hd, dpos + r0, nr, s.n_q_heads, s.n_kv_heads,
+                                   s.head_dim, ltab, ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(),
+                                   s.kv_dtype, ctx->d_attn + r0 * hq * hd, ctx->d_scratch,
+                                   ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs);
+    });
+  };
+  const double norm_bytes = R * dd * 6.0 + dd * 4.0;
+  const double rope_bytes = R * (hq + 2.0 * hkv) * hd * 4.0 + R * hd * 4.0;
+  for (int64_t l = 0; l < L; ++l) {
+    const LayerDev& W = ctx->layers[l];
+    const int32_t* ltab = dtab + l * ctx->nblk;
+    if (P.w_wait[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_w[l], 0));
+    CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+      return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, rows, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+    }));
+    CKP(gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
+    if (P.kv_wait_write[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+    CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
+      return mzc::launch_rope_kv_write(ctx->d_qkv, dpos, rows, s.n_q_heads, s.n_kv_heads, s.head_dim,
+                                       ctx->d_cos, ctx->d_sin, ltab, ctx->nblk, ctx->d_pool,
+                                       ctx->st.pool_blocks(), s.kv_dtype, ctx->d_q, ctx->d_status, cs);
+    }));
+    const bool split_launch = nrec > 0 && n > 0 && P.kv_wait_prompt[l] && !P.kv_wait_rec[l];
+    if (split_launch) {
+      // recompute rows read only resident keys: they run before the copy lands
+      CKP(attention(0, nrec, P.rec_end, ltab));
+      CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+      CKP(attention(nrec, n, max_keys, ltab));
+    } else {
+      if (P.kv_wait_prompt[l] || P.kv_wait_rec[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+      CKP(attention(0, rows, max_keys, ltab));
+    }
+    CKP(gemm(ctx->tm_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
+    CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+      return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, rows, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+    }));
+    CKP(gemm(ctx->tm_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
+    CKP(gemm(ctx->tm_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
+  }
+  ctx->lm_timed = false;
+  if (n > 0 && logits_out) {
+    CKP(cudaEventRecord(ctx->ev_l0, cs));
+    CKP(klaunch(ctx, MZC_K_LM_HEAD, 2.0 * s.vocab * dd, s.vocab * dd * 2.0 + s.vocab * 4.0 + dd * 8.0, 1, [&] {
+      return mzc::launch_lm_head(ctx->d_x + (rows - 1) * d, ctx->d_fnorm, static_cast<int32_t>(d), s.rms_eps,
+                                 ctx->d_lm, s.vocab, ctx->d_logits, ctx->num_sms, cs);
+    }));
+    CKP(cudaEventRecord(ctx->ev_l1, cs));
+    CKP(cudaMemcpyAsync(ctx->h_logits, ctx->d_logits, static_cast<size_t>(s.vocab) * 4, cudaMemcpyDeviceToHost, cs));
+    ctx->lm_timed = true;
+  }
+  CKP(cudaEventRecord(ctx->ev_t1, cs));
+  CKP(cudaStreamSynchronize(cs));
+  if (ctx->restore_issued) CKP(cudaStreamSynchronize(ctx->xs));
+#undef CKP
+  for (const auto& ke : ctx->kev) {
+    float ms = 0.0f;
+    if (cudaEventElapsedTime(&ms, ke.a, ke.b) == cudaSuccess) ctx->kstat[ke.cls].ms += ms;
+  }
+  ctx->kev.clear();
+  mzc_status st = check_status(ctx);
+  if (st != MZC_OK) {
+    ctx->st.abort_prefill(P);
+    return st;
+  }
+  if (n > 0 && logits_out) std::memcpy(logits_out, ctx->h_logits, static_cast<size_t>(s.vocab) * 4);
+  ctx->st.complete(n);
+  ctx->tokens.insert(ctx->tokens.end(), tokens, tokens + n);
+  ctx->last.rows_last = rows;
+  ctx->last.recompute_rows_last = nrec;
+  ctx->restore_issued = false;
+  return MZC_OK;
+}
+
+// Linear per-unit cost model of the two restore paths (Sec. 4.3: per-unit
+// times, total time linear in the number of units).
+struct CostModel {
+  mzc_model_shape s;
+  mzc_profile p;
+  double layer_weight_bytes, linear_flops_row, attn_flops_pair;
+  CostModel(const mzc_model_shape& s_, const mzc_profile& p_) : s(s_), p(p_) {
+    const double d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim, f = s.ffn_dim;
+    const double params = d * (hq + 2 * hkv) * hd + hq * hd * d + 3.0 * d * f;
+    layer_weight_bytes = 2.0 * params;
+    linear_flops_row = 2.0 * params;
+    attn_flops_pair = 4.0 * hd * hq;
+  }
+  double copy_s(int64_t tokens) const {
+    const double blocks = static_cast<double>(ceil_div(tokens, 16));
+    const double bytes = blocks * s.n_layers * 2.0 * s.n_kv_heads * 16 * s.head_dim * 2;
+    return bytes / (p.h2d_gbs * 1e9);
+  }
+  double compute_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
+    const double rows = static_cast<double>(s1 - p0 + n_prompt);
+    if (rows <= 0) return 0.0;
+    const double gemm = std::max(rows * linear_flops_row / (p.gemm_tflops * 1e12),
+                                 layer_weight_bytes / (p.hbm_gbs * 1e9));
+    // sum of (pos + 1) over recompute rows [p0, s1) and prompt rows [n_ctx, n_ctx + n_prompt)
+    auto tri = [](double a, double b) { return (b * (b + 1) - a * (a + 1)) / 2.0; };
+    const double pairs = tri(static_cast<double>(p0), static_cast<double>(s1)) +
+                         tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
+    const double attn = pairs * attn_flops_pair / (p.attn_tflops * 1e12);
+    return s.n_layers * (gemm + attn + p.launch_us * 1e-6);
+  }
+};
+
+}  // namespace
+
+extern "C" {
+
+mzc_status mzc_create(const mzc_model_shape* shape, const mzc_options* options,
+                      const mzc_weights* weights, mzc_ctx** out) {
+  if (!out) return MZC_ERR_INVALID;
+  *out = nullptr;
+  if (!shape) {
+    g_create_error = "shape is NULL";
+    return MZC_ERR_INVALID;
+  }
+  mzc_ctx* ctx = new mzc_ctx();
+  mzc_status s = create_impl(shape, options, weights, ctx);
+  if (s != MZC_OK) {
+    g_create_error = ctx->err;
+    destroy_impl(ctx);
+    return s;
+  }
+  *out = ctx;
+  return MZC_OK;
+}
+
+mzc_status mzc_destroy(mzc_ctx* ctx) { return destroy_impl(ctx); }
+
+mzc_status mzc_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* logits_out) {
+  if (!ctx) return MZC_ERR_INVALID;
+  if (n < 0 || (n > 0 && !tokens)) return ctx->fail(MZC_ERR_INVALID, "bad token buffer");
+  CK(cudaSetDevice(ctx->opt.device));
+  return run_prefill(ctx, tokens, n, logits_out);
+}
+
+mzc_status mzc_evict(mzc_ctx* ctx, int32_t l0, int32_t l1, int64_t t0, int64_t t1, int32_t mode) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  if (mode == MZC_AUTO) {
+    if (l0 != 0 || l1 != ctx->shape.n_layers)
+      return ctx->fail(MZC_ERR_INVALID, "AUTO eviction covers every layer");
+    const int64_t n_ctx = ctx->st.n_ctx();
+    if (t0 < 0 || t0 >= n_ctx) return ctx->fail(MZC_ERR_RANGE, "token range outside the context");
+    const int64_t p = t0 / 16 * 16;
+    int64_t split = n_ctx;
+    if (ctx->policy == MZC_POLICY_COPY) split = p;
+    else if (ctx->policy == MZC_POLICY_HYBRID) {
+      mzc_status e = mzc_plan_split(&ctx->shape, &ctx->prof, p, n_ctx, 0, &split);
+      if (e != MZC_OK) return ctx->fail(e, "hybrid split failed");
+    }
+    if (split > p) {
+      mzc_status e = mzc_evict(ctx, 0, l1, p, split, MZC_DROP);
+      if (e != MZC_OK) return e;
+    }
+    if (split < n_ctx) return mzc_evict(ctx, 0, l1, split, n_ctx, MZC_COPY);
+    return MZC_OK;
+  }
+  std::vector<int32_t> freed;
+  if (mode == MZC_DROP && t0 >= 0 && t1 <= ctx->st.n_ctx() && t0 < t1 && l0 >= 0 && l1 <= ctx->shape.n_layers) {
+    for (int32_t l = l0; l < l1; ++l)
+      for (int64_t b = t0 / 16; b < ceil_div(t1, 16); ++b)
+        if (ctx->st.at(l, b).phys >= 0) freed.push_back(ctx->st.at(l, b).phys);
+  }
+  if (mode == MZC_COPY) {
+    mzc_status e = ensure_store(ctx);
+    if (e != MZC_OK) return e;
+  }
+  std::vector<mzc::EvictMove> moves;
+  mzc_status s = ctx->st.evict_range(l0, l1, t0, t1, mode, &moves);
+  if (s != MZC_OK) return ctx->from_state(s);
+  if (mode == MZC_COPY) return copy_out(ctx, moves);
+  return poison(ctx, freed);
+}
+
+mzc_status mzc_evict_blocks(mzc_ctx* ctx, const int32_t* layer, const int64_t* blk, int64_t n, int32_t mode) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  if (mode == MZC_COPY) {
+    mzc_status e = ensure_store(ctx);
+    if (e != MZC_OK) return e;
+  }
+  std::vector<mzc::EvictMove> moves;
+  mzc_status s = ctx->st.evict_blocks(layer, blk, n, mode, &moves);
+  if (s != MZC_OK) return ctx->from_state(s);
+  return copy_out(ctx, moves);
+}
+
+mzc_status mzc_evict_weights(mzc_ctx* ctx, int32_t l0, int32_t l1) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  mzc_status s = ctx->st.evict_weights(l0, l1);
+  if (s != MZC_OK) return ctx->from_state(s);
+  for (int32_t l = l0; l < l1; ++l) {
+    LayerDev& Ld = ctx->layers[l];
+    if (!Ld.host_master) CK(cudaHostAlloc(&Ld.host_master, Ld.bytes, cudaHostAllocDefault));
+    CK(cudaMemcpyAsync(Ld.host_master, Ld.base, Ld.bytes, cudaMemcpyDeviceToHost, ctx->cs));
+    CK(cudaMemsetAsync(Ld.base, 0xFF, Ld.bytes, ctx->cs));  // NaN until restored
+  }
+  CK(cudaStreamSynchronize(ctx->cs));
+  return MZC_OK;
+}
+
+mzc_status mzc_restore_async(mzc_ctx* ctx) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  std::vector<mzc_copy_run> runs;
+  std::vector<int32_t> wl;
+  mzc_status s = ctx->st.plan_restore(&runs, &wl);
+  if (s != MZC_OK) return ctx->from_state(s);
+  if (!ctx->st.restore_in_flight()) return MZC_OK;
+  cudaStream_t xs = ctx->xs;
+  CK(cudaEventRecord(ctx->ev_c0, xs));
+  size_t ri = 0, wi = 0;
+  int64_t bytes = 0, copies = 0;
+  for (int32_t l = 0; l < ctx->shape.n_layers; ++l) {
+    if (wi < wl.size() && wl[wi] == l) {
+      const LayerDev& Ld = ctx->layers[l];
+      CK(cudaMemcpyAsync(Ld.base, Ld.host_master, Ld.bytes, cudaMemcpyHostToDevice, xs));
+      bytes += static_cast<int64_t>(Ld.bytes);
+      ++copies;
+      ++wi;
+    }
+    CK(cudaEventRecord(ctx->ev_w[l], xs));
+    while (ri < runs.size() && runs[ri].layer == l) {
+      const mzc_copy_run& r = runs[ri++];
+      const int64_t nb = static_cast<int64_t>(r.n_blocks) * ctx->block_bytes;
+      CK(cudaMemcpyAsync(ctx->d_pool + r.phys_begin * ctx->block_bytes, ctx->h_store + r.host_off,
+                         nb, cudaMemcpyHostToDevice, xs));
+      bytes += nb;
+      ++copies;
+    }
+    CK(cudaEventRecord(ctx->ev_kv[l], xs));
+  }
+  CK(cudaEventRecord(ctx->ev_c1, xs));
+  ctx->restore_issued = true;
+  ctx->last.bytes_h2d_last = bytes;
+  ctx->last.copies_last = copies;
+  return MZC_OK;
+}
+
+mzc_status mzc_recompute_tail(mzc_ctx* ctx, int64_t p, int64_t n) {
+  if (!ctx) return MZC_ERR_INVALID;
+  return ctx->from_state(ctx->st.recompute_tail(p, n));
+}
+
+mzc_status mzc_set_policy(mzc_ctx* ctx, int32_t policy, const mzc_profile* profile) {
+  if (!ctx) return MZC_ERR_INVALID;
+  if (policy < MZC_POLICY_COPY || policy > MZC_POLICY_HYBRID)
+    return ctx->fail(MZC_ERR_INVALID, "unknown policy");
+  ctx->policy = policy;
+  if (profile) ctx->prof = *profile;
+  return MZC_OK;
+}
+
+mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profile, int64_t p,
+                          int64_t n_ctx, int64_t n_prompt, int64_t* s_out) {
+  if (!shape || !s_out || p < 0 || n_ctx < p || n_prompt < 0) return MZC_ERR_INVALID;
+  const mzc_profile prof = profile ? *profile : default_profile();
+  if (prof.h2d_gbs <= 0 || prof.hbm_gbs <= 0 || prof.gemm_tflops <= 0 || prof.attn_tflops <= 0)
+    return MZC_ERR_INVALID;
+  CostModel cm(*shape, prof);
+  int64_t best = p;
+  double best_t = INFINITY;
+  // candidates: block boundaries from p, and n_ctx itself
+  for (int64_t s = p;; s += 16) {
+    const int64_t sc = std::min(s, n_ctx);
+    const double t = std::max(cm.compute_s(p, sc, n_ctx, n_prompt), cm.copy_s(n_ctx - sc));
+    if (t < best_t) {
+      best_t = t;
+      best = sc;
+    }
+    if (sc >= n_ctx) break;
+  }
+  *s_out = best;
+  return MZC_OK;
+}
+
+mzc_status mzc_truncate(mzc_ctx* ctx, int64_t n_ctx) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  std::vector<int32_t> freed;
+  if (n_ctx >= 0 && n_ctx <= ctx->st.n_ctx())
+    for (int32_t l = 0; l < ctx->shape.n_layers; ++l)
+      for (int64_t b = ceil_div(n_ctx, 16); b < ceil_div(ctx->st.n_ctx(), 16); ++b)
+        if (ctx->st.at(l, b).st == MZC_RESIDENT && ctx->st.at(l, b).phys >= 0)
+          freed.push_back(ctx->st.at(l, b).phys);
+  mzc_status s = ctx->st.truncate(n_ctx);
+  if (s != MZC_OK) return ctx->from_state(s);
+  ctx->tokens.resize(static_cast<size_t>(n_ctx));
+  return poison(ctx, freed);
+}
+
+mzc_status mzc_sync(mzc_ctx* ctx) {
+  if (!ctx) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  if (ctx->st.recompute_pending()) return run_prefill(ctx, nullptr, 0, nullptr);
+  CK(cudaStreamSynchronize(ctx->cs));
+  CK(cudaStreamSynchronize(ctx->xs));
+  mzc_status s = check_status(ctx);
+  if (s != MZC_OK) return s;
+  if (ctx->st.restore_in_flight()) {
+    ctx->st.complete(0);
+    ctx->restore_issued = false;
+  }
+  return MZC_OK;
+}
+
+mzc_status mzc_query(mzc_ctx* ctx, int32_t layer, int64_t b, int32_t* state, int32_t* phys) {
+  if (!ctx) return MZC_ERR_INVALID;
+  if (layer < 0 || layer >= ctx->shape.n_layers || b < 0 || b >= ctx->nblk)
+    return ctx->fail(MZC_ERR_RANGE, "index out of range");
+  const mzc::BlockEntry& e = ctx->st.at(layer, b);
+  if (state) *state = e.st;
+  if (phys) *phys = e.phys;
+  return MZC_OK;
+}
+
+mzc_status mzc_read_kv(mzc_ctx* ctx, int32_t layer, int64_t b, void* k_host, void* v_host) {
+  if (!ctx || !k_host || !v_host) return MZC_ERR_INVALID;
+  if (layer < 0 || layer >= ctx->shape.n_layers || b < 0 || b >= ceil_div(ctx->st.n_ctx(), 16))
+    return ctx->fail(MZC_ERR_RANGE, "block outside the context");
+  const mzc::BlockEntry& e = ctx->st.at(layer, b);
+  if (e.st != MZC_RESIDENT) return ctx->fail(MZC_ERR_STATE, "block is not resident");
+  CK(cudaSetDevice(ctx->opt.device));
+  const int64_t half = ctx->block_bytes / 2;
+  const uint8_t* src = ctx->d_pool + static_cast<int64_t>(e.phys) * ctx->block_bytes;
+  CK(cudaMemcpy(k_host, src, half, cudaMemcpyDeviceToHost));
+  CK(cudaMemcpy(v_host, src + half, half, cudaMemcpyDeviceToHost));
+  return MZC_OK;
+}
+
+mzc_status mzc_read_kv_all(mzc_ctx* ctx, int64_t n, float* k_host, float* v_host) {
+  if (!ctx || !k_host || !v_host) return MZC_ERR_INVALID;
+  if (n < 0 || n > ctx->st.n_ctx()) return ctx->fail(MZC_ERR_RANGE, "n beyond the context");
+  CK(cudaSetDevice(ctx->opt.device));
+  const mzc_model_shape& s = ctx->shape;
+  const int64_t hkv = s.n_kv_heads, hd = s.head_dim, nb = ceil_div(n, 16);
+  for (int32_t l = 0; l < s.n_layers; ++l) {
+    for (int64_t b = 0; b < nb; ++b) {
+      const mzc::BlockEntry& e = ctx->st.at(l, b);
+      if (e.st != MZC_RESIDENT) return ctx->fail(MZC_ERR_STATE, "block is not resident");
+      ctx->h_list[b] = e.phys;
+    }
+    if (nb == 0) continue;
+    CK(cudaMemcpyAsync(ctx->d_list, ctx->h_list, nb * 4, cudaMemcpyHostToDevice, ctx->cs));
+    CK(mzc::launch_gather_blocks(ctx->d_pool, ctx->d_list, nb, ctx->block_bytes, ctx->d_staging, ctx->cs));
+    CK(cudaMemcpyAsync(ctx->h_staging, ctx->d_staging, nb * ctx->block_bytes, cudaMemcpyDeviceToHost, ctx->cs));
+    CK(cudaStreamSynchronize(ctx->cs));
+    const uint16_t* blocks = reinterpret_cast<const uint16_t*>(ctx->h_staging);
+    for (int64_t p = 0; p < n; ++p) {
+      const int64_t b = p / 16, slot = p % 16;
+      for (int64_t h = 0; h < hkv; ++h) {
+        const uint16_t* kb = blocks + b * 2 * hkv * 16 * hd + (h * 16 + slot) * hd;
+        const uint16_t* vb = kb + hkv * 16 * hd;
+        float* ko = k_host + ((static_cast<int64_t>(l) * n + p) * hkv + h) * hd;
+        float* vo = v_host + ((static_cast<int64_t>(l) * n + p) * hkv + h) * hd;
+        for (int64_t c = 0; c < hd; ++c) {
+          if (s.kv_dtype == MZC_KV_FP16) {
+            __half_raw rk, rv;
+            rk.x = kb[c];
+            rv.x = vb[c];
+            ko[c] = __half2float(__half(rk));
+            vo[c] = __half2float(__half(rv));
+          } else {
+            uint32_t uk = static_cast<uint32_t>(kb[c]) << 16, uv = static_cast<uint32_t>(vb[c]) << 16;
+            std::memcpy(&ko[c], &uk, 4);
+            std::memcpy(&vo[c], &uv, 4);
+          }
+        }
+      }
+    }
+  }
+  return MZC_OK;
+}
+
+mzc_status mzc_stats(mzc_ctx* ctx, mzc_stats_t* out) {
+  if (!ctx || !out) return MZC_ERR_INVALID;
+  ctx->st.counts(out);
+  out->bytes_h2d_last = ctx->last.bytes_h2d_last;
+  out->copies_last = ctx->last.copies_last;
+  out->rows_last = ctx->last.rows_last;
+  out->recompute_rows_last = ctx->last.recompute_rows_last;
+  return MZC_OK;
+}
+
+mzc_status mzc_last_times(mzc_ctx* ctx, float* ms3) {  // ms3 holds 4 floats
+  if (!ctx || !ms3) return MZC_ERR_INVALID;
+  ms3[0] = ms3[1] = ms3[2] = ms3[3] = 0.0f;
+  if (cudaEventElapsedTime(&ms3[0], ctx->ev_t0, ctx->ev_t1) != cudaSuccess) ms3[0] = -1.0f;
+  if (!ctx->ttft_from_copy || cudaEventElapsedTime(&ms3[1], ctx->ev_c0, ctx->ev_c1) != cudaSuccess) ms3[1] = -1.0f;
+  if (!ctx->lm_timed || cudaEventElapsedTime(&ms3[2], ctx->ev_l0, ctx->ev_l1) != cudaSuccess) ms3[2] = -1.0f;
+  if (cudaEventElapsedTime(&ms3[3], ctx->ttft_from_copy ? ctx->ev_c0 : ctx->ev_t0, ctx->ev_t1) != cudaSuccess)
+    ms3[3] = -1.0f;
+  cudaGetLastError();
+  return MZC_OK;
+}
+
+mzc_status mzc_set_kernel_timing(mzc_ctx* ctx, int32_t on) {
+  if (!ctx) return MZC_ERR_INVALID;
+  ctx->ktime = on != 0;
+  for (auto& k : ctx->kstat) k = mzc_kernel_stat{};
+  return MZC_OK;
+}
+
+mzc_status mzc_kernel_stats(mzc_ctx* ctx, int32_t cls, mzc_kernel_stat* out) {
+  if (!ctx || !out || cls < 0 || cls >= MZC_K_NCLASS) return MZC_ERR_INVALID;
+  *out = ctx->kstat[cls];
+  return MZC_OK;
+}
+
+const char* mzc_last_error(mzc_ctx* ctx) {
+  if (!ctx) return g_create_error.c_str();
+  return ctx->err.c_str();
+}
+
+mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
+  if (!ctx || !out) return MZC_ERR_INVALID;
+  CK(cudaSetDevice(ctx->opt.device));
+  mzc_profile p = ctx->prof;
+  cudaEvent_t a, b;
+  CK(cudaEventCreate(&a));
+  CK(cudaEventCreate(&b));
+  float ms = 0.0f;
+  // host link: 256 MiB (or the store) pinned -> device, on the copy stream
+  {
+    const int64_t bytes = std::min<int64_t>(256LL << 20, ctx->st.pool_blocks() * ctx->block_bytes);
+    uint8_t* h = nullptr;
+    CK(cudaHostAlloc(&h, bytes, cudaHostAllocDefault));
+    std::memset(h, 1, bytes);
+    CK(cudaMemcpyAsync(ctx->d_pool, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
+    CK(cudaEventRecord(a, ctx->xs));
+    for (int i = 0; i < 4; ++i) CK(cudaMemcpyAsync(ctx->d_pool, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
+    CK(cudaEventRecord(b, ctx->xs));
+    CK(cudaEventSynchronize(b));
+    CK(cudaEventElapsedTime(&ms, a, b));
+    p.h2d_gbs = 4.0 * bytes / (ms * 1e-3) / 1e9;
+    CK(cudaFreeHost(h));
+    CK(cudaMemset(ctx->d_pool, 0, bytes));
+  }
+  // HBM: device-to-device copy of the activation buffers
+  {
+    const int64_t bytes = ctx->max_rows * ctx->shape.d_model * 2;
+    CK(cudaMemcpyAsync(ctx->d_attn, ctx->d_h, bytes, cudaMemcpyDeviceToDevice, ctx->cs));
+    CK(cudaEventRecord(a, ctx->cs));
+    for (int i = 0; i < 10; ++i) CK(cudaMemcpyAsync(ctx->d_attn, ctx->d_h, bytes, cudaMemcpyDeviceToDevice, ctx->cs));
+    CK(cudaEventRecord(b, ctx->cs));
+    CK(cudaEventSynchronize(b));
+    CK(cudaEventElapsedTime(&ms, a, b));
+    if (ms > 0) p.hbm_gbs = 10.0 * 2.0 * bytes / (ms * 1e-3) / 1e9;
+  }
+  // GEMM: layer 0's projections at recompute sizes on scratch activations
+  {
+    const int64_t m = std::min<int64_t>(ctx->max_rows, 4096), d = ctx->shape.d_model;
+    const LayerDev& W = ctx->layers[0];
+    auto run = [&]() -> cudaError_t {
+      cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, ctx->d_status, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, ctx->d_status, ctx->cs);
+      return e;
+    };
+    CK(run());
+    CK(cudaEventRecord(a, ctx->cs));
+    for (int i = 0; i < 5; ++i) CK(run());
+    CK(cudaEventRecord(b, ctx->cs));
+    CK(cudaEventSynchronize(b));
+    CK(cudaEventElapsedTime(&ms, a, b));
+    const double flops = 5.0 * 2.0 * m * d * (ctx->qkv_dim + 2 * ctx->f_pad);
+    if (ms > 0) p.gemm_tflops = flops / (ms * 1e-3) / 1e12;
+  }
+  // attention over the resident context, when there is one
+  {
+    const int64_t n_ctx = ctx->st.n_ctx();
+    bool resident = n_ctx >= 1024;
+    for (int32_t l = 0; l < ctx->shape.n_layers && resident; ++l)
+      for (int64_t blk = 0; blk < ceil_div(n_ctx, 16) && resident; ++blk)
+        resident = ctx->st.at(l, blk).st == MZC_RESIDENT;
+    if (resident) {
+      const int64_t rows = std::min<int64_t>(ctx->max_rows, 1024);
+      int32_t* hp = reinterpret_cast<int32_t*>(ctx->h_meta);
+      for (int64_t i = 0; i < rows; ++i) hp[i] = static_cast<int32_t>(n_ctx - rows + i);
+      std::vector<int32_t> tab;
+      ctx->st.block_table(&tab);
+      std::memcpy(hp + rows, tab.data(), ctx->nblk * 4);
+      int32_t* dp = reinterpret_cast<int32_t*>(ctx->d_meta);
+      CK(cudaMemcpyAsync(dp, hp, (rows + ctx->nblk) * 4, cudaMemcpyHostToDevice, ctx->cs));
+      const mzc_model_shape& s = ctx->shape;
+      auto run = [&]() {
+        return mzc::launch_attention(ctx->d_q, dp, rows, s.n_q_heads, s.n_kv_heads, s.head_dim, dp + rows,
+                                     ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(), s.kv_dtype,
+                                     ctx->d_attn, ctx->d_scratch, ctx->scratch_bytes, n_ctx,
+                                     ctx->num_sms, ctx->d_status, ctx->cs);
+      };
+      CK(run());
+      CK(cudaEventRecord(a, ctx->cs));
+      for (int i = 0; i < 3; ++i) CK(run());
+      CK(cudaEventRecord(b, ctx->cs));
+      CK(cudaEventSynchronize(b));
+      CK(cudaEventElapsedTime(&ms, a, b));
+      double pairs = 0;
+      for (int64_t i = 0; i < rows; ++i) pairs += static_cast<double>(n_ctx - rows + i + 1);
+      const double flops = 3.0 * pairs * 4.0 * s.head_dim * s.n_q_heads;
+      if (ms > 0) p.attn_tflops = flops / (ms * 1e-3) / 1e12;
+    }
+  }
+  // per-layer launch cost: the 8 launches of one layer at one row
+  {
+    auto run = [&]() -> cudaError_t {
+      cudaError_t e = cudaSuccess;
+      for (int i = 0; i < 8 && e == cudaSuccess; ++i)
+        e = mzc::launch_rmsnorm(ctx->d_x, ctx->layers[0].attn_norm, 1, ctx->shape.d_model, 1e-5f, ctx->d_h, ctx->cs);
+      return e;
+    };
+    CK(run());
+    CK(cudaEventRecord(a, ctx->cs));
+    for (int i = 0; i < 20; ++i) CK(run());
+    CK(cudaEventRecord(b, ctx->cs));
+    CK(cudaEventSynchronize(b));
+    CK(cudaEventElapsedTime(&ms, a, b));
+    p.launch_us = ms * 1e3 / 20.0;
+  }
+  CK(cudaEventDestroy(a));
+  CK(cudaEventDestroy(b));
+  mzc_status s = check_status(ctx);
+  if (s != MZC_OK) return s;
+  ctx->prof = p;
+  *out = p;
+  return MZC_OK;
+}
+
+// ---- single kernels ---------------------------------------------------------
+
+static int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+#define KCK(expr) return (expr) == cudaSuccess ? MZC_OK : MZC_ERR_CUDA
+
+mzc_status mzc_k_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
+                         uint16_t* y, void* stream) {
+  if (!x || !g || !y || d % 8 != 0 || n < 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_rmsnorm(x, g, n, d, eps, y, static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_gemm(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
+                      int64_t k, int32_t epilogue, void* stream) {
+  if (!a || !w || !out || m < 0 || n <= 0 || k <= 0 || k % 8 != 0 || n % 16 != 0)
+    return MZC_ERR_INVALID;
+  if (epilogue < 0 || epilogue > 2) return MZC_ERR_INVALID;
+  if (epilogue == mzc::EPI_SWIGLU_BF16 && n % (2 * mzc::kSwigluGroup) != 0) return MZC_ERR_INVALID;
+  if (m == 0) return MZC_OK;
+  CUtensorMap ta;
+  mzc::GemmWeight tw;
+  if (!mzc::make_tmap_f16(&ta, a, static_cast<uint64_t>(m), static_cast<uint64_t>(k), 128) ||
+      !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
+    return MZC_ERR_CUDA;
+  KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, nullptr, static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_swiglu_pack(const uint16_t* gate, const uint16_t* up, int64_t f, int64_t d,
+                             uint16_t* out_host) {
+  if (!gate || !up || !out_host || f <= 0 || d <= 0 || f % mzc::kSwigluGroup != 0) return MZC_ERR_INVALID;
+  const int64_t G = mzc::kSwigluGroup;
+  for (int64_t j = 0; j < f; ++j) {
+    const int64_t grp = j / G, r = j % G;
+    std::memcpy(out_host + (grp * 2 * G + r) * d, gate + j * d, sizeof(uint16_t) * d);
+    std::memcpy(out_host + (grp * 2 * G + G + r) * d, up + j * d, sizeof(uint16_t) * d);
+  }
+  return MZC_OK;
+}
+
+mzc_status mzc_k_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_t n, int32_t hq,
+                               int32_t hkv, int32_t hd, const float* cos_t, const float* sin_t,
+                               const int32_t* block_table, int64_t n_logical, void* pool,
+                               int64_t pool_blocks, int32_t kv_dtype, uint16_t* q_out,
+                               int32_t* status, void* stream) {
+  if (!qkv || !pos || !cos_t || !sin_t || !block_table || !pool || !q_out || n < 0) return MZC_ERR_INVALID;
+  if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_rope_kv_write(qkv, pos, n, hq, hkv, hd, cos_t, sin_t, block_table, n_logical,
+                                pool, pool_blocks, kv_dtype, q_out, status, static_cast<cudaStream_t>(stream)));
+}
+
+int64_t mzc_k_attention_scratch_bytes(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys) {
+  if (n <= 0 || hkv <= 0) return 0;
+  int sp = 1, per = 0;
+  mzc::attention_split(n, hq, hkv, max_keys, sm_count(), &sp, &per);
+  return mzc::attention_scratch_bytes(n, hq, hd, sp);
+}
+
+mzc_status mzc_k_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
+                           int32_t hkv, int32_t hd, const int32_t* block_table, int64_t n_logical,
+                           const void* pool, int64_t pool_blocks, int32_t kv_dtype, uint16_t* out,
+                           int64_t max_keys, void* scratch, int64_t scratch_bytes, int32_t* status,
+                           void* stream) {
+  if (!q || !pos || !block_table || !pool || !out || n < 0 || max_keys <= 0) return MZC_ERR_INVALID;
+  if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_attention(q, pos, n, hq, hkv, hd, block_table, n_logical, pool, pool_blocks,
+                            kv_dtype, out, scratch, scratch_bytes, max_keys, sm_count(), status,
+                            static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_lm_head(const float* x_row, const float* g, int32_t d, float eps,
+                         const uint16_t* w, int64_t vocab, float* logits, void* stream) {
+  if (!x_row || !g || !w || !logits || d % 8 != 0 || vocab <= 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_lm_head(x_row, g, d, eps, w, vocab, logits, sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
+                       int64_t vocab, float* x, int32_t* status, void* stream) {
+  if (!tokens || !embed || !x || d % 8 != 0 || n < 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_embed(tokens, n, embed, d, vocab, x, status, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,444 @@
+// Host bookkeeping of the evictable LLM memory state (see state.hpp).
+#include "state.hpp"
+
+#include <algorithm>
+#include <cstring>
+
+namespace mzc {
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// ---- RangeAlloc ---------------------------------------------------------
+
+void RangeAlloc::reset(int64_t capacity) {
+  free_.clear();
+  capacity_ = capacity;
+  free_total_ = capacity;
+  if (capacity > 0) free_[0] = capacity;
+}
+
+int64_t RangeAlloc::alloc_contig(int64_t n) {
+  if (n <= 0) return -1;
+  for (auto it = free_.begin(); it != free_.end(); ++it) {
+    if (it->second >= n) {
+      int64_t start = it->first, len = it->second;
+      free_.erase(it);
+      if (len > n) free_[start + n] = len - n;
+      free_total_ -= n;
+      return start;
+    }
+  }
+  return -1;
+}
+
+std::vector<std::pair<int64_t, int64_t>> RangeAlloc::alloc_runs(int64_t n) {
+  std::vector<std::pair<int64_t, int64_t>> out;
+  if (n <= 0 || free_total_ < n) return out;
+  int64_t s = alloc_contig(n);
+  if (s >= 0) {
+    out.emplace_back(s, n);
+    return out;
+  }
+  int64_t need = n;
+  while (need > 0) {
+    auto it = free_.begin();
+    int64_t start = it->first, len = it->second;
+    int64_t take = std::min(len, need);
+    free_.erase(it);
+    if (len > take) free_[start + take] = len - take;
+    free_total_ -= take;
+    out.emplace_back(start, take);
+    need -= take;
+  }
+  return out;
+}
+
+void RangeAlloc::release(int64_t start, int64_t n) {
+  if (n <= 0) return;
+  free_total_ += n;
+  auto next = free_.lower_bound(start);
+  if (next != free_.begin()) {
+    auto prev = std::prev(next);
+    if (prev->first + prev->second == start) {
+      start = prev->first;
+      n += prev->second;
+      free_.erase(prev);
+    }
+  }
+  next = free_.lower_bound(start);
+  if (next != free_.end() && start + n == next->first) {
+    n += next->second;
+    free_.erase(next);
+  }
+  free_[start] = n;
+}
+
+// ---- State --------------------------------------------------------------
+
+mzc_status State::init(const mzc_model_shape& s, int64_t pool_blocks, int64_t host_store_bytes) {
+  if (s.n_layers <= 0 || s.d_model <= 0 || s.n_q_heads <= 0 || s.n_kv_heads <= 0 ||
+      s.head_dim <= 0 || s.ffn_dim <= 0 || s.vocab <= 0 || s.max_ctx <= 0)
+    return fail(MZC_ERR_INVALID, "shape fields must be positive");
+  if (s.block_tokens != 16) return fail(MZC_ERR_INVALID, "block_tokens must be 16");
+  if (s.n_q_heads % s.n_kv_heads != 0)
+    return fail(MZC_ERR_INVALID, "n_q_heads must be a multiple of n_kv_heads");
+  if (s.kv_dtype != MZC_KV_BF16 && s.kv_dtype != MZC_KV_FP16)
+    return fail(MZC_ERR_INVALID, "kv_dtype must be MZC_KV_BF16 or MZC_KV_FP16");
+  shape_ = s;
+  nblk_max_ = ceil_div(s.max_ctx, 16);
+  block_bytes_ = 2LL * s.n_kv_heads * 16 * s.head_dim * 2;
+  pool_blocks_ = pool_blocks > 0 ? pool_blocks : 2LL * s.n_layers * nblk_max_;
+  if (pool_blocks_ >= (1LL << 31)) return fail(MZC_ERR_INVALID, "pool_blocks too large");
+  host_bytes_ = host_store_bytes > 0 ? host_store_bytes : (int64_t)s.n_layers * nblk_max_ * block_bytes_;
+  tab_.assign((size_t)s.n_layers * nblk_max_, BlockEntry{});
+  regions_.clear();
+  w_state_.assign(s.n_layers, MZC_RESIDENT);
+  pool_.reset(pool_blocks_);
+  host_.reset(host_bytes_);
+  n_ctx_ = 0;
+  drop_t0_ = drop_t1_ = -1;
+  rec_pending_ = inflight_ = false;
+  return MZC_OK;
+}
+
+void State::drop_region_slot(int32_t r) {
+  Region& R = regions_[r];
+  if (--R.live == 0) {
+    host_.release(R.host_off, (int64_t)R.n_slots * block_bytes_);
+    R.n_slots = 0;
+  }
+}
+
+mzc_status State::evict_range(int32_t l0, int32_t l1, int64_t t0, int64_t t1, int32_t mode,
+                              std::vector<EvictMove>* moves) {
+  const int32_t L = shape_.n_layers;
+  if (mode != MZC_COPY && mode != MZC_DROP) return fail(MZC_ERR_INVALID, "mode must be COPY or DROP");
+  if (l0 < 0 || l1 > L || l0 >= l1) return fail(MZC_ERR_RANGE, "layer range out of bounds");
+  if (t0 < 0 || t1 > n_ctx_ || t0 >= t1) return fail(MZC_ERR_RANGE, "token range outside the context");
+  if (inflight_ || rec_pending_) return fail(MZC_ERR_STATE, "a restore or recompute is pending");
+  const int64_t b0 = t0 / 16, b1 = ceil_div(t1, 16);
+  for (int32_t l = l0; l < l1; ++l)
+    for (int64_t b = b0; b < b1; ++b)
+      if (at(l, b).st != MZC_RESIDENT)
+        return fail(MZC_ERR_STATE, "block " + std::to_string(b) + " of layer " +
+                                       std::to_string(l) + " is not resident");
+  if (mode == MZC_DROP) {
+    if (l0 != 0 || l1 != L)
+      return fail(MZC_ERR_INVALID, "DROP must cover every layer (recompute regenerates all layers)");
+    const int64_t d0 = b0 * 16, d1 = std::min(b1 * 16, n_ctx_);
+    if (has_drop() && !(d1 == drop_t0_ || d0 == drop_t1_))
+      return fail(MZC_ERR_INVALID, "dropped positions must stay one contiguous range");
+    for (int32_t l = 0; l < L; ++l)
+      for (int64_t b = b0; b < b1; ++b) {
+        BlockEntry& e = at(l, b);
+        pool_.release(e.phys, 1);
+        e = BlockEntry{};
+        e.st = MZC_DROPPED;
+      }
+    if (has_drop()) {
+      drop_t0_ = std::min(drop_t0_, d0);
+      drop_t1_ = std::max(drop_t1_, d1);
+    } else {
+      drop_t0_ = d0;
+      drop_t1_ = d1;
+    }
+    return MZC_OK;
+  }
+  // COPY: one packed region per layer, blocks in logical order.
+  const int64_t per_layer = (b1 - b0) * block_bytes_;
+  std::vector<int64_t> offs;
+  for (int32_t l = l0; l < l1; ++l) {
+    int64_t off = host_.alloc_contig(per_layer);
+    if (off < 0) {
+      for (size_t i = 0; i < offs.size(); ++i) host_.release(offs[i], per_layer);
+      return fail(MZC_ERR_OOM, "pinned swap store is full");
+    }
+    offs.push_back(off);
+  }
+  for (int32_t l = l0; l < l1; ++l) {
+    Region R;
+    R.layer = l;
+    R.host_off = offs[l - l0];
+    R.n_slots = (int32_t)(b1 - b0);
+    R.live = R.n_slots;
+    int32_t rid = (int32_t)regions_.size();
+    regions_.push_back(R);
+    EvictMove mv{l, R.host_off, {}};
+    for (int64_t b = b0; b < b1; ++b) {
+      BlockEntry& e = at(l, b);
+      mv.phys.push_back(e.phys);
+      pool_.release(e.phys, 1);
+      e.st = MZC_SWAPPED;
+      e.phys = -1;
+      e.region = rid;
+      e.idx = (int32_t)(b - b0);
+    }
+    if (moves) moves->push_back(std::move(mv));
+  }
+  return MZC_OK;
+}
+
+mzc_status State::evict_blocks(const int32_t* layer, const int64_t* blk, int64_t n, int32_t mode,
+                               std::vector<EvictMove>* moves) {
+  if (mode != MZC_COPY) return fail(MZC_ERR_INVALID, "scattered eviction supports COPY only");
+  if (n < 0 || (n > 0 && (!layer || !blk))) return fail(MZC_ERR_INVALID, "null block list");
+  if (inflight_ || rec_pending_) return fail(MZC_ERR_STATE, "a restore or recompute is pending");
+  const int32_t L = shape_.n_layers;
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  std::vector<std::vector<int64_t>> per(L);
+  for (int64_t i = 0; i < n; ++i) {
+    if (layer[i] < 0 || layer[i] >= L || blk[i] < 0 || blk[i] >= nb)
+      return fail(MZC_ERR_RANGE, "block index outside the context");
+    if (at(layer[i], blk[i]).st != MZC_RESIDENT)
+      return fail(MZC_ERR_STATE, "block is not resident");
+    per[layer[i]].push_back(blk[i]);
+  }
+  for (int32_t l = 0; l < L; ++l) {
+    auto& v = per[l];
+    std::sort(v.begin(), v.end());
+    if (std::adjacent_find(v.begin(), v.end()) != v.end())
+      return fail(MZC_ERR_INVALID, "duplicate block in the list");
+  }
+  std::vector<int64_t> offs(L, -1);
+  for (int32_t l = 0; l < L; ++l) {
+    if (per[l].empty()) continue;
+    offs[l] = host_.alloc_contig((int64_t)per[l].size() * block_bytes_);
+    if (offs[l] < 0) {
+      for (int32_t j = 0; j < l; ++j)
+        if (offs[j] >= 0) host_.release(offs[j], (int64_t)per[j].size() * block_bytes_);
+      return fail(MZC_ERR_OOM, "pinned swap store is full");
+    }
+  }
+  for (int32_t l = 0; l < L; ++l) {
+    if (per[l].empty()) continue;
+    Region R;
+    R.layer = l;
+    R.host_off = offs[l];
+    R.n_slots = (int32_t)per[l].size();
+    R.live = R.n_slots;
+    int32_t rid = (int32_t)regions_.size();
+    regions_.push_back(R);
+    EvictMove mv{l, R.host_off, {}};
+    for (size_t i = 0; i < per[l].size(); ++i) {
+      BlockEntry& e = at(l, per[l][i]);
+      mv.phys.push_back(e.phys);
+      pool_.release(e.phys, 1);
+      e.st = MZC_SWAPPED;
+      e.phys = -1;
+      e.region = rid;
+      e.idx = (int32_t)i;
+    }
+    if (moves) moves->push_back(std::move(mv));
+  }
+  return MZC_OK;
+}
+
+mzc_status State::evict_weights(int32_t l0, int32_t l1) {
+  if (l0 < 0 || l1 > shape_.n_layers || l0 >= l1) return fail(MZC_ERR_RANGE, "layer range out of bounds");
+  if (inflight_) return fail(MZC_ERR_STATE, "a restore is pending");
+  for (int32_t l = l0; l < l1; ++l)
+    if (w_state_[l] != MZC_RESIDENT) return fail(MZC_ERR_STATE, "layer weights are not resident");
+  for (int32_t l = l0; l < l1; ++l) w_state_[l] = MZC_SWAPPED;
+  return MZC_OK;
+}
+
+mzc_status State::recompute_tail(int64_t p, int64_t n) {
+  if (!has_drop()) return fail(MZC_ERR_STATE, "nothing is dropped");
+  if (p != drop_t0_ || n != drop_t1_ - drop_t0_)
+    return fail(MZC_ERR_RANGE, "recompute range must equal the dropped range [" +
+                                   std::to_string(drop_t0_) + ", " + std::to_string(drop_t1_) + ")");
+  rec_pending_ = true;
+  return MZC_OK;
+}
+
+mzc_status State::plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int32_t>* weight_layers) {
+  if (inflight_) return fail(MZC_ERR_STATE, "a restore is already in flight");
+  const int32_t L = shape_.n_layers;
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  int64_t need = 0;
+  for (int32_t l = 0; l < L; ++l)
+    for (int64_t b = 0; b < nb; ++b) need += at(l, b).st == MZC_SWAPPED;
+  if (need > pool_.free_total()) return fail(MZC_ERR_OOM, "KV pool cannot hold the restored blocks");
+  if (runs) runs->clear();
+  if (weight_layers) weight_layers->clear();
+  bool any = false;
+  for (int32_t l = 0; l < L; ++l) {  // forward-in: earliest layer first
+    if (w_state_[l] == MZC_SWAPPED) {
+      w_state_[l] = MZC_INFLIGHT;
+      if (weight_layers) weight_layers->push_back(l);
+      any = true;
+    }
+    // swapped blocks of layer l grouped by region, slot order
+    std::map<int32_t, std::vector<int64_t>> by_region;
+    for (int64_t b = 0; b < nb; ++b)
+      if (at(l, b).st == MZC_SWAPPED) by_region[at(l, b).region].push_back(b);
+    for (auto& kv : by_region) {
+      const Region& R = regions_[kv.first];
+      auto& blocks = kv.second;  // ascending logical index == ascending slot
+      auto ranges = pool_.alloc_runs((int64_t)blocks.size());
+      size_t bi = 0;
+      for (auto& rg : ranges) {
+        for (int64_t j = 0; j < rg.second; ++j, ++bi) {
+          BlockEntry& e = at(l, blocks[bi]);
+          e.st = MZC_INFLIGHT;
+          e.phys = (int32_t)(rg.first + j);
+          int64_t off = R.host_off + (int64_t)e.idx * block_bytes_;
+          // extend the previous run when host and device are both contiguous
+          if (runs && !runs->empty()) {
+            mzc_copy_run& pr = runs->back();
+            if (pr.layer == l && pr.phys_begin + pr.n_blocks == e.phys &&
+                pr.host_off + (int64_t)pr.n_blocks * block_bytes_ == off) {
+              pr.n_blocks += 1;
+              continue;
+            }
+          }
+          if (runs) runs->push_back(mzc_copy_run{l, 1, off, (int64_t)e.phys});
+        }
+      }
+      any = true;
+    }
+  }
+  inflight_ = any;
+  return MZC_OK;
+}
+
+mzc_status State::prepare_prefill(int64_t n_prompt, int64_t max_rows, PrefillPlan* plan) {
+  const int32_t L = shape_.n_layers;
+  if (n_prompt < 0) return fail(MZC_ERR_INVALID, "negative token count");
+  if (n_ctx_ + n_prompt > shape_.max_ctx) return fail(MZC_ERR_RANGE, "context would exceed max_ctx");
+  if (has_drop() && !rec_pending_)
+    return fail(MZC_ERR_STATE, "dropped blocks without a pending recompute");
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  for (int32_t l = 0; l < L; ++l) {
+    if (w_state_[l] == MZC_SWAPPED) return fail(MZC_ERR_STATE, "layer weights swapped, no restore in flight");
+    for (int64_t b = 0; b < nb; ++b)
+      if (at(l, b).st == MZC_SWAPPED) return fail(MZC_ERR_STATE, "swapped blocks without a restore in flight");
+  }
+  PrefillPlan P;
+  P.rec_begin = rec_pending_ ? drop_t0_ : 0;
+  P.rec_end = rec_pending_ ? drop_t1_ : 0;
+  P.prompt_begin = n_ctx_;
+  P.prompt_end = n_ctx_ + n_prompt;
+  const int64_t rows = (P.rec_end - P.rec_begin) + n_prompt;
+  if (rows > max_rows) return fail(MZC_ERR_OOM, "rows exceed max_rows");
+  // blocks to allocate per layer: dropped [db0, db1) and new [nb0, nb1)
+  const int64_t db0 = P.rec_begin / 16, db1 = ceil_div(P.rec_end, 16);
+  const int64_t nb0 = ceil_div(n_ctx_, 16), nb1 = ceil_div(n_ctx_ + n_prompt, 16);
+  const int64_t per_layer = (db1 - db0) + (nb1 - nb0);
+  if (per_layer * L > pool_.free_total()) return fail(MZC_ERR_OOM, "KV pool is full");
+  for (int32_t l = 0; l < L; ++l) {
+    auto ranges = pool_.alloc_runs(per_layer);
+    std::vector<int32_t> ids;
+    for (auto& rg : ranges)
+      for (int64_t j = 0; j < rg.second; ++j) ids.push_back((int32_t)(rg.first + j));
+    size_t k = 0;
+    for (int64_t b = db0; b < db1; ++b) at(l, b).phys = ids[k++];  // stays DROPPED until complete()
+    for (int64_t b = nb0; b < nb1; ++b) {
+      BlockEntry& e = at(l, b);
+      e = BlockEntry{};
+      e.st = MZC_EMPTY;  // becomes RESIDENT in complete()
+      e.phys = ids[k++];
+    }
+  }
+  P.kv_wait_prompt.assign(L, 0);
+  P.kv_wait_rec.assign(L, 0);
+  P.kv_wait_write.assign(L, 0);
+  P.w_wait.assign(L, 0);
+  const int64_t last_partial = (n_ctx_ % 16) ? n_ctx_ / 16 : -1;
+  for (int32_t l = 0; l < L; ++l) {
+    P.w_wait[l] = w_state_[l] == MZC_INFLIGHT;
+    for (int64_t b = 0; b < nb; ++b) {
+      if (at(l, b).st != MZC_INFLIGHT) continue;
+      P.kv_wait_prompt[l] = 1;
+      if (b * 16 < P.rec_end) P.kv_wait_rec[l] = 1;
+      if (b == last_partial && n_prompt > 0) P.kv_wait_write[l] = 1;
+    }
+  }
+  *plan = std::move(P);
+  return MZC_OK;
+}
+
+void State::abort_prefill(const PrefillPlan& P) {
+  const int64_t db0 = P.rec_begin / 16, db1 = ceil_div(P.rec_end, 16);
+  const int64_t nb0 = ceil_div(P.prompt_begin, 16), nb1 = ceil_div(P.prompt_end, 16);
+  for (int32_t l = 0; l < shape_.n_layers; ++l) {
+    for (int64_t b = db0; b < db1; ++b) {
+      BlockEntry& e = at(l, b);
+      if (e.phys >= 0) pool_.release(e.phys, 1);
+      e.phys = -1;
+    }
+    for (int64_t b = nb0; b < nb1; ++b) {
+      BlockEntry& e = at(l, b);
+      if (e.phys >= 0) pool_.release(e.phys, 1);
+      e = BlockEntry{};
+    }
+  }
+}
+
+void State::complete(int64_t n_prompt) {
+  const int32_t L = shape_.n_layers;
+  const int64_t nb_new = ceil_div(n_ctx_ + n_prompt, 16);
+  for (int32_t l = 0; l < L; ++l) {
+    if (w_state_[l] == MZC_INFLIGHT) w_state_[l] = MZC_RESIDENT;
+    for (int64_t b = 0; b < nb_new; ++b) {
+      BlockEntry& e = at(l, b);
+      if (e.st == MZC_INFLIGHT) {
+        drop_region_slot(e.region);
+        e.st = MZC_RESIDENT;
+        e.region = e.idx = -1;
+      } else if (e.st == MZC_DROPPED && rec_pending_) {
+        e.st = MZC_RESIDENT;
+      } else if (e.st == MZC_EMPTY && e.phys >= 0) {
+        e.st = MZC_RESIDENT;
+      }
+    }
+  }
+  if (rec_pending_) {
+    rec_pending_ = false;
+    drop_t0_ = drop_t1_ = -1;
+  }
+  inflight_ = false;
+  n_ctx_ += n_prompt;
+}
+
+mzc_status State::truncate(int64_t n) {
+  if (n < 0 || n > n_ctx_) return fail(MZC_ERR_RANGE, "truncate beyond the context");
+  if (inflight_ || rec_pending_) return fail(MZC_ERR_STATE, "a restore or recompute is pending");
+  const int64_t keep = ceil_div(n, 16), nb = ceil_div(n_ctx_, 16);
+  for (int32_t l = 0; l < shape_.n_layers; ++l)
+    for (int64_t b = keep; b < nb; ++b) {
+      BlockEntry& e = at(l, b);
+      if (e.st == MZC_RESIDENT && e.phys >= 0) pool_.release(e.phys, 1);
+      if (e.st == MZC_SWAPPED) drop_region_slot(e.region);
+      e = BlockEntry{};
+    }
+  n_ctx_ = n;
+  if (has_drop()) {
+    drop_t1_ = std::min(drop_t1_, n);
+    if (drop_t1_ <= drop_t0_) drop_t0_ = drop_t1_ = -1;
+  }
+  return MZC_OK;
+}
+
+void State::counts(mzc_stats_t* o) const {
+  std::memset(o, 0, sizeof(*o));
+  o->context_tokens = n_ctx_;
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  for (int32_t l = 0; l < shape_.n_layers; ++l) {
+    for (int64_t b = 0; b < nb; ++b) {
+      uint8_t s = at(l, b).st;
+      o->blocks_resident += s == MZC_RESIDENT;
+      o->blocks_swapped += s == MZC_SWAPPED || s == MZC_INFLIGHT;
+      o->blocks_dropped += s == MZC_DROPPED;
+    }
+    o->weights_evicted_layers += w_state_[l] != MZC_RESIDENT;
+  }
+  o->pool_free_blocks = pool_.free_total();
+}
+
+void State::block_table(std::vector<int32_t>* out) const {
+  out->resize(tab_.size());
+  for (size_t i = 0; i < tab_.size(); ++i) (*out)[i] = tab_[i].phys;
+}
+
+}  // namespace mzc

@@ -1,0 +1,193 @@
+"""CPU checks of the C ABI: the library loads without a GPU and exports every
+entry point include/mzc.h declares; the host bookkeeping (mzc_state_*)
+matches the plain-Python state model; the hybrid split solver against brute
+force of its own cost definition."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2609_01338_gb300 as m
+from paper_2609_01338_gb300 import mzc as M
+from oracle.state_model import StateModel
+from synth import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    txt = open(os.path.join(ROOT, "include", "mzc.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(mzc_\w+)\s*\(", txt)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = m.load()
+    names = _declared()
+    assert len(names) >= 30
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) >= set(M._SIGS) | set(M._RESTYPES)
+
+
+def test_struct_sizes_match_c_layout():
+    assert ctypes.sizeof(M.mzc_model_shape) == 56
+    assert ctypes.sizeof(M.mzc_options) == 32
+    assert ctypes.sizeof(M.mzc_copy_run) == 24
+    assert ctypes.sizeof(M.mzc_stats_t) == 80
+
+
+SMALL = W.scaled(W.TINY, n_layers=3, max_ctx=640)
+
+
+def _states(st, L, nblk):
+    return [[m.mzc_state_query(st, l, b)[0] for b in range(nblk)] for l in range(L)]
+
+
+def _check_phys_valid(st, L, nblk, pool):
+    seen = set()
+    for l in range(L):
+        for b in range(nblk):
+            s, p = m.mzc_state_query(st, l, b)
+            if s in (m.MZC_RESIDENT, m.MZC_INFLIGHT):
+                assert 0 <= p < pool and p not in seen
+                seen.add(p)
+
+
+def _apply(st, model, op):
+    kind = op[0]
+    if kind == "append":
+        return M.status_of("mzc_state_append", st, op[1]), model.append(op[1])
+    if kind == "evict":
+        return M.status_of("mzc_state_evict", st, *op[1:]), model.evict(*op[1:])
+    if kind == "recompute":
+        return M.status_of("mzc_state_recompute_tail", st, *op[1:]), model.recompute_tail(*op[1:])
+    if kind == "restore":
+        runs = (M.mzc_copy_run * 4096)()
+        n = ctypes.c_int64()
+        return (M.status_of("mzc_state_plan_restore", st, runs, 4096, ctypes.byref(n)),
+                model.restore())
+    if kind == "truncate":
+        return M.status_of("mzc_state_truncate", st, op[1]), model.truncate(op[1])
+    if kind == "blocks":
+        pairs = op[1]
+        ls = np.array([p[0] for p in pairs], np.int32)
+        bs = np.array([p[1] for p in pairs], np.int64)
+        return (M.status_of("mzc_state_evict_blocks", st, ls.ctypes.data, bs.ctypes.data,
+                            len(pairs), 0), model.evict_blocks(pairs))
+    raise ValueError(kind)
+
+
+def test_state_machine_scripted_sequence():
+    pool = 200
+    st = m.mzc_state_create(SMALL, pool_blocks=pool)
+    model = StateModel(3, 640)
+    script = [
+        ("append", 300), ("evict", 0, 3, 200, 300, 1), ("evict", 0, 3, 100, 120, 0),
+        ("evict", 0, 3, 100, 120, 0),          # double evict -> STATE
+        ("evict", 0, 2, 50, 60, 1),            # DROP of a layer subset -> INVALID
+        ("append", 5),                         # dropped without recompute -> STATE
+        ("recompute", 192, 100),               # wrong range -> RANGE
+        ("recompute", 192, 108), ("restore",), ("append", 20),
+        ("evict", 1, 2, 0, 320, 0), ("restore",), ("append", 0), ("truncate", 250),
+        ("evict", 0, 3, 240, 250, 1), ("evict", 0, 3, 200, 240, 1), ("recompute", 192, 58),
+        ("append", 7), ("truncate", 0), ("append", 640), ("append", 1),
+    ]
+    for op in script:
+        got, want = _apply(st, model, op)
+        assert got == want, (op, got, want)
+        assert _states(st, 3, model.nblk) == model.st, op
+        _check_phys_valid(st, 3, model.nblk, pool)
+    M._call("mzc_state_destroy", st)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_state_machine_random_sequences(seed):
+    rng = np.random.default_rng(seed)
+    pool = 160
+    st = m.mzc_state_create(SMALL, pool_blocks=pool)
+    model = StateModel(3, 640)
+    for _ in range(60):
+        k = rng.integers(0, 7)
+        n = model.n_ctx
+        if k == 0:
+            op = ("append", int(rng.integers(0, 80)))
+        elif k == 1 and n > 0:
+            t0 = int(rng.integers(0, n)); t1 = int(rng.integers(t0 + 1, n + 1))
+            l0 = int(rng.integers(0, 3)); l1 = int(rng.integers(l0 + 1, 4))
+            op = ("evict", l0, l1, t0, t1, int(rng.integers(0, 2)))
+        elif k == 2 and n > 0:
+            t0 = int(rng.integers(0, n))
+            op = ("evict", 0, 3, t0, n, 1)
+        elif k == 3:
+            d = model.drop or (0, 0)
+            op = ("recompute", d[0], d[1] - d[0])
+        elif k == 4:
+            op = ("restore",)
+        elif k == 5 and n > 0:
+            nb = -(-n // 16)
+            cnt = int(rng.integers(1, 6))
+            pairs = list({(int(rng.integers(0, 3)), int(rng.integers(0, nb))) for _ in range(cnt)})
+            op = ("blocks", pairs)
+        elif k == 6:
+            op = ("truncate", int(rng.integers(0, n + 1)))
+        else:
+            op = ("append", 16)
+        got, want = _apply(st, model, op)
+        if got == 4:  # OOM from the physical pool: the model has no capacity, skip the op
+            continue
+        assert got == want, (op, got, want)
+        assert _states(st, 3, model.nblk) == model.st, op
+        _check_phys_valid(st, 3, model.nblk, pool)
+    M._call("mzc_state_destroy", st)
+
+
+def test_restore_plan_packs_runs_forward_in():
+    st = m.mzc_state_create(SMALL, pool_blocks=400)
+    M._call("mzc_state_append", st, 640)
+    # scattered blocks of layer 2 and 0, then a tail of layer 1
+    ls = np.array([2, 2, 0, 0, 0], np.int32)
+    bs = np.array([5, 9, 1, 2, 3], np.int64)
+    M._call("mzc_state_evict_blocks", st, ls.ctypes.data, bs.ctypes.data, 5, 0)
+    M._call("mzc_state_evict", st, 1, 2, 320, 640, 0)
+    runs = m.mzc_state_plan_restore(st)
+    layers = [r[0] for r in runs]
+    assert layers == sorted(layers)  # forward-in: earliest layer first
+    # with enough contiguous free blocks each layer's swapped set is one copy
+    assert len(runs) == 3
+    assert sum(r[1] for r in runs) == 5 + 20
+    bb = 2 * SMALL["n_kv_heads"] * 16 * SMALL["head_dim"] * 2
+    for l, nb, off, p0 in runs:
+        assert off % bb == 0 and p0 >= 0
+
+
+def test_hybrid_split_bruteforce_and_limits():
+    prof = M.mzc_profile(200.0, 6000.0, 1000.0, 400.0, 30.0)
+    sh = W.THREE_B
+
+    def cost(p, s, n, P):
+        d, hq, hkv, hd, f, L = (sh[k] for k in ("d_model", "n_q_heads", "n_kv_heads", "head_dim",
+                                                  "ffn_dim", "n_layers"))
+        params = d * (hq + 2 * hkv) * hd + hq * hd * d + 3 * d * f
+        rows = s - p + P
+        comp = 0.0
+        if rows > 0:
+            gemm = max(rows * 2 * params / 1000e12, 2 * params / 6000e9)
+            pairs = sum(range(p + 1, s + 1)) + sum(range(n + 1, n + P + 1))
+            comp = L * (gemm + pairs * 4 * hd * hq / 400e12 + 30e-6)
+        copy = -(-(n - s) // 16) * L * 2 * hkv * 16 * hd * 2 / 200e9
+        return max(comp, copy)
+
+    for p, n, P in ((16384, 32768, 128), (0, 4096, 0), (31744, 32768, 512), (1000 // 16 * 16, 1000, 3)):
+        s = m.mzc_plan_split(sh, prof, p, n, P)
+        assert p <= s <= n and ((s - p) % 16 == 0 or s == n)
+        cands = list(range(p, n, 16)) + [n]
+        best = min(cost(p, c, n, P) for c in cands)
+        assert cost(p, s, n, P) <= best * (1 + 1e-9)
+    # a link much faster than compute -> copy everything; much slower -> recompute everything
+    fast = M.mzc_profile(1e6, 6000.0, 1000.0, 400.0, 30.0)
+    slow = M.mzc_profile(1e-3, 6000.0, 1000.0, 400.0, 30.0)
+    assert m.mzc_plan_split(sh, fast, 0, 4096, 16) == 0
+    assert m.mzc_plan_split(sh, slow, 0, 4096, 16) == 4096

@@ -1,0 +1,232 @@
+"""Kernel parity on the GPU: each sm_103a kernel, called through the C ABI,
+against the CPU oracle's definition of the same operation on the same seeded
+inputs.  Tolerances follow from the arithmetic: fp16 outputs are within one
+fp16 rounding (2^-11 relative) of an fp32 reference plus fp32 accumulation-
+order noise; the attention's P operand is rounded to the KV type."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_01338_gb300 as m
+import synth
+from tests.gpu_util import (bf16_dev, f32_dev, i32_dev, to_np_u16, kv_bits_to_f32,
+                            f32_to_kv_bits, rel_err, f16_bits, f16_to_f32,
+                            bf16_weights_exact_in_f16)
+
+pytestmark = pytest.mark.gpu
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _rand_bf16(tid, shape, sigma=1.0):
+    return synth.normal_bf16(7, tid, shape, sigma=sigma)
+
+
+# ---- GEMM (tcgen05 / TMEM / TMA) -------------------------------------------
+
+GEMM_SHAPES = [(1, 64, 64), (7, 80, 72), (128, 256, 512), (130, 384, 320), (300, 1024, 2048),
+               (1000, 512, 256), (4224, 3072, 2048)]
+
+
+def _act16(tid, shape):
+    return f16_bits(synth.bf16_bits_to_f32(_rand_bf16(tid, shape)))
+
+
+@pytest.mark.parametrize("mm,nn,kk", GEMM_SHAPES)
+def test_gemm_store_f16(mm, nn, kk):
+    torch = _torch()
+    a = _act16(1, (mm, kk))
+    wb, wh = bf16_weights_exact_in_f16(_rand_bf16(2, (nn, kk), sigma=0.05))
+    out = torch.zeros((mm, nn), dtype=torch.int16, device="cuda")
+    m.mzc_k_gemm(bf16_dev(a), bf16_dev(wh), out, mm, nn, kk, 0)
+    torch.cuda.synchronize()
+    got = f16_to_f32(to_np_u16(out))
+    rows = np.unique(np.linspace(0, mm - 1, min(mm, 256)).astype(int))
+    ref = oracle.linear(f16_to_f32(a[rows]), wb)
+    err = np.abs(got[rows] - ref)
+    assert np.all(err <= 2.0 ** -10 * np.abs(ref) + 1e-5 * np.max(np.abs(ref)))
+
+
+@pytest.mark.parametrize("mm,nn,kk", [(5, 64, 128), (200, 256, 768), (4224, 2048, 2048)])
+def test_gemm_residual_add(mm, nn, kk):
+    torch = _torch()
+    a = _act16(3, (mm, kk))
+    wb, wh = bf16_weights_exact_in_f16(_rand_bf16(4, (nn, kk), sigma=0.05))
+    x0 = np.random.default_rng(0).standard_normal((mm, nn)).astype(np.float32)
+    out = f32_dev(x0)
+    m.mzc_k_gemm(bf16_dev(a), bf16_dev(wh), out, mm, nn, kk, 1)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    rows = np.unique(np.linspace(0, mm - 1, min(mm, 256)).astype(int))
+    ref = x0[rows] + oracle.linear(f16_to_f32(a[rows]), wb)
+    assert np.max(np.abs(got[rows] - ref)) <= 1e-4 * np.max(np.abs(ref))
+
+
+@pytest.mark.parametrize("mm,f,kk", [(3, 128, 256), (260, 384, 512), (70, 704, 256),
+                                     (4224, 1024, 2048)])
+def test_gemm_swiglu(mm, f, kk):
+    torch = _torch()
+    a = _act16(5, (mm, kk))
+    wg, wgh = bf16_weights_exact_in_f16(_rand_bf16(6, (f, kk), sigma=0.05))
+    wu, wuh = bf16_weights_exact_in_f16(_rand_bf16(8, (f, kk), sigma=0.05))
+    packed = m.mzc_k_swiglu_pack(wgh, wuh)
+    out = torch.zeros((mm, f), dtype=torch.int16, device="cuda")
+    m.mzc_k_gemm(bf16_dev(a), bf16_dev(packed), out, mm, 2 * f, kk, 2)
+    torch.cuda.synchronize()
+    got = f16_to_f32(to_np_u16(out))
+    rows = np.unique(np.linspace(0, mm - 1, min(mm, 128)).astype(int))
+    af = f16_to_f32(a[rows])
+    ref = oracle.swiglu(oracle.linear(af, wg), oracle.linear(af, wu))
+    err = np.abs(got[rows] - ref)
+    assert np.all(err <= 2.0 ** -9 * np.abs(ref) + 2e-5 * np.max(np.abs(ref)))
+
+
+# ---- RMSNorm, embedding, LM head --------------------------------------------
+
+@pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072)])
+def test_rmsnorm(n, d):
+    torch = _torch()
+    rng = np.random.default_rng(n)
+    x = (rng.standard_normal((n, d)) * rng.uniform(0.01, 3.0, (n, 1))).astype(np.float32)
+    g = rng.uniform(0.5, 1.5, d).astype(np.float32)
+    y = torch.zeros((n, d), dtype=torch.int16, device="cuda")
+    m.mzc_k_rmsnorm(f32_dev(x), f32_dev(g), n, d, 1e-5, y)
+    torch.cuda.synchronize()
+    got = f16_to_f32(to_np_u16(y))
+    ref = oracle.rmsnorm(x, g, 1e-5)
+    assert np.all(np.abs(got - ref) <= 2.0 ** -10 * np.abs(ref) + 1e-6)
+
+
+def test_embed_exact_and_bad_token_flagged():
+    torch = _torch()
+    V, d = 1000, 512
+    E = _rand_bf16(9, (V, d), sigma=0.02)
+    toks = synth.tokens(1, 9, 77, V)
+    x = torch.zeros((77, d), dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    m.mzc_k_embed(i32_dev(toks), 77, bf16_dev(E), d, V, x, status)
+    torch.cuda.synchronize()
+    assert np.array_equal(x.cpu().numpy(), synth.bf16_bits_to_f32(E[toks]))
+    assert int(status.item()) == 0
+    bad = toks.copy()
+    bad[3] = V + 5
+    m.mzc_k_embed(i32_dev(bad), 77, bf16_dev(E), d, V, x, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == m.MZC_ERR_DEVICE
+
+
+@pytest.mark.parametrize("V,d", [(1024, 256), (128256, 2048), (50000, 3072)])
+def test_lm_head(V, d):
+    torch = _torch()
+    rng = np.random.default_rng(V)
+    x = rng.standard_normal(d).astype(np.float32)
+    g = rng.uniform(0.5, 1.5, d).astype(np.float32)
+    W = _rand_bf16(10, (V, d), sigma=0.02)
+    logits = torch.zeros(V, dtype=torch.float32, device="cuda")
+    m.mzc_k_lm_head(f32_dev(x), f32_dev(g), d, 1e-5, bf16_dev(W), V, logits)
+    torch.cuda.synchronize()
+    h = oracle.rmsnorm(x[None], g, 1e-5)
+    ref = oracle.linear(h, W)[0]
+    assert np.max(np.abs(logits.cpu().numpy() - ref)) <= 1e-5 * np.max(np.abs(ref)) * np.sqrt(d)
+
+
+# ---- rotary + KV-block write -------------------------------------------------
+
+def _pool_layout(n_blocks_logical, pool_blocks, seed):
+    perm = synth.permutation(synth.SEED_EVICT, seed, pool_blocks)[:n_blocks_logical]
+    return perm.astype(np.int32)
+
+
+@pytest.mark.parametrize("hq,hkv,hd,kvd", [(4, 2, 64, 0), (32, 8, 64, 1), (24, 8, 128, 0)])
+def test_rope_kv_write(hq, hkv, hd, kvd):
+    torch = _torch()
+    n_logical, pool_blocks = 40, 64
+    # ragged positions: a recompute range and a prompt range
+    pos = np.concatenate([np.arange(100, 180), np.arange(600, 637)]).astype(np.int32)
+    n = pos.size
+    qkv = _act16(11, (n, (hq + 2 * hkv) * hd))
+    table = _pool_layout(n_logical, pool_blocks, hd + kvd)
+    cos_t, sin_t = oracle.rope_table(n_logical * 16, hd, 500000.0)
+    blk_elems = 2 * hkv * 16 * hd
+    pool = torch.zeros(pool_blocks * blk_elems, dtype=torch.int16, device="cuda")
+    q_out = torch.zeros((n, hq, hd), dtype=torch.int16, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    m.mzc_k_rope_kv_write(bf16_dev(qkv), i32_dev(pos), n, hq, hkv, hd, f32_dev(cos_t),
+                          f32_dev(sin_t), i32_dev(table), n_logical, pool, pool_blocks, kvd,
+                          q_out, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    x = f16_to_f32(qkv).reshape(n, hq + 2 * hkv, hd)
+    q_ref = oracle.round_kv(oracle.rope(x[:, :hq], pos, 500000.0), kvd)
+    k_ref = oracle.round_kv(oracle.rope(x[:, hq:hq + hkv], pos, 500000.0), kvd)
+    v_ref = oracle.round_kv(x[:, hq + hkv:], kvd)
+    ulp = 2.0 ** (-10 if kvd == 1 else -7)
+    q_got = kv_bits_to_f32(to_np_u16(q_out), kvd)
+    assert np.all(np.abs(q_got - q_ref) <= ulp * np.abs(q_ref) + 1e-7)
+    pool_np = to_np_u16(pool).reshape(pool_blocks, 2, hkv, 16, hd)
+    k_got = np.stack([pool_np[table[p // 16], 0, :, p % 16] for p in pos])
+    v_got = np.stack([pool_np[table[p // 16], 1, :, p % 16] for p in pos])
+    assert np.all(np.abs(kv_bits_to_f32(k_got, kvd) - k_ref) <= ulp * np.abs(k_ref) + 1e-7)
+    assert np.array_equal(kv_bits_to_f32(v_got, kvd), v_ref)
+    # nothing else in the pool was written
+    written = np.zeros((pool_blocks, 16), bool)
+    for p in pos:
+        written[table[p // 16], p % 16] = True
+    untouched = pool_np.transpose(0, 3, 1, 2, 4)[~written]
+    assert not untouched.any()
+
+
+# ---- block-table attention ----------------------------------------------------
+
+def _attention_case(hq, hkv, hd, kvd, ctx, pos, seed, use_scratch=True):
+    torch = _torch()
+    n = pos.size
+    n_logical = -(-ctx // 16)
+    pool_blocks = n_logical + 13
+    table = _pool_layout(n_logical, pool_blocks, seed)
+    rng = np.random.default_rng(seed)
+    kf = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
+    vf = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
+    qf = f32_to_kv_bits((rng.standard_normal((n, hq, hd)) * 2.0).astype(np.float32), kvd)
+    pool_np = np.zeros((pool_blocks, 2, hkv, 16, hd), np.uint16)
+    for p in range(ctx):
+        pool_np[table[p // 16], 0, :, p % 16] = kf[p]
+        pool_np[table[p // 16], 1, :, p % 16] = vf[p]
+    pool = torch.from_numpy(pool_np.view(np.int16)).cuda()
+    out = torch.zeros((n, hq, hd), dtype=torch.int16, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    sb = m.mzc_k_attention_scratch_bytes(n, hq, hkv, hd, ctx) if use_scratch else 0
+    scratch = torch.empty(max(sb, 4), dtype=torch.uint8, device="cuda") if sb else None
+    m.mzc_k_attention(torch.from_numpy(qf.view(np.int16)).cuda(), i32_dev(pos), n, hq, hkv, hd,
+                      i32_dev(table), n_logical, pool, pool_blocks, kvd, out, ctx, scratch, sb,
+                      status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    got = f16_to_f32(to_np_u16(out))
+    ref = oracle.attention(kv_bits_to_f32(qf, kvd), pos, kv_bits_to_f32(kf, kvd),
+                           kv_bits_to_f32(vf, kvd))
+    return got, ref, sb
+
+
+@pytest.mark.parametrize("hq,hkv,hd,kvd", [(4, 2, 64, 0), (32, 8, 64, 1), (24, 8, 128, 0),
+                                           (8, 8, 128, 1)])
+def test_attention_ragged_rows(hq, hkv, hd, kvd):
+    ctx = 700
+    pos = np.concatenate([np.arange(300, 383), np.arange(680, 700), [0, 17]]).astype(np.int32)
+    got, ref, _ = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=hq + hd)
+    assert rel_err(got, ref) < 1e-2
+    assert np.mean(np.abs(got - ref)) < 2e-3 * np.max(np.abs(ref))
+
+
+@pytest.mark.parametrize("hq,hkv,hd,kvd", [(32, 8, 64, 1), (24, 8, 128, 0)])
+def test_attention_split_kv_long_context(hq, hkv, hd, kvd):
+    ctx = 5000
+    pos = np.arange(ctx - 9, ctx).astype(np.int32)
+    got, ref, sb = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=3)
+    assert sb > 0  # the split path ran
+    assert rel_err(got, ref) < 1e-2
+    got2, ref2, _ = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=3, use_scratch=False)
+    assert rel_err(got2, ref2) < 1e-2
