@@ -42,6 +42,21 @@ sys.path.insert(0, ROOT)
 METRIC = "TTFT ms vs evicted fraction (1 GB300); recompute tok/s; % BF16 tensor peak"
 
 
+def _traffic(kernel_class):
+    """Per-launch DRAM bytes from the committed ncu capture, or None when the
+    kernel's source changed since the counters were taken."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
+            t = json.load(f)[kernel_class]
+        src = open(os.path.join(ROOT, t["source"]), "rb").read()
+        if hashlib.sha256(src).hexdigest()[:16] != t["source_sha"]:
+            return None
+        return t["bytes_per_launch"]
+    except Exception:
+        return None
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -282,7 +297,7 @@ def run_reference(args, name, sc, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="mzc", choices=["mzc", "reference"])
     ap.add_argument("--workload", default="1b_recompute",
@@ -367,14 +382,14 @@ def main():
             ach = k.flops / (k.ms * 1e-3) / 1e12
             peak = peaks["bf16_tflops_sustained"]
             roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 2), "peak": peak,
-                    "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
+                    "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom),
                     "peak_source": f"{src} bf16 sustained (fp16 operands: nominal fp16/bf16 ratio 1.0)",
                     "avg_launch_ms": round(k.ms / per, 4), "flops_per_launch": k.flops / per}
         else:
             ach = k.bytes / (k.ms * 1e-3) / 1e9
             peak = peaks["hbm_gbs"]
             roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": peak,
-                    "unit": "GB/s", "frac": round(ach / peak, 4), "traffic": None,
+                    "unit": "GB/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom),
                     "peak_source": f"{src} HBM copy", "avg_launch_ms": round(k.ms / per, 4),
                     "bytes_per_launch": k.bytes / per}
     rows = stats.rows_last
