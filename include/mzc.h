@@ -331,6 +331,32 @@ mzc_status mzc_k_attention(const uint16_t *q, const int32_t *pos, int64_t n, int
 int64_t mzc_k_attention_scratch_bytes(int64_t n, int32_t hq, int32_t hkv, int32_t hd,
                                       int64_t max_keys);
 
+/* The paper has no counterpart to this entry point: it is a convenience of
+ * this library.  Same arguments and result as mzc_k_attention, but the
+ * split-KV partials live in a fixed device array inside the library
+ * (MZC_ATTENTION_NOALLOC_SCRATCH_BYTES = 8 MiB, held by every GPU that loads
+ * the library until the process exits), so the call allocates nothing: no
+ * cudaMalloc, no cudaFree, no allocating library routine.  It is for callers
+ * that cannot allocate device memory when they call: a process whose device
+ * memory is being reclaimed (the memory pressure this library restores
+ * from) cannot count on an allocation succeeding at request time, a host
+ * framework may own all device memory through its own allocator, and
+ * cudaFree synchronizes the device.
+ * The first call on a device looks up the array's device address (a CUDA
+ * runtime query, no allocation); make that first call before any stream
+ * capture.  All calls share the array: calls that overlap on the GPU (for
+ * example on two streams) race on it.  Nothing in it has to start at zero.
+ * Errors: MZC_ERR_RANGE, with nothing launched, when the call's partials
+ * would exceed the array (mzc_k_attention_scratch_bytes() gives the need);
+ * MZC_ERR_INVALID for bad arguments; MZC_ERR_CUDA if the address lookup or
+ * the launch fails.  mzc_last_error(NULL) holds the text. */
+#define MZC_ATTENTION_NOALLOC_SCRATCH_BYTES (8LL << 20)
+mzc_status mzc_k_attention_noalloc(const uint16_t *q, const int32_t *pos, int64_t n, int32_t hq,
+                                   int32_t hkv, int32_t hd, const int32_t *block_table,
+                                   int64_t n_logical, const void *pool, int64_t pool_blocks,
+                                   int32_t kv_dtype, uint16_t *out, int64_t max_keys,
+                                   int32_t *status, void *stream);
+
 /* logits fp32 [vocab] = RMSNorm(x_row) * g  W^T, x_row fp32 [d], W bf16 [vocab][d]. */
 mzc_status mzc_k_lm_head(const float *x_row, const float *g, int32_t d, float eps,
                          const uint16_t *w, int64_t vocab, float *logits, void *stream);

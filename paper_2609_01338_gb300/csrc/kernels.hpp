@@ -51,6 +51,16 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,
                              uint16_t* out, void* scratch, int64_t scratch_bytes,
                              int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st);
+// Attention whose split-KV partials use a fixed array inside the library
+// (kAttnNoallocScratchBytes) instead of caller memory; no allocation.
+constexpr int64_t kAttnNoallocScratchBytes = 8LL << 20;
+int64_t attention_noalloc_need(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys,
+                               int num_sms);
+cudaError_t launch_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
+                                     int32_t hkv, int32_t hd, const int32_t* table,
+                                     int64_t n_logical, const void* pool, int64_t pool_blocks,
+                                     int32_t kv_dtype, uint16_t* out, int64_t max_keys,
+                                     int num_sms, int32_t* status, cudaStream_t st);
 cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float eps,
                            const uint16_t* w, int64_t vocab, float* logits, int num_sms,
                            cudaStream_t st);

@@ -1106,6 +1106,37 @@ mzc_status mzc_k_attention(const uint16_t* q, const int32_t* pos, int64_t n, int
                             static_cast<cudaStream_t>(stream)));
 }
 
+mzc_status mzc_k_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
+                                   int32_t hkv, int32_t hd, const int32_t* block_table,
+                                   int64_t n_logical, const void* pool, int64_t pool_blocks,
+                                   int32_t kv_dtype, uint16_t* out, int64_t max_keys,
+                                   int32_t* status, void* stream) {
+  if (!q || !pos || !block_table || !pool || !out || n < 0 || max_keys <= 0) {
+    g_create_error = "mzc_k_attention_noalloc: null pointer or negative size";
+    return MZC_ERR_INVALID;
+  }
+  if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) {
+    g_create_error = "mzc_k_attention_noalloc: unsupported head shape";
+    return MZC_ERR_INVALID;
+  }
+  const int64_t need = mzc::attention_noalloc_need(n, hq, hkv, hd, max_keys, sm_count());
+  if (need > mzc::kAttnNoallocScratchBytes) {
+    g_create_error = "mzc_k_attention_noalloc: this call's split-KV partials need " +
+                     std::to_string(need) + " bytes, more than the library's fixed " +
+                     std::to_string(mzc::kAttnNoallocScratchBytes) +
+                     "-byte array; use mzc_k_attention with caller scratch";
+    return MZC_ERR_RANGE;
+  }
+  cudaError_t e = mzc::launch_attention_noalloc(q, pos, n, hq, hkv, hd, block_table, n_logical,
+                                                pool, pool_blocks, kv_dtype, out, max_keys,
+                                                sm_count(), status, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    g_create_error = std::string("mzc_k_attention_noalloc: ") + cudaGetErrorString(e);
+    return MZC_ERR_CUDA;
+  }
+  return MZC_OK;
+}
+
 mzc_status mzc_k_lm_head(const float* x_row, const float* g, int32_t d, float eps,
                          const uint16_t* w, int64_t vocab, float* logits, void* stream) {
   if (!x_row || !g || !w || !logits || d % 8 != 0 || vocab <= 0) return MZC_ERR_INVALID;

@@ -116,6 +116,8 @@ _SIGS = {
                             c_vp, c_i64, c_i32, c_vp, c_vp, c_vp],
     "mzc_k_attention": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64, c_i32,
                         c_vp, c_i64, c_vp, c_i64, c_vp, c_vp],
+    "mzc_k_attention_noalloc": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64,
+                                c_i32, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_embed": [c_vp, c_i64, c_vp, c_i32, c_i64, c_vp, c_vp, c_vp],
 }
@@ -157,7 +159,7 @@ class MzcError(RuntimeError):
 def _call(fn, *args, ctx=None):
     s = getattr(load(), fn)(*args)
     if s != MZC_OK:
-        msg = load().mzc_last_error(ctx).decode() if fn.startswith("mzc_") else ""
+        msg = load().mzc_last_error(ctx).decode()
         raise MzcError(fn, s, msg)
     return s
 
@@ -389,6 +391,17 @@ def mzc_k_attention(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks,
     return _call("mzc_k_attention", _ptr(q), _ptr(pos), n, hq, hkv, hd, _ptr(table), n_logical,
                  _ptr(pool), pool_blocks, kv_dtype, _ptr(out), max_keys, _ptr(scratch),
                  scratch_bytes, _ptr(status), stream)
+
+
+MZC_ATTENTION_NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def mzc_k_attention_noalloc(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks,
+                            kv_dtype, out, max_keys, status, stream=None):
+    """Attention with the library's fixed split-KV array: allocates nothing."""
+    return _call("mzc_k_attention_noalloc", _ptr(q), _ptr(pos), n, hq, hkv, hd, _ptr(table),
+                 n_logical, _ptr(pool), pool_blocks, kv_dtype, _ptr(out), max_keys,
+                 _ptr(status), stream)
 
 
 def mzc_k_lm_head(x_row, g, d, eps, w, vocab, logits, stream=None):
