@@ -1,21 +1,32 @@
 // Causal grouped-query flash attention for prefill over a block-table KV
 // cache (the paper's single-pass attention over non-contiguous KV chunks with
-// online softmax, Sec. 4.2).
+// online softmax, Sec. 4.2), on the 5th-generation tensor cores.
 //
-// Rows: for KV head g, the n tokens x (hq/hkv) query heads sharing g are
-// flattened token-major (row r = token r / group, head g*group + r % group),
-// so one CTA's 64 rows reuse every K/V tile group times.  Each CTA walks
-// 64-key tiles of its key range: the 16-token blocks of a tile are located
-// through the block table and copied into shared memory with cp.async
-// (double-buffered, 16-byte chunks, XOR-swizzled rows), S = Q K^T and
-// O += P V run on warp-level tensor-core MMA (m16n8k16, fp32 accumulate),
-// and the softmax is the online (running max / running sum) form in base 2.
-// Keys past the tile's largest query position are zero-filled, never read.
-//
+// One CTA owns two tiles of 128 query rows of one KV head g: the n tokens x
+// (hq/hkv) query heads that share g are flattened token-major (row r = token
+// r / group, head g*group + r % group), so every K/V tile serves both Q tiles
+// and `group` heads.  Per BN-key tile of its key range:
+//   - warp 8 (one thread) looks each 16-token block of the tile up in the
+//     block table and fetches its K and V rows with TMA (a 16-row box per
+//     block and 64-column slice, 128-byte swizzle) into a 3-stage ring;
+//   - warp 9 (one thread) issues tcgen05.mma: S_t = Q_t K^T for both Q tiles
+//     into their TMEM S buffers (M=128, N=BN, K-major operands), and, once a
+//     softmax warpgroup has written P_t, O_t += P_t V into that tile's TMEM
+//     accumulator (A = P K-major, B = V MN-major, V in its stored layout);
+//   - warps 0-3 and 4-7 are the softmax warpgroups of the two Q tiles, one
+//     thread per row: the whole S row comes out of TMEM (the S buffer is
+//     released right away, so the next S runs on the tensor cores during the
+//     exponentials), is masked by the row's position on diagonal tiles,
+//     exponentiated in base 2 against a running reference maximum and stored
+//     as P (the KV type) into shared memory in the UMMA K-major swizzled
+//     layout.  O is rescaled in TMEM only when the maximum grows by more than
+//     2^8 ("lazy" rescale), so P stays <= 256.  The two warpgroups never wait
+//     for each other, so one exponentiates while the other waits on its S.
 // Long key ranges with few rows are split across CTAs (split-KV); each split
-// writes its normalised partial output and log-sum-exp to scratch and a
-// combine kernel merges them.
+// writes its normalised partial output and base-2 log-sum-exp, and a combine
+// kernel merges them.
 #include <cmath>
+#include <mutex>
 
 #include "kernels.hpp"
 #include "ptx.cuh"
@@ -24,240 +35,438 @@ namespace mzc {
 
 namespace {
 
-constexpr int kRows = 64;  // query rows per CTA (4 warps x 16)
-constexpr int kKeys = 64;  // keys per tile
+constexpr int kRowsPerCta = 256;  // two Q tiles of 128 rows
 
-__device__ __forceinline__ uint32_t swz(int row, int chunk) {
-  return static_cast<uint32_t>(chunk ^ (row & 7));
+template <int HD>
+struct AttnCfg {
+  static constexpr int BM = 128;                  // rows per Q tile (TMEM lanes)
+  static constexpr int BN = HD == 64 ? 128 : 64;  // keys per tile
+  static constexpr int STAGES = 3;
+  static constexpr int CB = HD / 64;              // 64-column slices of the head dim
+  static constexpr int Q_BYTES = BM * HD * 2;     // one Q tile
+  static constexpr int KV_BYTES = BN * HD * 2;    // K or V of one key tile
+  static constexpr int P_BYTES = BM * BN * 2;     // one P tile
+  static constexpr int OFF_K = 2 * Q_BYTES;
+  static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
+  static constexpr int OFF_P = OFF_V + STAGES * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;  // + barriers + alignment slack
+  // TMEM columns: S of tile t at t*BN, O of tile t at 2*BN + t*HD
+  static constexpr uint32_t O_COL = 2 * BN;
+  static constexpr uint32_t TMEM_COLS = 512;
+};
+
+// kind::f16 instruction descriptor: fp32 D, A/B fp16 (or bf16), A K-major,
+// B K-major or MN-major (bit 16), N >> 3 at bit 17, M >> 4 at bit 24.
+template <bool F16>
+__host__ __device__ constexpr uint32_t idesc_attn(int m, int n, bool b_mn_major) {
+  return (1u << 4) | (F16 ? 0u : (1u << 7) | (1u << 10)) | (b_mn_major ? (1u << 16) : 0u) |
+         (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(m >> 4) << 24);
 }
 
-template <int HD, bool F16>
-__global__ void __launch_bounds__(128) attn_kernel(
-    const uint16_t* __restrict__ q, const int32_t* __restrict__ pos, int n, int hq, int hkv,
-    const int32_t* __restrict__ table, int64_t n_logical, const uint16_t* __restrict__ pool,
-    int64_t pool_blocks, uint16_t* __restrict__ out, float* __restrict__ part_o,
-    float* __restrict__ part_lse, int keys_per_split, int n_splits, float scale_log2,
-    int32_t* status) {
-  constexpr int CH = HD / 8;  // 16-byte chunks per row
-  extern __shared__ __align__(128) uint8_t smem[];
-  uint16_t* sQ = reinterpret_cast<uint16_t*>(smem);
-  uint16_t* sK = sQ + kRows * HD;
-  uint16_t* sV = sK + 2 * kKeys * HD;
-  __shared__ int s_maxpos;
+// MN-major operand with 128-byte swizzle: 8 K-rows of 128 bytes (64 MN
+// elements) form an atom; LBO = byte stride between 64-element MN atoms,
+// SBO = byte stride between 8-row K groups.
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t lbo_bytes) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
 
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Bounded wait that also gives up at once when another thread of the CTA
+// already timed out (abort flag), so a failure cannot chain into long waits.
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, int32_t* status,
+                                         volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      set_status(status, kStatusTimeout);
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_ld_row(uint32_t taddr, float* v) {
+  if constexpr (N == 64) {
+    tmem_ld64w(taddr, v);
+  } else {
+    static_assert(N == 32, "row slices of 32 or 64 columns");
+    tmem_ld32w(taddr, v);
+  }
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_st_row(uint32_t taddr, const float* v) {
+  if constexpr (N == 64) {
+    tmem_st64w(taddr, v);
+  } else {
+    static_assert(N == 32, "row slices of 32 or 64 columns");
+    tmem_st32w(taddr, v);
+  }
+}
+
+// Threads: warps 0-3 and 4-7 are the softmax warpgroups of Q tiles 0 and 1
+// (thread = row of its tile, whole rows of S), warp 8 is the TMA producer and
+// TMEM owner, warp 9 issues the UMMAs.  Both Q tiles share every K/V tile.
+template <int HD, bool F16>
+__global__ void __launch_bounds__(320, 1) attn_tc_kernel(
+    const uint16_t* __restrict__ q, const int32_t* __restrict__ pos, int n, int hq, int hkv,
+    const int32_t* __restrict__ table, int64_t n_logical,
+    const __grid_constant__ CUtensorMap pool_map, int64_t pool_blocks,
+    uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
+    int keys_per_split, int n_splits, float scale_log2, int32_t* status) {
+  using C = AttnCfg<HD>;
+  constexpr int BN = C::BN;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = smem;  // [2 tiles]
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint8_t* sP = smem + C::OFF_P;  // [2 tiles]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* k_full = bars;                    // [STAGES]
+  uint64_t* v_full = bars + C::STAGES;        // [STAGES]
+  uint64_t* kv_empty = bars + 2 * C::STAGES;  // [STAGES]
+  uint64_t* s_full = bars + 3 * C::STAGES;    // [2 tiles] S(j) in TMEM
+  uint64_t* s_free = s_full + 2;              // [2 tiles] S(j) read into registers
+  uint64_t* p_full = s_free + 2;              // [2 tiles] P(j) in shared memory
+  uint64_t* p_free = p_full + 2;              // [2 tiles] P(j) V(j) done
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_maxpos;
+  __shared__ int s_abort;
+  volatile int* abort_flag = &s_abort;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = blockIdx.y;
   const int group = hq / hkv;
   const int R = n * group;
-  const int r0 = blockIdx.x * kRows;
+  const int r0 = blockIdx.x * kRowsPerCta;
   const int split = blockIdx.z;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int64_t blk_elems = 2LL * hkv * 16 * HD;
-  const int64_t v_off = static_cast<int64_t>(hkv) * 16 * HD;
 
-  if (tid == 0) s_maxpos = -1;
-  // Q tile
-  for (int i = tid; i < kRows * CH; i += 128) {
-    const int r = i / CH, c = i % CH;
-    const int rr = r0 + r;
-    uint16_t* dst = sQ + r * HD + swz(r, c) * 8;
-    if (rr < R) {
-      const int t = rr / group, h = g * group + rr % group;
-      cp_async16(smem_u32(dst), q + (static_cast<int64_t>(t) * hq + h) * HD + c * 8);
-    } else {
-      *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+  if (tid == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
     }
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(&s_full[t], 1);
+      mbar_init(&s_free[t], 4);  // one arrival per softmax warp of the tile
+      mbar_init(&p_full[t], 4);
+      mbar_init(&p_free[t], 1);
+    }
+    fence_barrier_init();
+    s_maxpos = -1;
+    s_abort = 0;
+    tma_prefetch_desc(&pool_map);
   }
-  cp_async_commit();
+  if (warp == 8) tmem_alloc(&s_tmem, C::TMEM_COLS);
+
+  // softmax threads: tile and row; the Q tiles in the UMMA K-major layout
+  const int qt = tid >> 7;  // Q tile of warps 0-7
+  const int row = tid & 127;
+  const int rr = r0 + qt * C::BM + row;
+  int row_pos = -1;
+  if (warp < 8) {
+    const int t = rr / group, h = g * group + rr % group;
+    if (rr < R) row_pos = pos[t];
+    uint8_t* q_tile = sQ + qt * C::Q_BYTES;
+#pragma unroll
+    for (int c = 0; c < HD / 8; ++c) {
+      uint8_t* dst = q_tile + (c >> 3) * (C::BM * 128) + row * 128 + (((c & 7) ^ (row & 7)) << 4);
+      if (rr < R)
+        cp_async16(smem_u32(dst), q + (static_cast<int64_t>(t) * hq + h) * HD + c * 8);
+      else
+        *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+    }
+    cp_async_commit();
+  }
   __syncthreads();
-  if (tid < kRows && r0 + tid < R) atomicMax(&s_maxpos, pos[(r0 + tid) / group]);
+  if (warp < 8 && row_pos >= 0) atomicMax(&s_maxpos, row_pos);
+  if (warp < 8) {
+    cp_async_wait<0>();
+    fence_async_smem();  // Q (generic-proxy writes) visible to the tensor core
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
   const int kv_len = s_maxpos + 1;
   const int k_begin = split * keys_per_split;
   const int k_end = min(kv_len, k_begin + keys_per_split);
+  const int T = k_end > k_begin ? (k_end - k_begin + BN - 1) / BN : 0;
 
-  // this thread's two rows in the m16n8 accumulator layout
-  const int rowA = r0 + warp * 16 + (lane >> 2);
-  const int rowB = rowA + 8;
-  const int posA = rowA < R ? pos[rowA / group] : -1;
-  const int posB = rowB < R ? pos[rowB / group] : -1;
-
-  float o[HD / 8][4];
+  if (warp == 8) {
+    if (lane == 0 && T > 0) {
+      // ---- TMA producer ----
+      const int64_t head_rows = static_cast<int64_t>(hkv) * 16;
+      int issued = 0;
+      for (int j = 0; j < T; ++j) {
+        const int s = j % C::STAGES;
+        const int kb = k_begin + j * BN;
+        int32_t phys[BN / 16];
+        int32_t first = -1;
 #pragma unroll
-  for (int j = 0; j < HD / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.0f;
-  float mA = -INFINITY, mB = -INFINITY, lA = 0.0f, lB = 0.0f;
-
-  auto load_tile = [&](int kb, int buf) {
-    uint16_t* dk = sK + buf * kKeys * HD;
-    uint16_t* dv = sV + buf * kKeys * HD;
-    for (int i = tid; i < kKeys * CH; i += 128) {
-      const int kr = i / CH, c = i % CH;
-      const int key = kb + kr;
-      const uint32_t off = kr * HD + swz(kr, c) * 8;
-      bool ok = key < k_end;
-      int32_t phys = -1;
+        for (int b = 0; b < BN / 16; ++b) {
+          const int key0 = kb + b * 16;
+          int32_t p = -1;
+          if (key0 < k_end) {
+            const int64_t blk = key0 >> 4;
+            p = blk < n_logical ? table[blk] : -1;
+            if (p < 0 || p >= pool_blocks) {
+              set_status(status, kStatusDevice);
+              p = -1;
+            }
+          }
+          if (b == 0) first = p < 0 ? 0 : p;
+          // blocks past the key range: any valid block (its keys are masked)
+          phys[b] = p < 0 ? first : p;
+        }
+        if (j >= C::STAGES &&
+            !wait_bar(&kv_empty[s], ((j / C::STAGES) - 1) & 1, status, abort_flag))
+          break;
+        mbar_arrive_expect_tx(&k_full[s], C::KV_BYTES);
+#pragma unroll
+        for (int b = 0; b < BN / 16; ++b) {
+          const int32_t y = static_cast<int32_t>((static_cast<int64_t>(phys[b]) * 2) * head_rows + g * 16);
+#pragma unroll
+          for (int c = 0; c < C::CB; ++c)
+            tma_load_2d(sK + s * C::KV_BYTES + c * (BN * 128) + b * 16 * 128, &pool_map,
+                        &k_full[s], c * 64, y);
+        }
+        mbar_arrive_expect_tx(&v_full[s], C::KV_BYTES);
+#pragma unroll
+        for (int b = 0; b < BN / 16; ++b) {
+          const int32_t y = static_cast<int32_t>((static_cast<int64_t>(phys[b]) * 2 + 1) * head_rows + g * 16);
+#pragma unroll
+          for (int c = 0; c < C::CB; ++c)
+            tma_load_2d(sV + s * C::KV_BYTES + c * (BN * 128) + b * 16 * 128, &pool_map,
+                        &v_full[s], c * 64, y);
+        }
+        issued = j + 1;
+      }
+      // drain: every fill issued has landed before shared memory is released
+      for (int j = issued - C::STAGES < 0 ? 0 : issued - C::STAGES; j < issued; ++j) {
+        wait_bar(&k_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+        wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+      }
+    }
+  } else if (warp == 9) {
+    if (lane == 0 && T > 0) {
+      // ---- UMMA issuer: S_0(j+1), S_1(j+1), P_0 V(j), P_1 V(j) ----
+      constexpr uint32_t id_s = idesc_attn<F16>(128, BN, false);
+      constexpr uint32_t id_o = idesc_attn<F16>(128, HD, true);
+      auto issue_s = [&](int t, int j) {
+        const int s = j % C::STAGES;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const int cb = kk >> 2, w = kk & 3;
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sQ + t * C::Q_BYTES + cb * (C::BM * 128) + w * 32));
+          const uint64_t bd = sdesc_k_sw128(smem_u32(sK + s * C::KV_BYTES + cb * (BN * 128) + w * 32));
+          umma_f16(tmem + t * BN, ad, bd, id_s, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[t]);
+      };
+      auto issue_pv = [&](int t, int j) {
+        const int s = j % C::STAGES;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const int pcb = kk >> 2, w = kk & 3;
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sP + t * C::P_BYTES + pcb * (C::BM * 128) + w * 32));
+          const uint64_t bd = sdesc_mn_sw128(smem_u32(sV + s * C::KV_BYTES + kk * 16 * 128), BN * 128);
+          umma_f16(tmem + C::O_COL + t * HD, ad, bd, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&p_free[t]);
+      };
+      bool ok = wait_bar(&k_full[0], 0, status, abort_flag);
       if (ok) {
-        const int blk = key >> 4;
-        phys = blk < n_logical ? table[blk] : -1;
-        if (phys < 0 || phys >= pool_blocks) {
-          set_status(status, kStatusDevice);
-          ok = false;
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+      }
+      for (int j = 0; ok && j < T; ++j) {
+        const int s = j % C::STAGES;
+        const uint32_t ph = j & 1;
+        if (j + 1 < T) {
+          // the next S of each tile runs while the softmax exponentiates S(j)
+          if (!wait_bar(&k_full[(j + 1) % C::STAGES], ((j + 1) / C::STAGES) & 1, status, abort_flag)) break;
+          if (!wait_bar(&s_free[0], ph, status, abort_flag)) break;
+          tc_fence_after();
+          issue_s(0, j + 1);
+          if (!wait_bar(&s_free[1], ph, status, abort_flag)) break;
+          tc_fence_after();
+          issue_s(1, j + 1);
+        }
+        if (!wait_bar(&v_full[s], (j / C::STAGES) & 1, status, abort_flag)) break;
+        if (!wait_bar(&p_full[0], ph, status, abort_flag)) break;
+        tc_fence_after();
+        issue_pv(0, j);
+        if (!wait_bar(&p_full[1], ph, status, abort_flag)) break;
+        tc_fence_after();
+        issue_pv(1, j);
+        umma_commit(&kv_empty[s]);
+      }
+    }
+  } else {
+    // ---- softmax: thread = row of Q tile qt, all BN columns ----
+    const uint32_t trow = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t s_col = qt * BN, o_col = C::O_COL + qt * HD;
+    uint8_t* prow = sP + qt * C::P_BYTES + row * 128;
+    float m_ref = -INFINITY, l = 0.0f;
+    bool ok = true;
+    for (int j = 0; j < T && ok; ++j) {
+      const uint32_t ph = j & 1;
+      const int kb = k_begin + j * BN;
+      ok = wait_bar(&s_full[qt], ph, status, abort_flag);
+      __syncwarp();
+      if (!__all_sync(0xffffffffu, ok)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float v[BN];
+#pragma unroll
+      for (int c = 0; c < BN; c += 64) tmem_ld64w(trow + s_col + c, v + c);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[qt]);
+      const bool full = __all_sync(0xffffffffu, (kb + BN - 1 <= row_pos) && (kb + BN <= k_end));
+      if (!full) {
+#pragma unroll
+        for (int i = 0; i < BN; ++i) {
+          const int key = kb + i;
+          if (!(key <= row_pos && key < k_end)) v[i] = -INFINITY;
         }
       }
-      if (ok) {
-        const uint16_t* src = pool + static_cast<int64_t>(phys) * blk_elems +
-                              (static_cast<int64_t>(g) * 16 + (key & 15)) * HD + c * 8;
-        cp_async16(smem_u32(dk + off), src);
-        cp_async16(smem_u32(dv + off), src + v_off);
-      } else {
-        *reinterpret_cast<uint4*>(dk + off) = make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4*>(dv + off) = make_uint4(0, 0, 0, 0);
+      float mx[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx[i] = v[i];
+#pragma unroll
+      for (int i = 8; i < BN; ++i) mx[i & 7] = fmaxf(mx[i & 7], v[i]);
+      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * scale_log2;
+      const float m_new = fmaxf(m_ref, tmax);
+      const bool need = m_new > m_ref + 8.0f;
+      // P(j-1) V(j-1) must be done before O is rebased or P is overwritten
+      if (j > 0) {
+        ok = wait_bar(&p_free[qt], (j - 1) & 1, status, abort_flag);
+        __syncwarp();
+        if (!__all_sync(0xffffffffu, ok)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
       }
-    }
-    cp_async_commit();
-  };
-
-  const int n_tiles = k_end > k_begin ? (k_end - k_begin + kKeys - 1) / kKeys : 0;
-  uint32_t qf[HD / 16][4];
-  if (n_tiles > 0) load_tile(k_begin, 0);
-  cp_async_wait<0>();  // (the Q tile is complete once the first K/V group is)
-  if (n_tiles > 0) {
-    // not all of tile 0 may be complete: wait_group 0 above waited for all groups
-  }
-  __syncthreads();
+      if (__any_sync(0xffffffffu, need)) {
+        if (j > 0) {
+          const float alpha = need ? ex2(m_ref - m_new) : 1.0f;
+#pragma unroll 1
+          for (int c = 0; c < HD; c += 32) {
+            float o[32];
+            tmem_ld32w(trow + o_col + c, o);
 #pragma unroll
-  for (int kk = 0; kk < HD / 16; ++kk) {
-    const int r = warp * 16 + (lane & 15);
-    const int c = kk * 2 + (lane >> 4);
-    ldsm_x4(smem_u32(sQ + r * HD + swz(r, c) * 8), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
-  }
-
-  for (int t = 0; t < n_tiles; ++t) {
-    const int buf = t & 1;
-    const int kb = k_begin + t * kKeys;
-    if (t + 1 < n_tiles) {
-      load_tile(kb + kKeys, buf ^ 1);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    __syncthreads();
-    const uint16_t* tk = sK + buf * kKeys * HD;
-    const uint16_t* tv = sV + buf * kKeys * HD;
-
-    float s[8][4];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.0f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int key = np * 16 + (lane & 7) + ((lane >> 4) << 3);
-        const int c = kk * 2 + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(smem_u32(tk + key * HD + swz(key, c) * 8), b0, b1, b2, b3);
-        mma_16816<F16>(s[2 * np], qf[kk], b0, b1);
-        mma_16816<F16>(s[2 * np + 1], qf[kk], b2, b3);
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32w(trow + o_col + c, o);
+          }
+          l *= alpha;
+        }
+        if (need) m_ref = m_new;
       }
-    }
-    // mask, scale, running max
-    float tmA = -INFINITY, tmB = -INFINITY;
+      const float nbase = m_ref == -INFINITY ? 0.0f : -m_ref;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+      for (int u = 0; u < BN / 8; ++u) {
+        uint32_t pk[4];
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int key = kb + j * 8 + 2 * (lane & 3) + e;
-        const bool va = key <= posA && key < k_end;
-        const bool vb = key <= posB && key < k_end;
-        s[j][e] = va ? s[j][e] * scale_log2 : -INFINITY;
-        s[j][2 + e] = vb ? s[j][2 + e] * scale_log2 : -INFINITY;
-        tmA = fmaxf(tmA, s[j][e]);
-        tmB = fmaxf(tmB, s[j][2 + e]);
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = ex2(fmaf(v[8 * u + 2 * e], scale_log2, nbase));
+          const float p1 = ex2(fmaf(v[8 * u + 2 * e + 1], scale_log2, nbase));
+          ls[e] += p0 + p1;
+          pk[e] = pack2<F16>(p0, p1);
+        }
+        // keys [8u, 8u+8) of this row in the swizzled K-major P tile
+        uint8_t* slice = prow + (u >> 3) * (C::BM * 128);
+        *reinterpret_cast<uint4*>(slice + (((u & 7) ^ (row & 7)) << 4)) =
+            make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
+      l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+      fence_async_smem();  // P visible to the tensor core
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[qt]);
     }
-#pragma unroll
-    for (int o2 = 1; o2 <= 2; o2 <<= 1) {
-      tmA = fmaxf(tmA, __shfl_xor_sync(0xffffffffu, tmA, o2));
-      tmB = fmaxf(tmB, __shfl_xor_sync(0xffffffffu, tmB, o2));
+    // ---- epilogue: O / l ----
+    bool have_o = false;
+    if (ok && T > 0) {
+      ok = wait_bar(&p_free[qt], (T - 1) & 1, status, abort_flag);
+      __syncwarp();
+      have_o = __all_sync(0xffffffffu, ok);
+      tc_fence_after();
     }
-    const float nmA = fmaxf(mA, tmA), nmB = fmaxf(mB, tmB);
-    const float baseA = nmA == -INFINITY ? 0.0f : nmA;
-    const float baseB = nmB == -INFINITY ? 0.0f : nmB;
-    const float alA = exp2f(mA - baseA), alB = exp2f(mB - baseB);
-    mA = nmA;
-    mB = nmB;
-    float rsA = 0.0f, rsB = 0.0f;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      s[j][0] = exp2f(s[j][0] - baseA);
-      s[j][1] = exp2f(s[j][1] - baseA);
-      s[j][2] = exp2f(s[j][2] - baseB);
-      s[j][3] = exp2f(s[j][3] - baseB);
-      rsA += s[j][0] + s[j][1];
-      rsB += s[j][2] + s[j][3];
-    }
-    lA = lA * alA + rsA;
-    lB = lB * alB + rsB;
-#pragma unroll
-    for (int j = 0; j < HD / 8; ++j) {
-      o[j][0] *= alA;
-      o[j][1] *= alA;
-      o[j][2] *= alB;
-      o[j][3] *= alB;
-    }
-    // O += P V
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t a[4];
-      a[0] = pack2<F16>(s[2 * kk][0], s[2 * kk][1]);
-      a[1] = pack2<F16>(s[2 * kk][2], s[2 * kk][3]);
-      a[2] = pack2<F16>(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-      a[3] = pack2<F16>(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-      for (int dp = 0; dp < HD / 16; ++dp) {
-        const int key = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
-        const int c = dp * 2 + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(smem_u32(tv + key * HD + swz(key, c) * 8), b0, b1, b2, b3);
-        mma_16816<F16>(o[2 * dp], a, b0, b1);
-        mma_16816<F16>(o[2 * dp + 1], a, b2, b3);
-      }
-    }
-    __syncthreads();
-  }
-
-#pragma unroll
-  for (int o2 = 1; o2 <= 2; o2 <<= 1) {
-    lA += __shfl_xor_sync(0xffffffffu, lA, o2);
-    lB += __shfl_xor_sync(0xffffffffu, lB, o2);
-  }
-  const float invA = lA > 0.0f ? 1.0f / lA : 0.0f;
-  const float invB = lB > 0.0f ? 1.0f / lB : 0.0f;
-  const int col0 = 2 * (lane & 3);
-#pragma unroll
-  for (int half = 0; half < 2; ++half) {
-    const int rr = half ? rowB : rowA;
-    if (rr >= R) continue;
-    const float inv = half ? invB : invA;
+    const float o_scale = l > 0.0f ? 1.0f / l : 0.0f;
     const int t = rr / group, h = g * group + rr % group;
     const int64_t orow = static_cast<int64_t>(t) * hq + h;
-    if (n_splits == 1) {
-      uint16_t* dst = out + orow * HD;
 #pragma unroll
-      for (int j = 0; j < HD / 8; ++j)
-        *reinterpret_cast<uint32_t*>(dst + j * 8 + col0) =
-            pack2<true>(o[j][2 * half] * inv, o[j][2 * half + 1] * inv);
-    } else {
-      float* dst = part_o + (static_cast<int64_t>(split) * n * hq + orow) * HD;
+    for (int c = 0; c < HD; c += 64) {
+      float o[64];
+      if (have_o) {
+        tmem_ld64w(trow + o_col + c, o);
+      } else {
 #pragma unroll
-      for (int j = 0; j < HD / 8; ++j)
-        *reinterpret_cast<float2*>(dst + j * 8 + col0) =
-            make_float2(o[j][2 * half] * inv, o[j][2 * half + 1] * inv);
-      if ((lane & 3) == 0) {
-        const float l = half ? lB : lA, m = half ? mB : mA;
-        part_lse[static_cast<int64_t>(split) * n * hq + orow] =
-            l > 0.0f ? m + log2f(l) : -INFINITY;
+        for (int i = 0; i < 64; ++i) o[i] = 0.0f;
+      }
+      if (rr < R) {
+        if (n_splits == 1) {
+          uint4* dst = reinterpret_cast<uint4*>(out + orow * HD + c);
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            dst[u] = make_uint4(pack2<true>(o[8 * u] * o_scale, o[8 * u + 1] * o_scale),
+                                pack2<true>(o[8 * u + 2] * o_scale, o[8 * u + 3] * o_scale),
+                                pack2<true>(o[8 * u + 4] * o_scale, o[8 * u + 5] * o_scale),
+                                pack2<true>(o[8 * u + 6] * o_scale, o[8 * u + 7] * o_scale));
+        } else {
+          float4* dst = reinterpret_cast<float4*>(
+              part_o + (static_cast<int64_t>(split) * n * hq + orow) * HD + c);
+#pragma unroll
+          for (int u = 0; u < 16; ++u)
+            dst[u] = make_float4(o[4 * u] * o_scale, o[4 * u + 1] * o_scale, o[4 * u + 2] * o_scale,
+                                 o[4 * u + 3] * o_scale);
+        }
       }
     }
+    if (rr < R && n_splits > 1)
+      part_lse[static_cast<int64_t>(split) * n * hq + orow] = l > 0.0f ? m_ref + log2f(l) : -INFINITY;
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 8) {
+    __syncwarp();
+    tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
 
@@ -292,28 +501,61 @@ __global__ void attn_combine_kernel(const float* __restrict__ part_o,
     *reinterpret_cast<uint32_t*>(dst + j) = pack2<true>(acc[j] * inv, acc[j + 1] * inv);
 }
 
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                              const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                              const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(p);
+  });
+  return fn;
+}
+
+// The pool as a 2-D tensor of 16-bit elements: [pool_blocks * 2 * hkv * 16 rows][hd],
+// read in boxes of 16 rows x 64 columns with 128-byte swizzle.
+bool make_pool_map(CUtensorMap* map, const void* pool, int64_t pool_blocks, int hkv, int hd) {
+  EncodeFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(hd), static_cast<cuuint64_t>(pool_blocks) * 2 * hkv * 16};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(hd) * 2};
+  cuuint32_t box[2] = {64, 16};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<void*>(pool), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int HD, bool F16>
 cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
-                      const int32_t* table, int64_t n_logical, const void* pool,
+                      const int32_t* table, int64_t n_logical, const CUtensorMap& map,
                       int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
                       int n_splits, int keys_per_split, int32_t* status, cudaStream_t st) {
-  constexpr int SMEM = (kRows + 4 * kKeys) * HD * 2;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, F16>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  using C = AttnCfg<HD>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(attn_tc_kernel<HD, F16>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
   const int group = hq / hkv;
   const int64_t R = n * group;
-  dim3 grid(static_cast<unsigned>((R + kRows - 1) / kRows), static_cast<unsigned>(hkv),
+  dim3 grid(static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta), static_cast<unsigned>(hkv),
             static_cast<unsigned>(n_splits));
-  const float scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
-  attn_kernel<HD, F16><<<grid, 128, SMEM, st>>>(
-      q, pos, static_cast<int>(n), hq, hkv, table, n_logical,
-      static_cast<const uint16_t*>(pool), pool_blocks, out, part_o, part_lse, keys_per_split,
-      n_splits, scale_log2, status);
+  const float scale_log2 =
+      static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
+  attn_tc_kernel<HD, F16><<<grid, 320, C::SMEM, st>>>(
+      q, pos, static_cast<int>(n), hq, hkv, table, n_logical, map, pool_blocks, out, part_o,
+      part_lse, keys_per_split, n_splits, scale_log2, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || n_splits == 1) return e;
   const int64_t rows = n * hq;
@@ -326,9 +568,9 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
 
 void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int num_sms,
                      int* n_splits, int* keys_per_split) {
-  const int64_t ctas = ((n * (hq / hkv) + kRows - 1) / kRows) * hkv;
+  const int64_t ctas = ((n * (hq / hkv) + kRowsPerCta - 1) / kRowsPerCta) * hkv;
   int s = 1;
-  const int64_t target = 2LL * num_sms;
+  const int64_t target = num_sms;  // one CTA per SM (shared memory bound)
   if (ctas < target && max_keys > 1024) {
     s = static_cast<int>((target + ctas - 1) / ctas);
     const int64_t max_s = (max_keys + 511) / 512;  // at least 512 keys per split
@@ -337,8 +579,8 @@ void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int n
     if (s < 1) s = 1;
   }
   int64_t per = (max_keys + s - 1) / s;
-  per = (per + kKeys - 1) / kKeys * kKeys;
-  if (per < kKeys) per = kKeys;
+  per = (per + 127) / 128 * 128;  // whole key tiles of either head size
+  if (per < 128) per = 128;
   *n_splits = s;
   *keys_per_split = static_cast<int>(per);
 }
@@ -358,20 +600,22 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   attention_split(n, hq, hkv, max_keys, num_sms, &s, &per);
   if (s > 1 && (scratch == nullptr || scratch_bytes < attention_scratch_bytes(n, hq, hd, s))) {
     s = 1;
-    per = static_cast<int>((max_keys + kKeys - 1) / kKeys * kKeys);
+    per = static_cast<int>((max_keys + 127) / 128 * 128);
   }
+  CUtensorMap map;
+  if (!make_pool_map(&map, pool, pool_blocks, hkv, hd)) return cudaErrorInvalidValue;
   float* part_o = static_cast<float*>(scratch);
   float* part_lse = s > 1 ? part_o + static_cast<int64_t>(s) * n * hq * hd : nullptr;
   const bool f16 = kv_dtype == 1;
   if (hd == 64)
-    return f16 ? launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
+    return f16 ? launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
                                      part_o, part_lse, s, per, status, st)
-               : launch_hd<64, false>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks,
+               : launch_hd<64, false>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
                                       out, part_o, part_lse, s, per, status, st);
   if (hd == 128)
-    return f16 ? launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks,
+    return f16 ? launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
                                       out, part_o, part_lse, s, per, status, st)
-               : launch_hd<128, false>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks,
+               : launch_hd<128, false>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
                                        out, part_o, part_lse, s, per, status, st);
   return cudaErrorInvalidValue;
 }

@@ -234,11 +234,11 @@ __global__ void gather_blocks_kernel(const uint4* __restrict__ pool, const int32
 }
 
 __global__ void poison_blocks_kernel(uint4* __restrict__ pool, const int32_t* __restrict__ phys,
-                                     int64_t chunks_per_block) {
+                                     int64_t chunks_per_block, uint32_t pattern2) {
   const int64_t b = blockIdx.x;
   uint4* d = pool + static_cast<int64_t>(phys[b]) * chunks_per_block;
-  const uint4 nan = make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu);
-  for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = nan;
+  const uint4 v = make_uint4(pattern2, pattern2, pattern2, pattern2);
+  for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = v;
 }
 
 }  // namespace
@@ -292,10 +292,14 @@ cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t 
 }
 
 cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
-                                 cudaStream_t st) {
+                                 int32_t kv_dtype, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
+  // the largest finite value of the KV type: finite, so a masked key (weight 0)
+  // contributes exactly 0, and far outside any real K/V, so a read of a block
+  // before its restore lands shows up in the results
+  const uint32_t v16 = kv_dtype == 1 ? 0x7BFFu : 0x7F7Fu;
   poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), phys,
-                                                                  block_bytes / 16);
+                                                                  block_bytes / 16, v16 | (v16 << 16));
   return cudaGetLastError();
 }
 

@@ -67,8 +67,8 @@ cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float 
 // Copies blocks phys[i] (block_bytes each) of the pool to dst + i*block_bytes.
 cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t n,
                                  int64_t block_bytes, void* dst, cudaStream_t st);
-// Fills blocks phys[i] with 0xFF bytes (NaN in bf16 and fp16).
+// Fills blocks phys[i] with the largest finite value of the KV type.
 cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
-                                 cudaStream_t st);
+                                 int32_t kv_dtype, cudaStream_t st);
 
 }  // namespace mzc

@@ -340,7 +340,8 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
 }
 
 // Moves `moves` (COPY eviction) out to the pinned store, then poisons the
-// freed physical blocks so that a missing wait shows up as NaN.
+// freed physical blocks (largest finite KV value) so that a read that does
+// not wait for its restore shows up in the results.
 mzc_status copy_out(mzc_ctx* ctx, const std::vector<mzc::EvictMove>& moves) {
   int64_t total = 0;
   for (auto& mv : moves) {
@@ -357,7 +358,7 @@ mzc_status copy_out(mzc_ctx* ctx, const std::vector<mzc::EvictMove>& moves) {
                        cudaMemcpyDeviceToHost, ctx->cs));
     at += nb;
   }
-  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, total, ctx->block_bytes, ctx->cs));
+  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, total, ctx->block_bytes, ctx->shape.kv_dtype, ctx->cs));
   CK(cudaStreamSynchronize(ctx->cs));
   return MZC_OK;
 }
@@ -366,7 +367,7 @@ mzc_status poison(mzc_ctx* ctx, const std::vector<int32_t>& phys) {
   if (phys.empty()) return MZC_OK;
   std::memcpy(ctx->h_list, phys.data(), phys.size() * 4);
   CK(cudaMemcpyAsync(ctx->d_list, ctx->h_list, phys.size() * 4, cudaMemcpyHostToDevice, ctx->cs));
-  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, static_cast<int64_t>(phys.size()), ctx->block_bytes, ctx->cs));
+  CK(mzc::launch_poison_blocks(ctx->d_pool, ctx->d_list, static_cast<int64_t>(phys.size()), ctx->block_bytes, ctx->shape.kv_dtype, ctx->cs));
   CK(cudaStreamSynchronize(ctx->cs));
   return MZC_OK;
 }
@@ -1041,7 +1042,12 @@ static int sm_count() {
   return n;
 }
 
-#define KCK(expr) return (expr) == cudaSuccess ? MZC_OK : MZC_ERR_CUDA
+static mzc_status kernel_status(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return MZC_OK;
+  g_create_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return MZC_ERR_CUDA;
+}
+#define KCK(expr) return kernel_status((expr), __func__)
 
 mzc_status mzc_k_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
                          uint16_t* y, void* stream) {
