@@ -39,6 +39,10 @@ struct GemmCfg {
 
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)); }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CUtensorMap tma,
                                                       const __grid_constant__ CUtensorMap tmw,
@@ -185,6 +189,248 @@ __global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CU
   }
 }
 
+// Persistent variant for M > 128: one CTA per SM walks 128 x BN tiles
+// (grouped order: a band of kBandN tiles of N down all of M, so a band of
+// weight tiles stays in L2 while the activations stream), with a
+// double-buffered TMEM accumulator so that the epilogue of tile i overlaps
+// the main loop of tile i+1.  Warp 0: TMA producer; warp 1: UMMA issuer
+// (and TMEM owner); warps 2-5: epilogue (warp w reads TMEM lanes
+// 32*(w%4)..+31).
+constexpr int kBandN = 4;
+
+template <int BN, int STAGES>
+struct PCfg {
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
+};
+
+__device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, int32_t* status,
+                                      volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      set_status(status, kStatusTimeout);
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int* mt, int* nt) {
+  const int band = tile / (num_m * kBandN);
+  const int width = min(kBandN, num_n - band * kBandN);
+  const int within = tile - band * num_m * kBandN;
+  *mt = within / width;
+  *nt = band * kBandN + within % width;
+}
+
+template <int BN, int STAGES, int EPI>
+__global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
+    const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw,
+    void* __restrict__ out, int m, int n, int k, int32_t* status) {
+  using C = PCfg<BN, STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* acc_full = empty + STAGES;  // [2]
+  uint64_t* acc_empty = acc_full + 2;   // [2]
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort;
+  volatile int* abort_flag = &s_abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_m = (m + BM - 1) / BM, num_n = (n + BN - 1) / BN;
+  const int tiles = num_m * num_n;
+  const int num_k = (k + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tma);
+    tma_prefetch_desc(&tmw);
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 4);  // one arrival per epilogue warp
+    }
+    fence_barrier_init();
+    s_abort = 0;
+  }
+  if (warp == 1) tmem_alloc(&s_tmem, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer over all tiles of this CTA ----
+      int it = 0;  // global k-block counter (ring position)
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x) {
+        int mt, nt;
+        tile_coords(tile, num_m, num_n, &mt, &nt);
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % STAGES;
+          if (it >= STAGES && !pwait(&empty[s], ((it / STAGES) - 1) & 1, status, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+          tma_load_2d(sA + s * C::A_BYTES, &tma, &full[s], kb * BK, mt * BM);
+          tma_load_2d(sB + s * C::B_BYTES, &tmw, &full[s], kb * BK, nt * BN);
+        }
+      }
+      // drain the last fill of every ring slot before shared memory is released
+      for (int i = it - STAGES < 0 ? 0 : it - STAGES; i < it; ++i)
+        pwait(&full[i % STAGES], (i / STAGES) & 1, status, abort_flag);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- UMMA issuer ----
+      constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+      int it = 0, local = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < tiles; tile += gridDim.x, ++local) {
+        const int a = local & 1;
+        // the epilogue has drained this accumulator (its use two tiles ago)
+        if (local >= 2 && !pwait(&acc_empty[a], ((local >> 1) - 1) & 1, status, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + a * BN;
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % STAGES;
+          if (!pwait(&full[s], (it / STAGES) & 1, status, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sA + s * C::A_BYTES));
+          const uint64_t bd = sdesc_k_sw128(smem_u32(sB + s * C::B_BYTES));
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            umma_f16(d, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+          umma_commit(&empty[s]);
+        }
+        if (ok) umma_commit(&acc_full[a]);
+      }
+    }
+  } else {
+    // ---- epilogue warps 2-5 ----
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    int local = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
+      const int a = local & 1;
+      bool ok = pwait(&acc_full[a], (local >> 1) & 1, status, abort_flag);
+      __syncwarp();
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      int mt, nt;
+      tile_coords(tile, num_m, num_n, &mt, &nt);
+      const int row = mt * BM + q * 32 + lane;
+      const uint32_t trow = tmem + a * BN + (static_cast<uint32_t>(q * 32) << 16);
+      const int n0 = nt * BN;
+      if constexpr (EPI == EPI_SWIGLU_BF16) {
+        const int nout = n / 2;
+#pragma unroll 1
+        for (int g = 0; g < BN / (2 * kSwigluGroup); ++g) {
+#pragma unroll 1
+          for (int c = 0; c < kSwigluGroup; c += 32) {
+            float vg[32], vu[32];
+            tmem_ld32w(trow + g * 2 * kSwigluGroup + c, vg);
+            tmem_ld32w(trow + g * 2 * kSwigluGroup + kSwigluGroup + c, vu);
+            const int col = n0 / 2 + g * kSwigluGroup + c;
+            if (row < m && col < nout) {
+              uint32_t pk[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i)
+                pk[i] = pack2<true>(silu_f(vg[2 * i]) * vu[2 * i], silu_f(vg[2 * i + 1]) * vu[2 * i + 1]);
+              uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + static_cast<size_t>(row) * nout + col);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32w(trow + c, v);
+          const int col = n0 + c;
+          if (row < m && col < n) {
+            const int cnt = min(32, n - col);  // n is a multiple of 16
+            if constexpr (EPI == EPI_STORE_BF16) {
+              uint32_t pk[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) pk[i] = pack2<true>(v[2 * i], v[2 * i + 1]);
+              uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + static_cast<size_t>(row) * n + col);
+#pragma unroll
+              for (int i = 0; i < 4; ++i)
+                if (i * 8 < cnt) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+            } else {
+              float4* o = reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<size_t>(row) * n + col);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                if (i * 4 < cnt) {
+                  float4 t = o[i];
+                  t.x += v[4 * i];
+                  t.y += v[4 * i + 1];
+                  t.z += v[4 * i + 2];
+                  t.w += v[4 * i + 3];
+                  o[i] = t;
+                }
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[a]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int BN, int STAGES, int EPI>
+cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void* out, int64_t m,
+                              int64_t n, int64_t k, int32_t* status, cudaStream_t st) {
+  using C = PCfg<BN, STAGES>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  static int sms = 0;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(gemm_persistent_kernel<BN, STAGES, EPI>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    int dev = 0;
+    if (attr_err == cudaSuccess) attr_err = cudaGetDevice(&dev);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  const int64_t tiles = ((m + BM - 1) / BM) * ((n + BN - 1) / BN);
+  const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
+  gemm_persistent_kernel<BN, STAGES, EPI><<<grid, 192, C::SMEM, st>>>(
+      ta, tw, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
+  return cudaGetLastError();
+}
+
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                               const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
                               const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
@@ -238,29 +484,39 @@ bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue) {
   (void)n;
+  if (m > 128) return 256;  // persistent 128 x 256 tiles
   if (epilogue == EPI_SWIGLU_BF16) return 128;
-  return m <= 128 ? 64 : 128;
+  return 64;
 }
 
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) {
-  return make_tmap_f16(&gw->box64, base, n, k, 64) && make_tmap_f16(&gw->box128, base, n, k, 128);
+  return make_tmap_f16(&gw->box64, base, n, k, 64) && make_tmap_f16(&gw->box128, base, n, k, 128) &&
+         make_tmap_f16(&gw->box256, base, n, k, 256);
 }
 
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
   if (m <= 0) return cudaSuccess;
-  const uint32_t bn = gemm_box_n(m, n, epilogue);
-  // the W tile the kernel expects (bn rows) is exactly the box of the map it gets
-  const CUtensorMap& tw = bn == 64 ? w.box64 : w.box128;
+  if (m > 128) {
+    // the W tile the kernel expects (256 rows) is exactly the box of the map it gets
+    switch (epilogue) {
+      case EPI_STORE_BF16:
+        return launch_persistent<256, 4, EPI_STORE_BF16>(ta, w.box256, out, m, n, k, status, st);
+      case EPI_ADD_F32:
+        return launch_persistent<256, 4, EPI_ADD_F32>(ta, w.box256, out, m, n, k, status, st);
+      case EPI_SWIGLU_BF16:
+        return launch_persistent<256, 4, EPI_SWIGLU_BF16>(ta, w.box256, out, m, n, k, status, st);
+      default:
+        return cudaErrorInvalidValue;
+    }
+  }
   switch (epilogue) {
     case EPI_STORE_BF16:
-      return bn == 64 ? launch_cfg<64, 4, EPI_STORE_BF16>(ta, tw, out, m, n, k, status, st)
-                      : launch_cfg<128, 3, EPI_STORE_BF16>(ta, tw, out, m, n, k, status, st);
+      return launch_cfg<64, 4, EPI_STORE_BF16>(ta, w.box64, out, m, n, k, status, st);
     case EPI_ADD_F32:
-      return bn == 64 ? launch_cfg<64, 4, EPI_ADD_F32>(ta, tw, out, m, n, k, status, st)
-                      : launch_cfg<128, 3, EPI_ADD_F32>(ta, tw, out, m, n, k, status, st);
+      return launch_cfg<64, 4, EPI_ADD_F32>(ta, w.box64, out, m, n, k, status, st);
     case EPI_SWIGLU_BF16:
-      return launch_cfg<128, 3, EPI_SWIGLU_BF16>(ta, tw, out, m, n, k, status, st);
+      return launch_cfg<128, 3, EPI_SWIGLU_BF16>(ta, w.box128, out, m, n, k, status, st);
     default:
       return cudaErrorInvalidValue;
   }

@@ -20,9 +20,9 @@ bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
                     uint32_t box_rows);
 
 // A weight operand W [n][k] with one tensor map per tile width the GEMM may
-// pick (box rows 64 and 128).
+// pick (box rows 64, 128 and 256).
 struct GemmWeight {
-  CUtensorMap box64, box128;
+  CUtensorMap box64, box128, box256;
 };
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 
