@@ -150,8 +150,7 @@ class Runner:
         self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device)
         self.t_create = time.time() - t
         t = time.time()
-        for a in range(0, sc["context"], max_rows - 1024):
-            m.mzc_prefill(self.c, self.ctx_tokens[a:a + max_rows - 1024])
+        m.mzc_prefill(self.c, self.ctx_tokens)  # long contexts run in causal chunks
         self.t_ctx = time.time() - t
         self.logits = np.empty(sh["vocab"], np.float32)
         self.N = sc["context"]
@@ -304,6 +303,8 @@ def main():
                     choices=["1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed", "3b_sweep"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-kernel-timing", action="store_true")
+    ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
+    ap.add_argument("--policies", default=None, help="comma list overriding the sweep's policies")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mzc":
         args.warmup = 3
@@ -313,6 +314,10 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     name = args.workload
     sc = _workload(name)
+    if args.fractions:
+        sc["fractions"] = tuple(float(x) for x in args.fractions.split(","))
+    if args.policies:
+        sc["policies"] = tuple(args.policies.split(","))
 
     if args.impl == "reference":
         run_reference(args, name, sc, rank)
@@ -443,16 +448,28 @@ def run_sweep(r, args, rank):
     pts = []
     for frac in r.sc["fractions"]:
         for pol in r.sc["policies"]:
-            vals = []
+            vals, comp, copy = [], [], []
+            m.mzc_set_kernel_timing(r.c, False)
             for i in range(args.warmup + args.steps):
+                if i == args.warmup:
+                    m.mzc_set_kernel_timing(r.c, True)
                 r.evict(pol, frac)
                 d, h, st, times = r.step()
                 if i >= args.warmup:
                     vals.append(d)
+                    comp.append(float(times[0]))
+                    copy.append(float(times[1]))
+            ks = {nm: round(m.mzc_kernel_stats(r.c, j).ms / args.steps, 3)
+                  for j, nm in enumerate(m.KERNEL_CLASS_NAMES)}
+            m.mzc_set_kernel_timing(r.c, False)
             pt = {"fraction": frac, "policy": pol, "ttft_ms": round(statistics.median(vals), 3),
                   "p10": round(float(np.percentile(vals, 10)), 3),
                   "p90": round(float(np.percentile(vals, 90)), 3),
-                  "recompute_rows": st.recompute_rows_last, "copied_bytes": st.bytes_h2d_last}
+                  "compute_stream_ms": round(statistics.median(comp), 3),
+                  "copy_stream_ms": round(statistics.median(copy), 3),
+                  "kernel_ms": ks,
+                  "recompute_rows": st.recompute_rows_last,
+                  "copied_bytes": st.bytes_h2d_last if pol != "recompute" else 0}
             pts.append(pt)
             print(json.dumps(pt), file=sys.stderr, flush=True)
     if rank == 0:
@@ -461,7 +478,7 @@ def run_sweep(r, args, rank):
             best.setdefault(p["fraction"], {})[p["policy"]] = p["ttft_ms"]
         print(json.dumps({"metric": METRIC, "workload": _describe("3b_sweep", r.sc),
                           "profile": {k: getattr(r.profile, k) for k, _ in r.profile._fields_},
-                          "sweep": best}), flush=True)
+                          "sweep": best, "points": pts}), flush=True)
 
 
 if __name__ == "__main__":

@@ -25,6 +25,7 @@
 // Long key ranges with few rows are split across CTAs (split-KV); each split
 // writes its normalised partial output and base-2 log-sum-exp, and a combine
 // kernel merges them.
+#include <algorithm>
 #include <cmath>
 #include <mutex>
 
@@ -570,13 +571,21 @@ void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int n
                      int* n_splits, int* keys_per_split) {
   const int64_t ctas = ((n * (hq / hkv) + kRowsPerCta - 1) / kRowsPerCta) * hkv;
   int s = 1;
-  const int64_t target = num_sms;  // one CTA per SM (shared memory bound)
-  if (ctas < target && max_keys > 1024) {
-    s = static_cast<int>((target + ctas - 1) / ctas);
-    const int64_t max_s = (max_keys + 511) / 512;  // at least 512 keys per split
-    if (s > max_s) s = static_cast<int>(max_s);
-    if (s > 64) s = 64;
-    if (s < 1) s = 1;
+  if (ctas < num_sms && max_keys > 1024) {
+    // one CTA per SM: pick the split count whose waves are fullest (ties -> more
+    // splits), with at least 512 keys per split
+    const int64_t max_s = std::min<int64_t>(64, (max_keys + 511) / 512);
+    double best = 0.0;
+    for (int64_t c = 1; c <= max_s; ++c) {
+      const int64_t total = ctas * c;
+      const int64_t waves = (total + num_sms - 1) / num_sms;
+      const double eff = static_cast<double>(total) / static_cast<double>(waves * num_sms);
+      if (eff >= best - 1e-9) {
+        best = eff;
+        s = static_cast<int>(c);
+      }
+      if (waves > 1 && eff < best) break;
+    }
   }
   int64_t per = (max_keys + s - 1) / s;
   per = (per + 127) / 128 * 128;  // whole key tiles of either head size

@@ -2,6 +2,7 @@
 // rotary embedding fused with the KV-block write, the LM-head GEMV, and the
 // block gather/poison used by eviction.  All global accesses are 16-byte
 // vectors along the contiguous dimension.
+#include <algorithm>
 #include <cstdio>
 
 #include "kernels.hpp"
@@ -225,6 +226,14 @@ __global__ void __launch_bounds__(256) lm_head_kernel(const float* __restrict__ 
   }
 }
 
+// dst[i] = src[i] for n 16-byte words; src may be mapped pinned host memory,
+// read over the host link by the SMs (no copy engine involved).
+__global__ void copy16_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst, int64_t n) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    dst[i] = src[i];
+}
+
 __global__ void gather_blocks_kernel(const uint4* __restrict__ pool, const int32_t* __restrict__ phys,
                                      int64_t chunks_per_block, uint4* __restrict__ dst) {
   const int64_t b = blockIdx.x;
@@ -280,6 +289,15 @@ cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float 
   const int grid = num_sms * 4;
   lm_head_kernel<<<grid, 256, static_cast<size_t>(d) * sizeof(float), st>>>(x_row, g, d, eps, w,
                                                                             vocab, logits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_copy16(const void* src, void* dst, int64_t bytes, cudaStream_t st) {
+  const int64_t n = (bytes + 15) / 16;
+  if (n <= 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((n + 255) / 256, 1024);
+  copy16_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(static_cast<const uint4*>(src),
+                                                                static_cast<uint4*>(dst), n);
   return cudaGetLastError();
 }
 

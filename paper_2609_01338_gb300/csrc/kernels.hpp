@@ -64,6 +64,9 @@ cudaError_t launch_attention_noalloc(const uint16_t* q, const int32_t* pos, int6
 cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float eps,
                            const uint16_t* w, int64_t vocab, float* logits, int num_sms,
                            cudaStream_t st);
+// Copies bytes (rounded up to 16) from src to dst with a kernel; src may be
+// mapped pinned host memory (read by the SMs, not by a copy engine).
+cudaError_t launch_copy16(const void* src, void* dst, int64_t bytes, cudaStream_t st);
 // Copies blocks phys[i] (block_bytes each) of the pool to dst + i*block_bytes.
 cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t n,
                                  int64_t block_bytes, void* dst, cudaStream_t st);

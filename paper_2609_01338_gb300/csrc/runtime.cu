@@ -76,6 +76,7 @@ struct mzc_ctx {
   CUtensorMap tm_h, tm_attn, tm_act;
   uint8_t* d_meta = nullptr;  // tokens | pos | block tables
   uint8_t* h_meta = nullptr;
+  uint8_t* h_meta_dev = nullptr;  // device view of the mapped h_meta
   size_t meta_bytes = 0;
   float* d_logits = nullptr;
   float* h_logits = nullptr;
@@ -316,9 +317,12 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   if (!ok) return ctx->fail(MZC_ERR_CUDA, "cuTensorMapEncodeTiled failed");
 
   // ---- per-call metadata, logits, scratch, status ----
-  ctx->meta_bytes = static_cast<size_t>(R) * 8 + static_cast<size_t>(L) * ctx->nblk * 4;
+  ctx->meta_bytes = align_up(static_cast<size_t>(s.max_ctx) * 8 + static_cast<size_t>(L) * ctx->nblk * 4, 16);
   CK(cudaMalloc(&ctx->d_meta, ctx->meta_bytes));
-  CK(cudaHostAlloc(&ctx->h_meta, ctx->meta_bytes, cudaHostAllocDefault));
+  // mapped: the prefill pulls its metadata in with a kernel, so the upload never
+  // queues behind restore copies on the host-to-device copy engine
+  CK(cudaHostAlloc(&ctx->h_meta, ctx->meta_bytes, cudaHostAllocMapped));
+  CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&ctx->h_meta_dev), ctx->h_meta, 0));
   CK(cudaMalloc(&ctx->d_logits, V * 4));
   CK(cudaHostAlloc(&ctx->h_logits, V * 4, cudaHostAllocDefault));
   int64_t scratch = 0;
@@ -466,7 +470,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
   } while (0)
   CKP(cudaEventRecord(ctx->ev_t0, cs));
   ctx->ttft_from_copy = ctx->restore_issued;
-  CKP(cudaMemcpyAsync(ctx->d_meta, ctx->h_meta, mbytes, cudaMemcpyHostToDevice, cs));
+  CKP(mzc::launch_copy16(ctx->h_meta_dev, ctx->d_meta, static_cast<int64_t>(mbytes), cs));
   if (!ctx->opt.overlap && ctx->restore_issued) CKP(cudaStreamWaitEvent(cs, ctx->ev_c1, 0));
   ctx->ev_next = 0;
   ctx->kev.clear();
@@ -482,67 +486,85 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     *fl = 4.0 * hd * hq * pairs;
     *by = 2.0 * hkv * hd * kvb * mx + 2.0 * nr * hq * hd * 2.0;
   };
-  const double dd = static_cast<double>(d), R = static_cast<double>(rows);
-  CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
-    return mzc::launch_embed(dtok, rows, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
-  }));
-  const int64_t max_keys = n > 0 ? P.prompt_end : P.rec_end;
-  auto gemm = [&](const CUtensorMap& ta, const mzc::GemmWeight& w, void* out, int64_t N, int64_t K, int epi) {
-    const double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
-    return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
-                   [&] { return mzc::launch_gemm(ta, w, out, rows, N, K, epi, ctx->d_status, cs); });
-  };
-  auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab) {
-    double fl, by;
-    attn_work(r0, nr, &fl, &by);
-    int sp = 1, per = 0;
-    mzc::attention_split(nr, s.n_q_heads, s.n_kv_heads, mk, ctx->num_sms, &sp, &per);
-    const bool fits = sp == 1 || ctx->scratch_bytes >= mzc::attention_scratch_bytes(nr, s.n_q_heads, s.head_dim, sp);
-    return klaunch(ctx, MZC_K_ATTENTION, fl, by, (sp > 1 && fits) ? 2 : 1, [&] {
-      return mzc::launch_attention(ctx->d_q + r0 * hq * hd, dpos + r0, nr, s.n_q_heads, s.n_kv_heads,
-                                   s.head_dim, ltab, ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(),
-                                   s.kv_dtype, ctx->d_attn + r0 * hq * hd, ctx->d_scratch,
-                                   ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs);
-    });
-  };
-  const double norm_bytes = R * dd * 6.0 + dd * 4.0;
-  const double rope_bytes = R * (hq + 2.0 * hkv) * hd * 4.0 + R * hd * 4.0;
-  for (int64_t l = 0; l < L; ++l) {
-    const LayerDev& W = ctx->layers[l];
-    const int32_t* ltab = dtab + l * ctx->nblk;
-    if (P.w_wait[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_w[l], 0));
-    CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-      return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, rows, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+  const double dd = static_cast<double>(d);
+  // Rows run in causal chunks of at most max_rows: every row of a chunk
+  // attends only to positions written by this chunk or an earlier one, and a
+  // chunk goes through all layers before the next starts.  The prompt rows
+  // come last, so the last chunk holds the row whose logits are returned.
+  const int64_t chunk = ctx->max_rows;
+  int64_t last_rows = 0;
+  for (int64_t c0 = 0; c0 < rows; c0 += chunk) {
+    const int64_t c1 = std::min(rows, c0 + chunk), cr = c1 - c0;
+    const int64_t rec_hi = std::min(c1, nrec);          // recompute rows [c0, rec_hi)
+    const int64_t n_rec_c = std::max<int64_t>(0, rec_hi - c0);
+    const int64_t n_prm_c = cr - n_rec_c;                // prompt rows of this chunk
+    const int64_t max_keys = static_cast<int64_t>(hpos[c1 - 1]) + 1;
+    const double R = static_cast<double>(cr);
+    int32_t* ctok = dtok + c0;
+    int32_t* cpos = dpos + c0;
+    CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
+      return mzc::launch_embed(ctok, cr, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
     }));
-    CKP(gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
-    if (P.kv_wait_write[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
-    CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
-      return mzc::launch_rope_kv_write(ctx->d_qkv, dpos, rows, s.n_q_heads, s.n_kv_heads, s.head_dim,
-                                       ctx->d_cos, ctx->d_sin, ltab, ctx->nblk, ctx->d_pool,
-                                       ctx->st.pool_blocks(), s.kv_dtype, ctx->d_q, ctx->d_status, cs);
-    }));
-    const bool split_launch = nrec > 0 && n > 0 && P.kv_wait_prompt[l] && !P.kv_wait_rec[l];
-    if (split_launch) {
-      // recompute rows read only resident keys: they run before the copy lands
-      CKP(attention(0, nrec, P.rec_end, ltab));
-      CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
-      CKP(attention(nrec, n, max_keys, ltab));
-    } else {
-      if (P.kv_wait_prompt[l] || P.kv_wait_rec[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
-      CKP(attention(0, rows, max_keys, ltab));
+    auto gemm = [&](const CUtensorMap& ta, const mzc::GemmWeight& w, void* out, int64_t N, int64_t K, int epi) {
+      const double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
+      return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
+                     [&] { return mzc::launch_gemm(ta, w, out, cr, N, K, epi, ctx->d_status, cs); });
+    };
+    // attention of chunk rows [r0, r0 + nr) (r0 relative to the chunk)
+    auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab) {
+      double fl, by;
+      attn_work(c0 + r0, nr, &fl, &by);
+      int sp = 1, per = 0;
+      mzc::attention_split(nr, s.n_q_heads, s.n_kv_heads, mk, ctx->num_sms, &sp, &per);
+      const bool fits = sp == 1 || ctx->scratch_bytes >= mzc::attention_scratch_bytes(nr, s.n_q_heads, s.head_dim, sp);
+      return klaunch(ctx, MZC_K_ATTENTION, fl, by, (sp > 1 && fits) ? 2 : 1, [&] {
+        return mzc::launch_attention(ctx->d_q + r0 * hq * hd, cpos + r0, nr, s.n_q_heads, s.n_kv_heads,
+                                     s.head_dim, ltab, ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(),
+                                     s.kv_dtype, ctx->d_attn + r0 * hq * hd, ctx->d_scratch,
+                                     ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs);
+      });
+    };
+    const double norm_bytes = R * dd * 6.0 + dd * 4.0;
+    const double rope_bytes = R * (hq + 2.0 * hkv) * hd * 4.0 + R * hd * 4.0;
+    for (int64_t l = 0; l < L; ++l) {
+      const LayerDev& W = ctx->layers[l];
+      const int32_t* ltab = dtab + l * ctx->nblk;
+      if (P.w_wait[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_w[l], 0));
+      CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+        return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+      }));
+      CKP(gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
+      if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+      CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
+        return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
+                                         ctx->d_cos, ctx->d_sin, ltab, ctx->nblk, ctx->d_pool,
+                                         ctx->st.pool_blocks(), s.kv_dtype, ctx->d_q, ctx->d_status, cs);
+      }));
+      const bool wait_rec = n_rec_c > 0 && P.kv_wait_rec[l];
+      const bool wait_prm = n_prm_c > 0 && P.kv_wait_prompt[l];
+      if (n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
+        // recompute rows read only resident keys: they run before the copy lands
+        CKP(attention(0, n_rec_c, static_cast<int64_t>(hpos[c0 + n_rec_c - 1]) + 1, ltab));
+        CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+        CKP(attention(n_rec_c, n_prm_c, max_keys, ltab));
+      } else {
+        if (wait_rec || wait_prm) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+        CKP(attention(0, cr, max_keys, ltab));
+      }
+      CKP(gemm(ctx->tm_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
+      CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+        return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+      }));
+      CKP(gemm(ctx->tm_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
+      CKP(gemm(ctx->tm_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
     }
-    CKP(gemm(ctx->tm_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
-    CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-      return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, rows, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
-    }));
-    CKP(gemm(ctx->tm_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
-    CKP(gemm(ctx->tm_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
+    last_rows = cr;
   }
   ctx->lm_timed = false;
   if (n > 0 && logits_out) {
     CKP(cudaEventRecord(ctx->ev_l0, cs));
     CKP(klaunch(ctx, MZC_K_LM_HEAD, 2.0 * s.vocab * dd, s.vocab * dd * 2.0 + s.vocab * 4.0 + dd * 8.0, 1, [&] {
-      return mzc::launch_lm_head(ctx->d_x + (rows - 1) * d, ctx->d_fnorm, static_cast<int32_t>(d), s.rms_eps,
+      return mzc::launch_lm_head(ctx->d_x + (last_rows - 1) * d, ctx->d_fnorm, static_cast<int32_t>(d), s.rms_eps,
                                  ctx->d_lm, s.vocab, ctx->d_logits, ctx->num_sms, cs);
     }));
     CKP(cudaEventRecord(ctx->ev_l1, cs));

@@ -219,3 +219,17 @@ def test_mid_hybrid_restore(mid):
     assert np.max(np.abs(lg - mid["lg_ref"])) < LOGIT_TOL
     _check_kv(mid, c, 637)
     m.mzc_destroy(c)
+
+
+def test_row_sets_beyond_max_rows_run_in_causal_chunks(tiny):
+    """max_rows=100: the 512-token context and the 288-row recompute + prompt
+    set both run in chunks of 100 rows; logits and KV still match the oracle."""
+    c = _new(tiny, max_rows=100)
+    m.mzc_prefill(c, tiny["ctx"])
+    m.mzc_evict(c, 0, 2, 256, 512, m.MZC_DROP)
+    m.mzc_recompute_tail(c, 256, 256)
+    lg = _logits(tiny, c, tiny["prm"])
+    assert np.max(np.abs(lg - tiny["lg_ref"])) < LOGIT_TOL
+    _check_kv(tiny, c, 544)
+    assert m.mzc_stats(c).rows_last == 288
+    m.mzc_destroy(c)
