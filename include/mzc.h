@@ -24,6 +24,9 @@
  *     ctxs share nothing.
  *   - Token ranges are in absolute positions of the context; KV blocks are
  *     block_tokens (16) consecutive positions of one layer.
+ *   - KV storage: K/V values are rounded to the shape's kv_dtype (bf16 or
+ *     fp16) and held in fp16 encoding in either case (every normal-range bf16
+ *     value is exactly an fp16 value), so attention reads one format.
  */
 #ifndef MZC_H
 #define MZC_H
@@ -95,14 +98,20 @@ typedef struct {
   const mzc_layer_weights *layers; /* [n_layers] */
 } mzc_weights;
 
-/* Per-unit restore rates (the paper's offline profiling, Sec. 4.3: each
- * path's time per unit, assumed linear in the number of units). */
+/* Per-unit costs of the two restore paths, measured on the device (the
+ * paper's offline profiling, Sec. 4.3: each path's time per unit).  Copy:
+ * bytes over the host link.  Recompute: the per-layer time of the fused
+ * (recomputed + prompt) rows, from measured pieces that the split planner
+ * interpolates. */
 typedef struct {
-  double h2d_gbs;     /* pinned host -> HBM copy rate, GB/s */
-  double hbm_gbs;     /* HBM streaming rate, GB/s (weight-bound small-M GEMMs) */
-  double gemm_tflops; /* BF16 GEMM rate at recompute sizes, TFLOP/s */
-  double attn_tflops; /* prefill attention rate, TFLOP/s */
-  double launch_us;   /* fixed cost per layer of one prefill call, microseconds */
+  double h2d_gbs;            /* pinned host -> HBM copy rate, GB/s */
+  double gemm_us_128;        /* one layer's four projections at 128 rows, us */
+  double gemm_us_512;        /* ... at 512 rows, us */
+  double gemm_us_2048;       /* ... at 2048 rows, us */
+  double attn_tflops;        /* attention of recompute-like rows (causal, mid-context), TFLOP/s */
+  double attn_prompt_tflops; /* attention of prompt rows over the whole context, TFLOP/s */
+  double row_ns;             /* per row and layer: norms and rotary/KV write, ns */
+  double layer_us;           /* per layer fixed cost (launch gaps), us */
 } mzc_profile;
 
 typedef struct {
@@ -136,9 +145,11 @@ mzc_status mzc_destroy(mzc_ctx *ctx);
  * for that layer's restore copies (zero-wait, Sec. 4.4).  Writes the fp32
  * logits of the last new token to logits_out[vocab] (host), or nothing when
  * logits_out is NULL or n == 0.  Returns after the logits are on the host.
+ * Row sets larger than options->max_rows run in causal chunks of max_rows
+ * rows (a chunk goes through all layers before the next).
  * Errors: MZC_ERR_STATE if any block the rows attend to is SWAPPED without a
  * restore in flight, or DROPPED without a pending recompute; MZC_ERR_OOM if
- * the rows exceed max_rows or the pool is full; MZC_ERR_RANGE past max_ctx. */
+ * the pool is full; MZC_ERR_RANGE past max_ctx. */
 mzc_status mzc_prefill(mzc_ctx *ctx, const int32_t *tokens, int64_t n, float *logits_out);
 
 /* Evicts layers [layer_begin, layer_end) x positions [tok_begin, tok_end).
@@ -177,10 +188,12 @@ mzc_status mzc_set_policy(mzc_ctx *ctx, int32_t policy, const mzc_profile *profi
 
 /* Hybrid split (pure host arithmetic): for an evicted tail [p, n_ctx) and a
  * prompt of n_prompt tokens, the block-aligned s in [p, n_ctx] at which the
- * recompute of [p, s) and the copy of [s, n_ctx) finish together, i.e. that
- * minimises max(T_recompute(p, s) + T_prompt, T_copy(s, n_ctx)) under the
+ * recompute of [p, s) (fused with the prompt) and the copy of [s, n_ctx)
+ * finish together, i.e. that minimises the predicted
+ * max(T_compute(p, s), T_copy(s, n_ctx) + last-layer tail) under the
  * profile's linear per-unit costs (Sec. 4.3, split in inverse proportion to
- * per-unit times). */
+ * per-unit times).  Returns s = p (copy only) unless the split is predicted
+ * to be at least 3% faster. */
 mzc_status mzc_plan_split(const mzc_model_shape *shape, const mzc_profile *profile, int64_t p,
                           int64_t n_ctx, int64_t n_prompt, int64_t *s_out);
 
@@ -198,8 +211,8 @@ mzc_status mzc_sync(mzc_ctx *ctx);
 /* Residency of (layer, logical_block) and its physical block (-1 if none). */
 mzc_status mzc_query(mzc_ctx *ctx, int32_t layer, int64_t logical_block, int32_t *state,
                      int32_t *phys);
-/* Reads one resident block's K and V ([n_kv_heads][16][head_dim], KV dtype
- * bits) into host buffers of block_bytes/2 each. */
+/* Reads one resident block's K and V ([n_kv_heads][16][head_dim], fp16 bits
+ * of the stored values) into host buffers of block_bytes/2 each. */
 mzc_status mzc_read_kv(mzc_ctx *ctx, int32_t layer, int64_t logical_block, void *k_host,
                        void *v_host);
 /* Reads K and V of every position [0, n) of every layer, widened to fp32,
@@ -231,9 +244,10 @@ typedef struct {
   double flops;     /* algorithmic FLOPs of those launches */
   double bytes;     /* algorithmic HBM bytes of those launches */
 } mzc_kernel_stat;
-/* on != 0: bracket every kernel of mzc_prefill with CUDA events on the
- * compute stream.  Either way, resets the per-class counters. */
-mzc_status mzc_set_kernel_timing(mzc_ctx *ctx, int32_t on);
+/* Bit c of class_mask (c = MZC_K_*): bracket every kernel of that class in
+ * mzc_prefill with CUDA events on the compute stream (-1: every class; 0:
+ * none).  Either way, resets the per-class counters. */
+mzc_status mzc_set_kernel_timing(mzc_ctx *ctx, int32_t class_mask);
 mzc_status mzc_kernel_stats(mzc_ctx *ctx, int32_t kernel_class, mzc_kernel_stat *out);
 
 /* ---------------------------------------------------------------------------
@@ -306,8 +320,9 @@ mzc_status mzc_k_swiglu_pack(const uint16_t *gate, const uint16_t *up, int64_t f
  * qkv fp16 [n][(hq + 2*hkv)*hd] (q heads, then k heads, then v heads),
  * pos int32 [n], cos/sin fp32 [max_pos][hd/2] (angle pos*theta^(-2i/hd)),
  * block_table int32 [n_logical] -> physical block, pool: block b holds
- * K [hkv][16][hd] then V [hkv][16][hd] in the KV dtype.
- * Out: q_out [n][hq][hd] rotated, in the KV dtype (the attention's operand type); K/V stored at pool[table[pos/16]]
+ * K [hkv][16][hd] then V [hkv][16][hd], fp16-encoded.
+ * Out: q_out [n][hq][hd] rotated, fp16; K/V rounded to kv_dtype precision and
+ * stored fp16-encoded at pool[table[pos/16]]
  * slot pos%16.  cos_t/sin_t must cover positions < n_logical*16.  status
  * (device int32, may be NULL) gets MZC_ERR_DEVICE on a bad index or block. */
 mzc_status mzc_k_rope_kv_write(const uint16_t *qkv, const int32_t *pos, int64_t n, int32_t hq,
@@ -318,7 +333,8 @@ mzc_status mzc_k_rope_kv_write(const uint16_t *qkv, const int32_t *pos, int64_t 
 
 /* Causal grouped-query attention over a block-table KV cache (the paper's
  * attention over non-contiguous KV chunks with online softmax, Sec. 4.2).
- * q [n][hq][hd] in the KV dtype at positions pos int32 [n]; row i attends to
+ * q fp16 [n][hq][hd] at positions pos int32 [n] over an fp16-encoded pool
+ * (kv_dtype is accepted for symmetry and ignored); row i attends to
  * every position <= pos[i] through block_table; out fp16 [n][hq][hd].
  * max_keys: an upper bound of pos[i] + 1 (sizes the split of long key
  * ranges).  scratch: device buffer of mzc_k_attention_scratch_bytes() bytes

@@ -615,17 +615,13 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   if (!make_pool_map(&map, pool, pool_blocks, hkv, hd)) return cudaErrorInvalidValue;
   float* part_o = static_cast<float*>(scratch);
   float* part_lse = s > 1 ? part_o + static_cast<int64_t>(s) * n * hq * hd : nullptr;
-  const bool f16 = kv_dtype == 1;
+  (void)kv_dtype;  // the pool is fp16-encoded for both KV types: q, K, P, V are fp16
   if (hd == 64)
-    return f16 ? launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
-                                     part_o, part_lse, s, per, status, st)
-               : launch_hd<64, false>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
-                                      out, part_o, part_lse, s, per, status, st);
+    return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
+                               part_o, part_lse, s, per, status, st);
   if (hd == 128)
-    return f16 ? launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
-                                      out, part_o, part_lse, s, per, status, st)
-               : launch_hd<128, false>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks,
-                                       out, part_o, part_lse, s, per, status, st);
+    return launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
+                                part_o, part_lse, s, per, status, st);
   return cudaErrorInvalidValue;
 }
 

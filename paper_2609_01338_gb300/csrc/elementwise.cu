@@ -32,6 +32,18 @@ __device__ __forceinline__ void unpack8_bf16(const uint4& v, float* f) {
   f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
 }
 
+// A value rounded to the KV storage precision (bf16 when !F16KV), encoded as
+// fp16: every normal-range bf16 value is exactly an fp16 value, so the pool
+// holds the stored values exactly while the attention reads one format.
+template <bool F16KV>
+__device__ __forceinline__ float kv_round(float x) {
+  if constexpr (F16KV) {
+    return x;
+  } else {
+    return __bfloat162float(__float2bfloat16_rn(x));
+  }
+}
+
 template <bool F16>
 __device__ __forceinline__ uint4 pack8(const float* f) {
   return make_uint4(pack2<F16>(f[0], f[1]), pack2<F16>(f[2], f[3]), pack2<F16>(f[4], f[5]),
@@ -95,11 +107,11 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restr
 }
 
 // Rotary embedding (pairs (i, i + hd/2), angle pos * theta^(-2i/hd) from the
-// fp32 tables) of q and k (fp16 projection output), then K/V stored into
-// their KV block slot:
+// fp32 tables) of q and k (fp16 projection output), then K/V rounded to the KV
+// storage precision and stored, fp16-encoded, into their KV block slot:
 // pool[table[pos/16]] = K [hkv][16][hd] then V [hkv][16][hd], slot pos % 16.
-// q goes to q_out [n][hq][hd] in the KV dtype.  One CTA per row.
-template <bool F16>
+// q goes to q_out [n][hq][hd] in fp16.  One CTA per row.
+template <bool F16KV>
 __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* __restrict__ pos,
                                int hq, int hkv, int hd, const float* __restrict__ cos_t,
                                const float* __restrict__ sin_t, const int32_t* __restrict__ table,
@@ -151,9 +163,14 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
       } else {
         if (!kv_ok) continue;
         dst = kbase + (static_cast<int64_t>(head - hq) * 16 + slot) * hd;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          y1[j] = kv_round<F16KV>(y1[j]);
+          y2[j] = kv_round<F16KV>(y2[j]);
+        }
       }
-      *reinterpret_cast<uint4*>(dst + c) = pack8<F16>(y1);
-      *reinterpret_cast<uint4*>(dst + c + half) = pack8<F16>(y2);
+      *reinterpret_cast<uint4*>(dst + c) = pack8<true>(y1);
+      *reinterpret_cast<uint4*>(dst + c + half) = pack8<true>(y2);
     } else {
       if (!kv_ok) continue;
       const int v = w - n_rot;
@@ -161,10 +178,12 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
       const uint16_t* src = row + static_cast<int64_t>(hq + hkv + head) * hd + c;
       uint4 raw = *reinterpret_cast<const uint4*>(src);
       uint16_t* dst = vbase + (static_cast<int64_t>(head) * 16 + slot) * hd + c;
-      if constexpr (!F16) {  // fp16 projection output -> bf16 KV
+      if constexpr (!F16KV) {  // fp16 projection output rounded to bf16 precision
         float f[8];
         unpack8_f16(raw, f);
-        raw = pack8<false>(f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) f[j] = kv_round<false>(f[j]);
+        raw = pack8<true>(f);
       }
       *reinterpret_cast<uint4*>(dst) = raw;
     }
@@ -312,10 +331,11 @@ cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t 
 cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
                                  int32_t kv_dtype, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  // the largest finite value of the KV type: finite, so a masked key (weight 0)
+  // the largest finite fp16 value: finite, so a masked key (weight 0)
   // contributes exactly 0, and far outside any real K/V, so a read of a block
   // before its restore lands shows up in the results
-  const uint32_t v16 = kv_dtype == 1 ? 0x7BFFu : 0x7F7Fu;
+  (void)kv_dtype;
+  const uint32_t v16 = 0x7BFFu;  // the pool is fp16-encoded for both KV types
   poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), phys,
                                                                   block_bytes / 16, v16 | (v16 << 16));
   return cudaGetLastError();

@@ -3,13 +3,11 @@
 // mantissa bits for the activations; the bf16 model weights convert exactly
 // at their scale.)
 //
-// One CTA computes a 128 x BN tile.  Warp 0 (one elected thread) streams
-// 128x64 A and BNx64 W tiles into a STAGES-deep shared-memory ring with TMA
-// (128-byte swizzle); warp 1 (one thread) issues tcgen05.mma (M=128, N=BN,
-// K=16 per instruction) accumulating fp32 in TMEM and releases each ring
-// slot with tcgen05.commit; then all four warps read the accumulator back
-// with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31 = tile rows) and apply
-// the epilogue:
+// A 128 x BN output tile: TMA streams 128x64 A and BNx64 W tiles (128-byte
+// swizzle) into a shared-memory ring, one thread issues tcgen05.mma (M=128,
+// N=BN, K=16 per instruction) accumulating fp32 in TMEM and releases each
+// ring slot with tcgen05.commit, and the epilogue warps read the accumulator
+// back with tcgen05.ld (one tile row per thread) and apply:
 //   EPI_STORE_BF16  out fp16 = C                      (QKV projection)
 //   EPI_ADD_F32     out fp32 += C                     (O / down projection + residual)
 //   EPI_SWIGLU_BF16 out fp16 = silu(C_gate) * C_up    (gate/up projection, rows interleaved
@@ -28,168 +26,13 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 fp16 = 128 bytes = one swizzle row
 
-template <int BN, int STAGES>
-struct GemmCfg {
-  static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
-  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
-  static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
-};
-
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)); }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-template <int BN, int STAGES, int EPI>
-__global__ void __launch_bounds__(128) gemm_tc_kernel(const __grid_constant__ CUtensorMap tma,
-                                                      const __grid_constant__ CUtensorMap tmw,
-                                                      void* __restrict__ out, int m, int n, int k,
-                                                      int32_t* status) {
-  using C = GemmCfg<BN, STAGES>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
-  uint64_t* empty = full + STAGES;
-  uint64_t* accum = empty + STAGES;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
-  const int num_k = (k + BK - 1) / BK;
-
-  if (threadIdx.x == 0) {
-    tma_prefetch_desc(&tma);
-    tma_prefetch_desc(&tmw);
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
-    }
-    mbar_init(accum, 1);
-    fence_barrier_init();
-  }
-  if (warp == 0) tmem_alloc(tmem_slot, C::TMEM_COLS);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  if (warp == 0 && lane == 0) {
-    // TMA producer
-    for (int kb = 0; kb < num_k; ++kb) {
-      const int s = kb % STAGES;
-      const uint32_t ph = (kb / STAGES) & 1;
-      if (kb >= STAGES && !mbar_wait(&empty[s], ph ^ 1, status)) break;
-      mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
-      tma_load_2d(sA + s * C::A_BYTES, &tma, &full[s], kb * BK, m0);
-      tma_load_2d(sB + s * C::B_BYTES, &tmw, &full[s], kb * BK, n0);
-    }
-  } else if (warp == 1 && lane == 0) {
-    // UMMA issuer
-    constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
-    for (int kb = 0; kb < num_k; ++kb) {
-      const int s = kb % STAGES;
-      const uint32_t ph = (kb / STAGES) & 1;
-      if (!mbar_wait(&full[s], ph, status)) break;
-      tc_fence_after();
-      const uint64_t ad = sdesc_k_sw128(smem_u32(sA + s * C::A_BYTES));
-      const uint64_t bd = sdesc_k_sw128(smem_u32(sB + s * C::B_BYTES));
-#pragma unroll
-      for (int kk = 0; kk < BK / 16; ++kk)
-        umma_f16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
-      umma_commit(&empty[s]);
-    }
-    umma_commit(accum);
-  }
-  __syncwarp();
-
-  // ---- epilogue: thread = one tile row ----
-  const bool ok = mbar_wait(accum, 0, status);
-  __syncwarp();
-  tc_fence_after();
-  const int row = m0 + warp * 32 + lane;
-  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  if (ok) {
-    if constexpr (EPI == EPI_SWIGLU_BF16) {
-      const int nout = n / 2;
-#pragma unroll 1
-      for (int g = 0; g < BN / (2 * kSwigluGroup); ++g) {
-#pragma unroll 1
-        for (int c = 0; c < kSwigluGroup; c += 32) {
-          float vg[32], vu[32];
-          tmem_ld32(trow + g * 2 * kSwigluGroup + c, vg);
-          tmem_ld32(trow + g * 2 * kSwigluGroup + kSwigluGroup + c, vu);
-          const int col = n0 / 2 + g * kSwigluGroup + c;
-          if (row < m && col < nout) {
-            uint32_t pk[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i)
-              pk[i] = pack2<true>(silu_f(vg[2 * i]) * vu[2 * i],
-                                   silu_f(vg[2 * i + 1]) * vu[2 * i + 1]);
-            uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) +
-                                                static_cast<size_t>(row) * nout + col);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-          }
-        }
-      }
-    } else {
-#pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        float v[32];
-        tmem_ld32(trow + c, v);
-        const int col = n0 + c;
-        if (row < m && col < n) {
-          const int cnt = min(32, n - col);  // n is a multiple of 16
-          if constexpr (EPI == EPI_STORE_BF16) {
-            uint32_t pk[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) pk[i] = pack2<true>(v[2 * i], v[2 * i + 1]);
-            uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) +
-                                                static_cast<size_t>(row) * n + col);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              if (i * 8 < cnt) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-          } else {
-            float4* o = reinterpret_cast<float4*>(static_cast<float*>(out) +
-                                                  static_cast<size_t>(row) * n + col);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              if (i * 4 < cnt) {
-                float4 t = o[i];
-                t.x += v[4 * i];
-                t.y += v[4 * i + 1];
-                t.z += v[4 * i + 2];
-                t.w += v[4 * i + 3];
-                o[i] = t;
-              }
-            }
-          }
-        }
-      }
-    }
-  }
-
-  // ---- teardown ----
-  if (warp == 0 && lane == 0) {
-    // drain: the last fill of every ring slot has landed before smem is released
-    for (int kb = num_k - STAGES < 0 ? 0 : num_k - STAGES; kb < num_k; ++kb)
-      mbar_wait(&full[kb % STAGES], (kb / STAGES) & 1, status);
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) {
-    __syncwarp();
-    tmem_dealloc(tmem, C::TMEM_COLS);
-  }
-}
-
-// Persistent variant for M > 128: one CTA per SM walks 128 x BN tiles
+// Persistent GEMM: one CTA per SM walks 128 x BN tiles
 // (grouped order: a band of kBandN tiles of N down all of M, so a band of
 // weight tiles stays in L2 while the activations stream), with a
 // double-buffered TMEM accumulator so that the epilogue of tile i overlaps
@@ -450,23 +293,6 @@ EncodeFn encode_fn() {
   return fn;
 }
 
-template <int BN, int STAGES, int EPI>
-cudaError_t launch_cfg(const CUtensorMap& ta, const CUtensorMap& tw, void* out, int64_t m,
-                       int64_t n, int64_t k, int32_t* status, cudaStream_t st) {
-  using C = GemmCfg<BN, STAGES>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, EPI>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  });
-  if (attr_err != cudaSuccess) return attr_err;
-  dim3 grid(static_cast<unsigned>((n + BN - 1) / BN), static_cast<unsigned>((m + BM - 1) / BM));
-  gemm_tc_kernel<BN, STAGES, EPI><<<grid, 128, C::SMEM, st>>>(
-      ta, tw, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
-  return cudaGetLastError();
-}
-
 }  // namespace
 
 bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
@@ -484,9 +310,8 @@ bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue) {
   (void)n;
-  if (m > 128) return 256;  // persistent 128 x 256 tiles
-  if (epilogue == EPI_SWIGLU_BF16) return 128;
-  return 64;
+  if (m > 512) return 256;                        // persistent 128 x 256 tiles
+  return epilogue == EPI_SWIGLU_BF16 ? 128 : 64;  // persistent narrow tiles, deep ring
 }
 
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) {
@@ -494,11 +319,14 @@ bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) 
          make_tmap_f16(&gw->box256, base, n, k, 256);
 }
 
+// Tile choice: above 512 rows the GEMM is tensor-bound and takes 128 x 256
+// tiles; at or below it is bound by streaming the weights, so it takes narrow
+// tiles (more CTAs pulling weight bytes) and a deeper ring (more bytes in
+// flight per SM).  The W map passed always has the box the kernel expects.
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
   if (m <= 0) return cudaSuccess;
-  if (m > 128) {
-    // the W tile the kernel expects (256 rows) is exactly the box of the map it gets
+  if (m > 512) {
     switch (epilogue) {
       case EPI_STORE_BF16:
         return launch_persistent<256, 4, EPI_STORE_BF16>(ta, w.box256, out, m, n, k, status, st);
@@ -512,11 +340,11 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
   }
   switch (epilogue) {
     case EPI_STORE_BF16:
-      return launch_cfg<64, 4, EPI_STORE_BF16>(ta, w.box64, out, m, n, k, status, st);
+      return launch_persistent<64, 8, EPI_STORE_BF16>(ta, w.box64, out, m, n, k, status, st);
     case EPI_ADD_F32:
-      return launch_cfg<64, 4, EPI_ADD_F32>(ta, w.box64, out, m, n, k, status, st);
+      return launch_persistent<64, 8, EPI_ADD_F32>(ta, w.box64, out, m, n, k, status, st);
     case EPI_SWIGLU_BF16:
-      return launch_cfg<128, 3, EPI_SWIGLU_BF16>(ta, w.box128, out, m, n, k, status, st);
+      return launch_persistent<128, 6, EPI_SWIGLU_BF16>(ta, w.box128, out, m, n, k, status, st);
     default:
       return cudaErrorInvalidValue;
   }

@@ -49,10 +49,13 @@ size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 mzc_profile default_profile() {
   mzc_profile p;
   p.h2d_gbs = 200.0;
-  p.hbm_gbs = 6000.0;
-  p.gemm_tflops = 1000.0;
-  p.attn_tflops = 400.0;
-  p.launch_us = 30.0;
+  p.gemm_us_128 = 110.0;
+  p.gemm_us_512 = 260.0;
+  p.gemm_us_2048 = 700.0;
+  p.attn_tflops = 500.0;
+  p.attn_prompt_tflops = 500.0;
+  p.row_ns = 150.0;
+  p.layer_us = 15.0;
   return p;
 }
 
@@ -93,7 +96,7 @@ struct mzc_ctx {
               ev_l0 = nullptr, ev_l1 = nullptr;
   bool restore_issued = false, lm_timed = false, ttft_from_copy = false;
   // per-class launch counts and optional CUDA-event timing
-  bool ktime = false;
+  int32_t ktime_mask = 0;
   mzc_kernel_stat kstat[MZC_K_NCLASS] = {};
   struct KEv {
     int cls;
@@ -412,7 +415,7 @@ cudaError_t klaunch(mzc_ctx* ctx, int cls, double flops, double bytes, int n_ker
   k.launches += n_kernels;
   k.flops += flops;
   k.bytes += bytes;
-  if (!ctx->ktime) return fn();
+  if (!((ctx->ktime_mask >> cls) & 1)) return fn();
   cudaEvent_t a = next_event(ctx), b = next_event(ctx);
   if (!a || !b) return cudaErrorMemoryAllocation;
   cudaError_t e = cudaEventRecord(a, ctx->cs);
@@ -594,35 +597,59 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
   return MZC_OK;
 }
 
-// Linear per-unit cost model of the two restore paths (Sec. 4.3: per-unit
-// times, total time linear in the number of units).
-struct CostModel {
-  mzc_model_shape s;
-  mzc_profile p;
+// Per-layer algorithmic sizes of a shape.
+struct CostModelShape {
   double layer_weight_bytes, linear_flops_row, attn_flops_pair;
-  CostModel(const mzc_model_shape& s_, const mzc_profile& p_) : s(s_), p(p_) {
+  explicit CostModelShape(const mzc_model_shape& s) {
     const double d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim, f = s.ffn_dim;
     const double params = d * (hq + 2 * hkv) * hd + hq * hd * d + 3.0 * d * f;
     layer_weight_bytes = 2.0 * params;
     linear_flops_row = 2.0 * params;
     attn_flops_pair = 4.0 * hd * hq;
   }
+};
+
+// Per-unit cost model of the two restore paths (Sec. 4.3: per-unit times
+// from offline profiling, total time linear in the number of units).
+// Copy: evicted blocks x bytes / host-link rate.  Compute of the fused rows
+// (recomputed tail + prompt), per layer: the projections interpolated from
+// their measured times at 128 / 512 / 2048 rows, attention pairs at the
+// measured rates of recompute-like and prompt-like rows, per-row
+// memory-bound kernels and a fixed per-layer cost.  The two paths overlap
+// layer by layer, so a step takes the longer of the two, plus the part of the
+// last layer that runs after its copy has landed.
+struct CostModel : CostModelShape {
+  mzc_model_shape s;
+  mzc_profile p;
+  CostModel(const mzc_model_shape& s_, const mzc_profile& p_) : CostModelShape(s_), s(s_), p(p_) {}
   double copy_s(int64_t tokens) const {
     const double blocks = static_cast<double>(ceil_div(tokens, 16));
     const double bytes = blocks * s.n_layers * 2.0 * s.n_kv_heads * 16 * s.head_dim * 2;
     return bytes / (p.h2d_gbs * 1e9);
   }
-  double compute_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
+  double gemm_s(double rows) const {
+    double us;
+    if (rows <= 128) us = p.gemm_us_128;
+    else if (rows <= 512) us = p.gemm_us_128 + (rows - 128) * (p.gemm_us_512 - p.gemm_us_128) / 384.0;
+    else us = p.gemm_us_512 + (rows - 512) * (p.gemm_us_2048 - p.gemm_us_512) / 1536.0;
+    return us * 1e-6;
+  }
+  double layer_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
     const double rows = static_cast<double>(s1 - p0 + n_prompt);
     if (rows <= 0) return 0.0;
-    const double gemm = std::max(rows * linear_flops_row / (p.gemm_tflops * 1e12),
-                                 layer_weight_bytes / (p.hbm_gbs * 1e9));
-    // sum of (pos + 1) over recompute rows [p0, s1) and prompt rows [n_ctx, n_ctx + n_prompt)
     auto tri = [](double a, double b) { return (b * (b + 1) - a * (a + 1)) / 2.0; };
-    const double pairs = tri(static_cast<double>(p0), static_cast<double>(s1)) +
-                         tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
-    const double attn = pairs * attn_flops_pair / (p.attn_tflops * 1e12);
-    return s.n_layers * (gemm + attn + p.launch_us * 1e-6);
+    const double rec_pairs = tri(static_cast<double>(p0), static_cast<double>(s1));
+    const double prm_pairs = tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
+    const double attn = rec_pairs * attn_flops_pair / (p.attn_tflops * 1e12) +
+                        prm_pairs * attn_flops_pair / (p.attn_prompt_tflops * 1e12);
+    return gemm_s(rows) + attn + rows * p.row_ns * 1e-9 + p.layer_us * 1e-6;
+  }
+  // predicted TTFT when [p0, s1) is recomputed and [s1, n_ctx) copied
+  double ttft_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
+    const double layer = layer_s(p0, s1, n_ctx, n_prompt);
+    const double compute = s.n_layers * layer;
+    const double copy = copy_s(n_ctx - s1);
+    return copy > 0.0 ? std::max(compute, copy + 0.75 * layer) : compute;
   }
 };
 
@@ -781,21 +808,25 @@ mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profi
                           int64_t n_ctx, int64_t n_prompt, int64_t* s_out) {
   if (!shape || !s_out || p < 0 || n_ctx < p || n_prompt < 0) return MZC_ERR_INVALID;
   const mzc_profile prof = profile ? *profile : default_profile();
-  if (prof.h2d_gbs <= 0 || prof.hbm_gbs <= 0 || prof.gemm_tflops <= 0 || prof.attn_tflops <= 0)
+  if (prof.h2d_gbs <= 0 || prof.gemm_us_128 <= 0 || prof.gemm_us_512 <= 0 || prof.gemm_us_2048 <= 0 ||
+      prof.attn_tflops <= 0 || prof.attn_prompt_tflops <= 0 || prof.row_ns < 0 || prof.layer_us < 0)
     return MZC_ERR_INVALID;
   CostModel cm(*shape, prof);
+  // candidates: block boundaries from p, and n_ctx itself; leave copy-only
+  // (s = p) only for a predicted gain of at least 5%
+  const double copy_only = cm.ttft_s(p, p, n_ctx, n_prompt);
   int64_t best = p;
-  double best_t = INFINITY;
-  // candidates: block boundaries from p, and n_ctx itself
-  for (int64_t s = p;; s += 16) {
+  double best_t = copy_only;
+  for (int64_t s = p + 16;; s += 16) {
     const int64_t sc = std::min(s, n_ctx);
-    const double t = std::max(cm.compute_s(p, sc, n_ctx, n_prompt), cm.copy_s(n_ctx - sc));
+    const double t = cm.ttft_s(p, sc, n_ctx, n_prompt);
     if (t < best_t) {
       best_t = t;
       best = sc;
     }
     if (sc >= n_ctx) break;
   }
+  if (best_t > 0.95 * copy_only) best = p;
   *s_out = best;
   return MZC_OK;
 }
@@ -879,18 +910,12 @@ mzc_status mzc_read_kv_all(mzc_ctx* ctx, int64_t n, float* k_host, float* v_host
         const uint16_t* vb = kb + hkv * 16 * hd;
         float* ko = k_host + ((static_cast<int64_t>(l) * n + p) * hkv + h) * hd;
         float* vo = v_host + ((static_cast<int64_t>(l) * n + p) * hkv + h) * hd;
-        for (int64_t c = 0; c < hd; ++c) {
-          if (s.kv_dtype == MZC_KV_FP16) {
-            __half_raw rk, rv;
-            rk.x = kb[c];
-            rv.x = vb[c];
-            ko[c] = __half2float(__half(rk));
-            vo[c] = __half2float(__half(rv));
-          } else {
-            uint32_t uk = static_cast<uint32_t>(kb[c]) << 16, uv = static_cast<uint32_t>(vb[c]) << 16;
-            std::memcpy(&ko[c], &uk, 4);
-            std::memcpy(&vo[c], &uv, 4);
-          }
+        for (int64_t c = 0; c < hd; ++c) {  // the pool is fp16-encoded for both KV types
+          __half_raw rk, rv;
+          rk.x = kb[c];
+          rv.x = vb[c];
+          ko[c] = __half2float(__half(rk));
+          vo[c] = __half2float(__half(rv));
         }
       }
     }
@@ -920,9 +945,9 @@ mzc_status mzc_last_times(mzc_ctx* ctx, float* ms3) {  // ms3 holds 4 floats
   return MZC_OK;
 }
 
-mzc_status mzc_set_kernel_timing(mzc_ctx* ctx, int32_t on) {
+mzc_status mzc_set_kernel_timing(mzc_ctx* ctx, int32_t class_mask) {
   if (!ctx) return MZC_ERR_INVALID;
-  ctx->ktime = on != 0;
+  ctx->ktime_mask = class_mask;
   for (auto& k : ctx->kstat) k = mzc_kernel_stat{};
   return MZC_OK;
 }
@@ -962,85 +987,97 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
     CK(cudaFreeHost(h));
     CK(cudaMemset(ctx->d_pool, 0, bytes));
   }
-  // HBM: device-to-device copy of the activation buffers
+  // A whole layer's four projections on scratch activations at 128, 512 and
+  // 2048 rows (capped by max_rows).
   {
-    const int64_t bytes = ctx->max_rows * ctx->shape.d_model * 2;
-    CK(cudaMemcpyAsync(ctx->d_attn, ctx->d_h, bytes, cudaMemcpyDeviceToDevice, ctx->cs));
-    CK(cudaEventRecord(a, ctx->cs));
-    for (int i = 0; i < 10; ++i) CK(cudaMemcpyAsync(ctx->d_attn, ctx->d_h, bytes, cudaMemcpyDeviceToDevice, ctx->cs));
-    CK(cudaEventRecord(b, ctx->cs));
-    CK(cudaEventSynchronize(b));
-    CK(cudaEventElapsedTime(&ms, a, b));
-    if (ms > 0) p.hbm_gbs = 10.0 * 2.0 * bytes / (ms * 1e-3) / 1e9;
-  }
-  // GEMM: layer 0's projections at recompute sizes on scratch activations
-  {
-    const int64_t m = std::min<int64_t>(ctx->max_rows, 4096), d = ctx->shape.d_model;
     const LayerDev& W = ctx->layers[0];
-    auto run = [&]() -> cudaError_t {
+    const int64_t d = ctx->shape.d_model, hq = ctx->shape.n_q_heads, hd = ctx->shape.head_dim;
+    auto layer_gemms = [&](int64_t m) -> cudaError_t {
       cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, ctx->d_status, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_attn, W.tm_o, ctx->d_x, m, d, hq * hd, mzc::EPI_ADD_F32, ctx->d_status, ctx->cs);
       if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, ctx->d_status, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_act, W.tm_2, ctx->d_x, m, d, ctx->f_pad, mzc::EPI_ADD_F32, ctx->d_status, ctx->cs);
       return e;
     };
-    CK(run());
-    CK(cudaEventRecord(a, ctx->cs));
-    for (int i = 0; i < 5; ++i) CK(run());
-    CK(cudaEventRecord(b, ctx->cs));
-    CK(cudaEventSynchronize(b));
-    CK(cudaEventElapsedTime(&ms, a, b));
-    const double flops = 5.0 * 2.0 * m * d * (ctx->qkv_dim + 2 * ctx->f_pad);
-    if (ms > 0) p.gemm_tflops = flops / (ms * 1e-3) / 1e12;
+    const int64_t sizes[3] = {128, 512, 2048};
+    double* outs[3] = {&p.gemm_us_128, &p.gemm_us_512, &p.gemm_us_2048};
+    for (int t = 0; t < 3; ++t) {
+      const int64_t m = std::min<int64_t>(ctx->max_rows, sizes[t]);
+      CK(layer_gemms(m));
+      CK(cudaEventRecord(a, ctx->cs));
+      for (int i = 0; i < 5; ++i) CK(layer_gemms(m));
+      CK(cudaEventRecord(b, ctx->cs));
+      CK(cudaEventSynchronize(b));
+      CK(cudaEventElapsedTime(&ms, a, b));
+      // rows beyond max_rows would run in chunks: scale linearly
+      if (ms > 0) *outs[t] = ms * 1e3 / 5.0 * static_cast<double>(sizes[t]) / static_cast<double>(m);
+    }
   }
-  // attention over the resident context, when there is one
+  // attention over the resident context, when there is one: 1024 rows in
+  // the middle of the context (recompute-like, causal) and 128 rows at its
+  // end (prompt-like, split over the whole context)
   {
     const int64_t n_ctx = ctx->st.n_ctx();
-    bool resident = n_ctx >= 1024;
+    bool resident = n_ctx >= 2048;
     for (int32_t l = 0; l < ctx->shape.n_layers && resident; ++l)
       for (int64_t blk = 0; blk < ceil_div(n_ctx, 16) && resident; ++blk)
         resident = ctx->st.at(l, blk).st == MZC_RESIDENT;
     if (resident) {
-      const int64_t rows = std::min<int64_t>(ctx->max_rows, 1024);
-      int32_t* hp = reinterpret_cast<int32_t*>(ctx->h_meta);
-      for (int64_t i = 0; i < rows; ++i) hp[i] = static_cast<int32_t>(n_ctx - rows + i);
+      const mzc_model_shape& s = ctx->shape;
       std::vector<int32_t> tab;
       ctx->st.block_table(&tab);
-      std::memcpy(hp + rows, tab.data(), ctx->nblk * 4);
-      int32_t* dp = reinterpret_cast<int32_t*>(ctx->d_meta);
-      CK(cudaMemcpyAsync(dp, hp, (rows + ctx->nblk) * 4, cudaMemcpyHostToDevice, ctx->cs));
-      const mzc_model_shape& s = ctx->shape;
-      auto run = [&]() {
-        return mzc::launch_attention(ctx->d_q, dp, rows, s.n_q_heads, s.n_kv_heads, s.head_dim, dp + rows,
-                                     ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(), s.kv_dtype,
-                                     ctx->d_attn, ctx->d_scratch, ctx->scratch_bytes, n_ctx,
-                                     ctx->num_sms, ctx->d_status, ctx->cs);
-      };
-      CK(run());
-      CK(cudaEventRecord(a, ctx->cs));
-      for (int i = 0; i < 3; ++i) CK(run());
-      CK(cudaEventRecord(b, ctx->cs));
-      CK(cudaEventSynchronize(b));
-      CK(cudaEventElapsedTime(&ms, a, b));
-      double pairs = 0;
-      for (int64_t i = 0; i < rows; ++i) pairs += static_cast<double>(n_ctx - rows + i + 1);
-      const double flops = 3.0 * pairs * 4.0 * s.head_dim * s.n_q_heads;
-      if (ms > 0) p.attn_tflops = flops / (ms * 1e-3) / 1e12;
+      for (int kind = 0; kind < 2; ++kind) {
+        const int64_t rows = std::min<int64_t>(ctx->max_rows, kind == 0 ? 1024 : 128);
+        const int64_t first = kind == 0 ? n_ctx / 2 : n_ctx - rows;
+        int32_t* hp = reinterpret_cast<int32_t*>(ctx->h_meta);
+        for (int64_t i = 0; i < rows; ++i) hp[i] = static_cast<int32_t>(first + i);
+        std::memcpy(hp + rows, tab.data(), ctx->nblk * 4);
+        int32_t* dp = reinterpret_cast<int32_t*>(ctx->d_meta);
+        CK(cudaMemcpyAsync(dp, hp, (rows + ctx->nblk) * 4, cudaMemcpyHostToDevice, ctx->cs));
+        const int64_t max_keys = first + rows;
+        auto run = [&]() {
+          return mzc::launch_attention(ctx->d_q, dp, rows, s.n_q_heads, s.n_kv_heads, s.head_dim, dp + rows,
+                                       ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(), s.kv_dtype,
+                                       ctx->d_attn, ctx->d_scratch, ctx->scratch_bytes, max_keys,
+                                       ctx->num_sms, ctx->d_status, ctx->cs);
+        };
+        CK(run());
+        CK(cudaEventRecord(a, ctx->cs));
+        for (int i = 0; i < 3; ++i) CK(run());
+        CK(cudaEventRecord(b, ctx->cs));
+        CK(cudaEventSynchronize(b));
+        CK(cudaEventElapsedTime(&ms, a, b));
+        double pairs = 0;
+        for (int64_t i = 0; i < rows; ++i) pairs += static_cast<double>(first + i + 1);
+        const double flops = 3.0 * pairs * 4.0 * s.head_dim * s.n_q_heads;
+        if (ms > 0) (kind == 0 ? p.attn_tflops : p.attn_prompt_tflops) = flops / (ms * 1e-3) / 1e12;
+      }
     }
   }
-  // per-layer launch cost: the 8 launches of one layer at one row
+  // memory-bound kernels per row (two RMSNorms and the rotary/KV write,
+  // approximated by three norms over 1024 rows) and the fixed per-layer cost
+  // (the same launches at one row)
   {
-    auto run = [&]() -> cudaError_t {
+    auto norms = [&](int64_t rows) -> cudaError_t {
       cudaError_t e = cudaSuccess;
-      for (int i = 0; i < 8 && e == cudaSuccess; ++i)
-        e = mzc::launch_rmsnorm(ctx->d_x, ctx->layers[0].attn_norm, 1, ctx->shape.d_model, 1e-5f, ctx->d_h, ctx->cs);
+      for (int i = 0; i < 3 && e == cudaSuccess; ++i)
+        e = mzc::launch_rmsnorm(ctx->d_x, ctx->layers[0].attn_norm, rows, ctx->shape.d_model, 1e-5f,
+                                ctx->d_h, ctx->cs);
       return e;
     };
-    CK(run());
-    CK(cudaEventRecord(a, ctx->cs));
-    for (int i = 0; i < 20; ++i) CK(run());
-    CK(cudaEventRecord(b, ctx->cs));
-    CK(cudaEventSynchronize(b));
-    CK(cudaEventElapsedTime(&ms, a, b));
-    p.launch_us = ms * 1e3 / 20.0;
+    float ms1 = 0.0f, msn = 0.0f;
+    const int64_t rows = std::min<int64_t>(ctx->max_rows, 1024);
+    for (int pass = 0; pass < 2; ++pass) {
+      const int64_t r = pass == 0 ? 1 : rows;
+      CK(norms(r));
+      CK(cudaEventRecord(a, ctx->cs));
+      for (int i = 0; i < 20; ++i) CK(norms(r));
+      CK(cudaEventRecord(b, ctx->cs));
+      CK(cudaEventSynchronize(b));
+      CK(cudaEventElapsedTime(pass == 0 ? &ms1 : &msn, a, b));
+    }
+    p.layer_us = ms1 * 1e3 / 20.0 * (8.0 / 3.0);  // ~8 launches per layer
+    p.row_ns = std::max(0.0, (static_cast<double>(msn) - ms1) * 1e6 / 20.0 / static_cast<double>(rows));
   }
   CK(cudaEventDestroy(a));
   CK(cudaEventDestroy(b));

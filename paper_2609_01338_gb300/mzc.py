@@ -50,8 +50,9 @@ class mzc_weights(ctypes.Structure):
 
 
 class mzc_profile(ctypes.Structure):
-    _fields_ = [("h2d_gbs", c_f64), ("hbm_gbs", c_f64), ("gemm_tflops", c_f64),
-                ("attn_tflops", c_f64), ("launch_us", c_f64)]
+    _fields_ = [("h2d_gbs", c_f64), ("gemm_us_128", c_f64), ("gemm_us_512", c_f64),
+                ("gemm_us_2048", c_f64), ("attn_tflops", c_f64), ("attn_prompt_tflops", c_f64),
+                ("row_ns", c_f64), ("layer_us", c_f64)]
 
 
 class mzc_stats_t(ctypes.Structure):
@@ -315,8 +316,9 @@ def mzc_last_times(ctx):
     return a
 
 
-def mzc_set_kernel_timing(ctx, on: bool):
-    return _call("mzc_set_kernel_timing", ctx, int(bool(on)), ctx=ctx)
+def mzc_set_kernel_timing(ctx, class_mask: int):
+    """Bit c times kernel class c (MZC_K_*); -1 every class; 0 none."""
+    return _call("mzc_set_kernel_timing", ctx, int(class_mask), ctx=ctx)
 
 
 def mzc_kernel_stats(ctx, cls) -> mzc_kernel_stat:

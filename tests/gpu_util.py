@@ -23,15 +23,16 @@ def to_np_u16(t) -> np.ndarray:
     return t.cpu().numpy().view(np.uint16)
 
 
-def kv_bits_to_f32(bits: np.ndarray, kv_dtype: int) -> np.ndarray:
-    if kv_dtype == 1:
-        return bits.view(np.float16).astype(np.float32)
-    return synth.bf16_bits_to_f32(bits)
+def kv_bits_to_f32(bits: np.ndarray, kv_dtype: int = 1) -> np.ndarray:
+    """Decode pool / q bits: the pool holds fp16-encoded values for both KV
+    types (bf16-rounded values when kv_dtype is bf16)."""
+    return np.asarray(bits).view(np.float16).astype(np.float32)
 
 
 def f32_to_kv_bits(x: np.ndarray, kv_dtype: int) -> np.ndarray:
+    """Round to the KV precision (bf16 or fp16), then fp16-encode."""
     import oracle
-    return oracle.to_f16_bits(x) if kv_dtype == 1 else oracle.to_bf16_bits(x)
+    return oracle.round_kv(np.asarray(x, np.float32), kv_dtype).astype(np.float16).view(np.uint16)
 
 
 def rel_err(got, ref) -> float:

@@ -160,12 +160,12 @@ def test_rope_kv_write(hq, hkv, hd, kvd):
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     x = f16_to_f32(qkv).reshape(n, hq + 2 * hkv, hd)
-    q_ref = oracle.round_kv(oracle.rope(x[:, :hq], pos, 500000.0), kvd)
     k_ref = oracle.round_kv(oracle.rope(x[:, hq:hq + hkv], pos, 500000.0), kvd)
     v_ref = oracle.round_kv(x[:, hq + hkv:], kvd)
     ulp = 2.0 ** (-10 if kvd == 1 else -7)
-    q_got = kv_bits_to_f32(to_np_u16(q_out), kvd)
-    assert np.all(np.abs(q_got - q_ref) <= ulp * np.abs(q_ref) + 1e-7)
+    q_got = f16_to_f32(to_np_u16(q_out))  # q is fp16 for both KV types
+    q_ref = oracle.rope(x[:, :hq], pos, 500000.0)
+    assert np.all(np.abs(q_got - q_ref) <= 2.0 ** -10 * np.abs(q_ref) + 1e-6)
     pool_np = to_np_u16(pool).reshape(pool_blocks, 2, hkv, 16, hd)
     k_got = np.stack([pool_np[table[p // 16], 0, :, p % 16] for p in pos])
     v_got = np.stack([pool_np[table[p // 16], 1, :, p % 16] for p in pos])
@@ -190,7 +190,7 @@ def _attention_case(hq, hkv, hd, kvd, ctx, pos, seed, use_scratch=True):
     rng = np.random.default_rng(seed)
     kf = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
     vf = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
-    qf = f32_to_kv_bits((rng.standard_normal((n, hq, hd)) * 2.0).astype(np.float32), kvd)
+    qf = f16_bits((rng.standard_normal((n, hq, hd)) * 2.0).astype(np.float32))
     pool_np = np.zeros((pool_blocks, 2, hkv, 16, hd), np.uint16)
     for p in range(ctx):
         pool_np[table[p // 16], 0, :, p % 16] = kf[p]
@@ -206,8 +206,7 @@ def _attention_case(hq, hkv, hd, kvd, ctx, pos, seed, use_scratch=True):
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     got = f16_to_f32(to_np_u16(out))
-    ref = oracle.attention(kv_bits_to_f32(qf, kvd), pos, kv_bits_to_f32(kf, kvd),
-                           kv_bits_to_f32(vf, kvd))
+    ref = oracle.attention(f16_to_f32(qf), pos, kv_bits_to_f32(kf), kv_bits_to_f32(vf))
     return got, ref, sb
 
 

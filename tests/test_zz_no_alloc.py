@@ -31,7 +31,7 @@ def _inputs(seed, hq, hkv, hd, kvd, ctx, n):
     rng = np.random.default_rng(seed)
     k = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
     v = f32_to_kv_bits(rng.standard_normal((ctx, hkv, hd)).astype(np.float32), kvd)
-    q = f32_to_kv_bits((rng.standard_normal((n, hq, hd)) * 2.0).astype(np.float32), kvd)
+    q = (rng.standard_normal((n, hq, hd)) * 2.0).astype(np.float16).view(np.uint16)
     pool = np.zeros((pool_blocks, 2, hkv, 16, hd), np.uint16)
     for p in range(ctx):
         pool[table[p // 16], 0, :, p % 16] = k[p]
