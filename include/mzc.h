@@ -108,7 +108,8 @@ typedef struct {
   double gemm_us_128;        /* one layer's four projections at 128 rows, us */
   double gemm_us_512;        /* ... at 512 rows, us */
   double gemm_us_2048;       /* ... at 2048 rows, us */
-  double attn_tflops;        /* attention of recompute-like rows (causal, mid-context), TFLOP/s */
+  double attn_tflops;        /* attention of recompute-like rows: marginal rate per key, TFLOP/s */
+  double attn_row_ns;        /* ... plus a fixed cost per row and layer, ns */
   double attn_prompt_tflops; /* attention of prompt rows over the whole context, TFLOP/s */
   double row_ns;             /* per row and layer: norms and rotary/KV write, ns */
   double layer_us;           /* per layer fixed cost (launch gaps), us */

@@ -52,7 +52,8 @@ mzc_profile default_profile() {
   p.gemm_us_128 = 110.0;
   p.gemm_us_512 = 260.0;
   p.gemm_us_2048 = 700.0;
-  p.attn_tflops = 500.0;
+  p.attn_tflops = 800.0;
+  p.attn_row_ns = 2000.0;
   p.attn_prompt_tflops = 500.0;
   p.row_ns = 150.0;
   p.layer_us = 15.0;
@@ -641,6 +642,7 @@ struct CostModel : CostModelShape {
     const double rec_pairs = tri(static_cast<double>(p0), static_cast<double>(s1));
     const double prm_pairs = tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
     const double attn = rec_pairs * attn_flops_pair / (p.attn_tflops * 1e12) +
+                        static_cast<double>(s1 - p0) * p.attn_row_ns * 1e-9 +
                         prm_pairs * attn_flops_pair / (p.attn_prompt_tflops * 1e12);
     return gemm_s(rows) + attn + rows * p.row_ns * 1e-9 + p.layer_us * 1e-6;
   }
@@ -809,7 +811,8 @@ mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profi
   if (!shape || !s_out || p < 0 || n_ctx < p || n_prompt < 0) return MZC_ERR_INVALID;
   const mzc_profile prof = profile ? *profile : default_profile();
   if (prof.h2d_gbs <= 0 || prof.gemm_us_128 <= 0 || prof.gemm_us_512 <= 0 || prof.gemm_us_2048 <= 0 ||
-      prof.attn_tflops <= 0 || prof.attn_prompt_tflops <= 0 || prof.row_ns < 0 || prof.layer_us < 0)
+      prof.attn_tflops <= 0 || prof.attn_row_ns < 0 || prof.attn_prompt_tflops <= 0 || prof.row_ns < 0 ||
+      prof.layer_us < 0)
     return MZC_ERR_INVALID;
   CostModel cm(*shape, prof);
   // candidates: block boundaries from p, and n_ctx itself; leave copy-only
@@ -1013,9 +1016,10 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
       if (ms > 0) *outs[t] = ms * 1e3 / 5.0 * static_cast<double>(sizes[t]) / static_cast<double>(m);
     }
   }
-  // attention over the resident context, when there is one: 1024 rows in
-  // the middle of the context (recompute-like, causal) and 128 rows at its
-  // end (prompt-like, split over the whole context)
+  // attention over the resident context, when there is one: 1024
+  // recompute-like rows (causal) starting at the middle and at the start of
+  // the context -- two points that give a per-key rate and a per-row cost --
+  // and 128 prompt-like rows at its end (split over the whole context)
   {
     const int64_t n_ctx = ctx->st.n_ctx();
     bool resident = n_ctx >= 2048;
@@ -1026,9 +1030,11 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
       const mzc_model_shape& s = ctx->shape;
       std::vector<int32_t> tab;
       ctx->st.block_table(&tab);
-      for (int kind = 0; kind < 2; ++kind) {
-        const int64_t rows = std::min<int64_t>(ctx->max_rows, kind == 0 ? 1024 : 128);
-        const int64_t first = kind == 0 ? n_ctx / 2 : n_ctx - rows;
+      double t_sec[3] = {0, 0, 0}, pairs_k[3] = {0, 0, 0};
+      int64_t rows_k[3] = {0, 0, 0};
+      for (int kind = 0; kind < 3; ++kind) {
+        const int64_t rows = std::min<int64_t>(ctx->max_rows, kind < 2 ? 1024 : 128);
+        const int64_t first = kind == 0 ? n_ctx / 2 : (kind == 1 ? 0 : n_ctx - rows);
         int32_t* hp = reinterpret_cast<int32_t*>(ctx->h_meta);
         for (int64_t i = 0; i < rows; ++i) hp[i] = static_cast<int32_t>(first + i);
         std::memcpy(hp + rows, tab.data(), ctx->nblk * 4);
@@ -1047,11 +1053,20 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
         CK(cudaEventRecord(b, ctx->cs));
         CK(cudaEventSynchronize(b));
         CK(cudaEventElapsedTime(&ms, a, b));
-        double pairs = 0;
-        for (int64_t i = 0; i < rows; ++i) pairs += static_cast<double>(first + i + 1);
-        const double flops = 3.0 * pairs * 4.0 * s.head_dim * s.n_q_heads;
-        if (ms > 0) (kind == 0 ? p.attn_tflops : p.attn_prompt_tflops) = flops / (ms * 1e-3) / 1e12;
+        for (int64_t i = 0; i < rows; ++i) pairs_k[kind] += static_cast<double>(first + i + 1);
+        t_sec[kind] = ms * 1e-3 / 3.0;
+        rows_k[kind] = rows;
       }
+      const double fpp = 4.0 * s.head_dim * s.n_q_heads;
+      if (t_sec[0] > t_sec[1] && pairs_k[0] > pairs_k[1] && rows_k[0] == rows_k[1]) {
+        const double sec_per_pair = (t_sec[0] - t_sec[1]) / (pairs_k[0] - pairs_k[1]);
+        p.attn_tflops = fpp / sec_per_pair / 1e12;
+        p.attn_row_ns = std::max(0.0, (t_sec[1] - pairs_k[1] * sec_per_pair) / rows_k[1] * 1e9);
+      } else if (t_sec[0] > 0) {
+        p.attn_tflops = pairs_k[0] * fpp / t_sec[0] / 1e12;
+        p.attn_row_ns = 0.0;
+      }
+      if (t_sec[2] > 0) p.attn_prompt_tflops = pairs_k[2] * fpp / t_sec[2] / 1e12;
     }
   }
   // memory-bound kernels per row (two RMSNorms and the rotary/KV write,

@@ -51,7 +51,8 @@ class mzc_weights(ctypes.Structure):
 
 class mzc_profile(ctypes.Structure):
     _fields_ = [("h2d_gbs", c_f64), ("gemm_us_128", c_f64), ("gemm_us_512", c_f64),
-                ("gemm_us_2048", c_f64), ("attn_tflops", c_f64), ("attn_prompt_tflops", c_f64),
+                ("gemm_us_2048", c_f64), ("attn_tflops", c_f64), ("attn_row_ns", c_f64),
+                ("attn_prompt_tflops", c_f64),
                 ("row_ns", c_f64), ("layer_us", c_f64)]
 
 

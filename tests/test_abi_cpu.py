@@ -166,13 +166,14 @@ def test_restore_plan_packs_runs_forward_in():
 def _prof(h2d=200.0):
     # h2d GB/s, projections at 128/512/2048 rows (us), attention rates (TFLOP/s),
     # per-row ns, per-layer us
-    return M.mzc_profile(h2d, 110.0, 260.0, 700.0, 500.0, 600.0, 150.0, 15.0)
+    return M.mzc_profile(h2d, 110.0, 260.0, 700.0, 800.0, 2000.0, 600.0, 150.0, 15.0)
 
 
 def test_hybrid_split_bruteforce_and_limits():
     """The solver returns the block-aligned split minimising the documented
     cost (per layer: projections interpolated from their 128/512/2048-row
-    times, recompute and prompt attention pairs at their rates, per-row and
+    times, recompute attention pairs at their rate plus a per-row cost, prompt
+    attention pairs at their rate, per-row and
     per-layer costs; TTFT = max(compute, copy + 0.75 layer)), and stays at
     copy-only unless that saves at least 5%."""
     prof = _prof()
@@ -192,7 +193,7 @@ def test_hybrid_split_bruteforce_and_limits():
                 g = pr.gemm_us_512 + (rows - 512) * (pr.gemm_us_2048 - pr.gemm_us_512) / 1536
             rec = sum(range(p + 1, s + 1))
             prm = sum(range(n + 1, n + P + 1))
-            layer = (g * 1e-6 + rec * 4 * hd * hq / (pr.attn_tflops * 1e12)
+            layer = (g * 1e-6 + rec * 4 * hd * hq / (pr.attn_tflops * 1e12) + (s - p) * pr.attn_row_ns * 1e-9
                      + prm * 4 * hd * hq / (pr.attn_prompt_tflops * 1e12)
                      + rows * pr.row_ns * 1e-9 + pr.layer_us * 1e-6)
         copy = -(-(n - s) // 16) * L * 2 * hkv * 16 * hd * 2 / (pr.h2d_gbs * 1e9)

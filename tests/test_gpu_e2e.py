@@ -153,7 +153,7 @@ def test_repeat_with_truncate_is_deterministic(tiny):
 
 
 def test_auto_policies_match(tiny):
-    prof = m.mzc_profile(200.0, 110.0, 260.0, 700.0, 500.0, 600.0, 150.0, 15.0)
+    prof = m.mzc_profile(200.0, 110.0, 260.0, 700.0, 800.0, 2000.0, 600.0, 150.0, 15.0)
     res = {}
     for pol in (m.MZC_POLICY_COPY, m.MZC_POLICY_RECOMPUTE, m.MZC_POLICY_HYBRID):
         c = _new(tiny)
