@@ -6,26 +6,34 @@
 // (hq/hkv) query heads that share g are flattened token-major (row r = token
 // r / group, head g*group + r % group), so every K/V tile serves both Q tiles
 // and `group` heads.  Per BN-key tile of its key range:
-//   - warp 8 (one thread) looks each 16-token block of the tile up in the
-//     block table and fetches its K and V rows with TMA (a 16-row box per
-//     block and 64-column slice, 128-byte swizzle) into a 3-stage ring;
-//   - warp 9 (one thread) issues tcgen05.mma: S_t = Q_t K^T for both Q tiles
-//     into their TMEM S buffers (M=128, N=BN, K-major operands), and, once a
-//     softmax warpgroup has written P_t, O_t += P_t V into that tile's TMEM
-//     accumulator (A = P K-major, B = V MN-major, V in its stored layout);
+//   - warp 8 looks the tile's 16-token blocks up in the block table (one lane
+//     per block, a tile ahead) and fetches their K and V rows with TMA into a
+//     4-5-stage ring, 128-byte swizzle: one box per 64-column slice when the
+//     blocks are consecutive in the pool, else one 16-row box per block;
+//   - warps 9 and 10 (one thread each, one per Q tile t, so neither tile's
+//     UMMAs queue behind the other's waits) issue tcgen05.mma: S_t = Q_t K^T
+//     into the tile's TMEM S buffer (M=128, N=BN, K-major operands from shared
+//     memory), and, once its softmax warpgroup has written P_t, O_t += P_t V
+//     into the tile's TMEM accumulator with P_t read from TMEM (A operand) and
+//     V from shared memory as an MN-major operand in its stored layout;
 //   - warps 0-3 and 4-7 are the softmax warpgroups of the two Q tiles, one
 //     thread per row: the whole S row comes out of TMEM (the S buffer is
 //     released right away, so the next S runs on the tensor cores during the
 //     exponentials), is masked by the row's position on diagonal tiles,
-//     exponentiated in base 2 against a running reference maximum and stored
-//     as P (the KV type) into shared memory in the UMMA K-major swizzled
-//     layout.  O is rescaled in TMEM only when the maximum grows by more than
-//     2^8 ("lazy" rescale), so P stays <= 256.  The two warpgroups never wait
-//     for each other, so one exponentiates while the other waits on its S.
+//     exponentiated in base 2 against a running reference maximum into fp16
+//     registers, and written as P into its TMEM columns once the previous P V
+//     has released them.  O is rescaled in TMEM only when the maximum grows by
+//     more than 2^8 ("lazy" rescale), so P stays <= 256.  The two warpgroups
+//     never wait for each other, so one exponentiates while the other waits on
+//     its S.
+// Keeping P in TMEM leaves shared-memory bandwidth to the K/V operands: at
+// head dim 64 an M=128 x N=64 P V with P in shared memory reads more bytes
+// per FLOP than the tensor core consumes.
 // Long key ranges with few rows are split across CTAs (split-KV); each split
 // writes its normalised partial output and base-2 log-sum-exp, and a combine
 // kernel merges them.
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <mutex>
 
@@ -37,24 +45,27 @@ namespace mzc {
 namespace {
 
 constexpr int kRowsPerCta = 256;  // two Q tiles of 128 rows
+constexpr int kThreads = 352;     // 8 softmax warps, TMA producer, 2 UMMA issuers
 
 template <int HD>
 struct AttnCfg {
   static constexpr int BM = 128;                  // rows per Q tile (TMEM lanes)
   static constexpr int BN = HD == 64 ? 128 : 64;  // keys per tile
-  static constexpr int STAGES = 3;
+  static constexpr int STAGES = HD == 64 ? 5 : 4;
   static constexpr int CB = HD / 64;              // 64-column slices of the head dim
   static constexpr int Q_BYTES = BM * HD * 2;     // one Q tile
   static constexpr int KV_BYTES = BN * HD * 2;    // K or V of one key tile
-  static constexpr int P_BYTES = BM * BN * 2;     // one P tile
   static constexpr int OFF_K = 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
-  static constexpr int OFF_P = OFF_V + STAGES * KV_BYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;  // + barriers + alignment slack
-  // TMEM columns: S of tile t at t*BN, O of tile t at 2*BN + t*HD
-  static constexpr uint32_t O_COL = 2 * BN;
+  // TMEM columns: S of tile t at t*BN (fp32), P of tile t at P_COL + t*BN/2
+  // (fp16 pairs), O of tile t at O_COL + t*HD (fp32)
+  static constexpr uint32_t P_COL = 2 * BN;
+  static constexpr uint32_t O_COL = 3 * BN;
   static constexpr uint32_t TMEM_COLS = 512;
+  static_assert(O_COL + 2 * HD <= TMEM_COLS, "S, P and O of both tiles fit in TMEM");
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 // kind::f16 instruction descriptor: fp32 D, A/B fp16 (or bf16), A K-major,
@@ -82,6 +93,37 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// Packed fp32 pairs (two registers as one 64-bit operand) for the f32x2 FMA
+// and add of the softmax: half the instructions of scalar fp32.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
+}
+
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// max(a, b, c) in one instruction
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 __device__ __forceinline__ void fence_async_smem() {
@@ -131,12 +173,14 @@ __device__ __forceinline__ void tmem_st_row(uint32_t taddr, const float* v) {
 
 // Threads: warps 0-3 and 4-7 are the softmax warpgroups of Q tiles 0 and 1
 // (thread = row of its tile, whole rows of S), warp 8 is the TMA producer and
-// TMEM owner, warp 9 issues the UMMAs.  Both Q tiles share every K/V tile.
+// TMEM owner, warps 9 and 10 issue the UMMAs of Q tiles 0 and 1.  Both Q tiles
+// share every K/V tile.
 template <int HD, bool F16>
-__global__ void __launch_bounds__(320, 1) attn_tc_kernel(
+__global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
     const uint16_t* __restrict__ q, const int32_t* __restrict__ pos, int n, int hq, int hkv,
     const int32_t* __restrict__ table, int64_t n_logical,
-    const __grid_constant__ CUtensorMap pool_map, int64_t pool_blocks,
+    const __grid_constant__ CUtensorMap pool_run, const __grid_constant__ CUtensorMap pool_blk,
+    int64_t pool_blocks,
     uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
     int keys_per_split, int n_splits, float scale_log2, int32_t* status) {
   using C = AttnCfg<HD>;
@@ -147,14 +191,13 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
   uint8_t* sQ = smem;  // [2 tiles]
   uint8_t* sK = smem + C::OFF_K;
   uint8_t* sV = smem + C::OFF_V;
-  uint8_t* sP = smem + C::OFF_P;  // [2 tiles]
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* k_full = bars;                    // [STAGES]
   uint64_t* v_full = bars + C::STAGES;        // [STAGES]
   uint64_t* kv_empty = bars + 2 * C::STAGES;  // [STAGES]
   uint64_t* s_full = bars + 3 * C::STAGES;    // [2 tiles] S(j) in TMEM
   uint64_t* s_free = s_full + 2;              // [2 tiles] S(j) read into registers
-  uint64_t* p_full = s_free + 2;              // [2 tiles] P(j) in shared memory
+  uint64_t* p_full = s_free + 2;              // [2 tiles] P(j) in TMEM
   uint64_t* p_free = p_full + 2;              // [2 tiles] P(j) V(j) done
   __shared__ uint32_t s_tmem;
   __shared__ int s_maxpos;
@@ -172,7 +215,7 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&kv_empty[s], 2);  // both Q tiles' P V done
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(&s_full[t], 1);
@@ -183,7 +226,8 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
     fence_barrier_init();
     s_maxpos = -1;
     s_abort = 0;
-    tma_prefetch_desc(&pool_map);
+    tma_prefetch_desc(&pool_run);
+    tma_prefetch_desc(&pool_blk);
   }
   if (warp == 8) tmem_alloc(&s_tmem, C::TMEM_COLS);
 
@@ -222,121 +266,126 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
   const int T = k_end > k_begin ? (k_end - k_begin + BN - 1) / BN : 0;
 
   if (warp == 8) {
-    if (lane == 0 && T > 0) {
-      // ---- TMA producer ----
-      const int64_t head_rows = static_cast<int64_t>(hkv) * 16;
+    if (T > 0) {
+      // ---- TMA producer (whole warp): lane b looks up block b of a key tile,
+      // one tile ahead of its use, so the table reads overlap the copies ----
+      constexpr int NB = BN / 16;
+      constexpr int32_t kPast = INT32_MIN;  // block past the key range
+      const int32_t yk = g * 16, yv = (hkv + g) * 16;
+      auto lookup = [&](int j) -> int32_t {
+        const int key0 = k_begin + j * BN + lane * 16;
+        if (lane >= NB || key0 >= k_end) return kPast;
+        const int64_t blk = key0 >> 4;
+        return blk < n_logical ? table[blk] : -1;
+      };
+      int32_t p_cur = lookup(0);
       int issued = 0;
       for (int j = 0; j < T; ++j) {
         const int s = j % C::STAGES;
-        const int kb = k_begin + j * BN;
-        int32_t phys[BN / 16];
-        int32_t first = -1;
+        const int32_t p_nxt = j + 1 < T ? lookup(j + 1) : kPast;
+        int32_t p = p_cur;
+        if (p != kPast && (p < 0 || p >= pool_blocks)) {
+          set_status(status, kStatusDevice);  // its keys read another block
+          p = kPast;
+        }
+        const bool valid = p != kPast;
+        const int32_t first_raw = __shfl_sync(0xffffffffu, p, 0);
+        const int32_t first = first_raw < 0 ? 0 : first_raw;
+        // the tile's blocks are consecutive in the pool: one box per operand slice
+        // (blocks past the key range are read too; their keys are masked)
+        const bool run = __all_sync(0xffffffffu, !valid || p == first + lane);
+        const int32_t mine = valid ? p : first;
+        bool ok = true;
+        if (lane == 0 && j >= C::STAGES)
+          ok = wait_bar(&kv_empty[s], ((j / C::STAGES) - 1) & 1, status, abort_flag);
+        if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&k_full[s], C::KV_BYTES);
+          mbar_arrive_expect_tx(&v_full[s], C::KV_BYTES);
+        }
+        __syncwarp();
+        if (run) {
+          if (lane == 0) {
 #pragma unroll
-        for (int b = 0; b < BN / 16; ++b) {
-          const int key0 = kb + b * 16;
-          int32_t p = -1;
-          if (key0 < k_end) {
-            const int64_t blk = key0 >> 4;
-            p = blk < n_logical ? table[blk] : -1;
-            if (p < 0 || p >= pool_blocks) {
-              set_status(status, kStatusDevice);
-              p = -1;
+            for (int c = 0; c < C::CB; ++c) {
+              tma_load_3d(sK + s * C::KV_BYTES + c * (BN * 128), &pool_run, &k_full[s], c * 64, yk, first);
+              tma_load_3d(sV + s * C::KV_BYTES + c * (BN * 128), &pool_run, &v_full[s], c * 64, yv, first);
             }
           }
-          if (b == 0) first = p < 0 ? 0 : p;
-          // blocks past the key range: any valid block (its keys are masked)
-          phys[b] = p < 0 ? first : p;
-        }
-        if (j >= C::STAGES &&
-            !wait_bar(&kv_empty[s], ((j / C::STAGES) - 1) & 1, status, abort_flag))
-          break;
-        mbar_arrive_expect_tx(&k_full[s], C::KV_BYTES);
+        } else if (lane < NB) {
 #pragma unroll
-        for (int b = 0; b < BN / 16; ++b) {
-          const int32_t y = static_cast<int32_t>((static_cast<int64_t>(phys[b]) * 2) * head_rows + g * 16);
-#pragma unroll
-          for (int c = 0; c < C::CB; ++c)
-            tma_load_2d(sK + s * C::KV_BYTES + c * (BN * 128) + b * 16 * 128, &pool_map,
-                        &k_full[s], c * 64, y);
-        }
-        mbar_arrive_expect_tx(&v_full[s], C::KV_BYTES);
-#pragma unroll
-        for (int b = 0; b < BN / 16; ++b) {
-          const int32_t y = static_cast<int32_t>((static_cast<int64_t>(phys[b]) * 2 + 1) * head_rows + g * 16);
-#pragma unroll
-          for (int c = 0; c < C::CB; ++c)
-            tma_load_2d(sV + s * C::KV_BYTES + c * (BN * 128) + b * 16 * 128, &pool_map,
-                        &v_full[s], c * 64, y);
+          for (int c = 0; c < C::CB; ++c) {
+            tma_load_3d(sK + s * C::KV_BYTES + c * (BN * 128) + lane * 16 * 128, &pool_blk, &k_full[s],
+                        c * 64, yk, mine);
+            tma_load_3d(sV + s * C::KV_BYTES + c * (BN * 128) + lane * 16 * 128, &pool_blk, &v_full[s],
+                        c * 64, yv, mine);
+          }
         }
         issued = j + 1;
+        p_cur = p_nxt;
       }
       // drain: every fill issued has landed before shared memory is released
-      for (int j = issued - C::STAGES < 0 ? 0 : issued - C::STAGES; j < issued; ++j) {
-        wait_bar(&k_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
-        wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+      if (lane == 0) {
+        for (int j = issued - C::STAGES < 0 ? 0 : issued - C::STAGES; j < issued; ++j) {
+          wait_bar(&k_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+          wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+        }
       }
     }
-  } else if (warp == 9) {
+  } else if (warp >= 9) {
+    // ---- UMMA issuers, one per Q tile t: S_t(j+1), then P_t V(j) ----
+    const int t = warp - 9;
     if (lane == 0 && T > 0) {
-      // ---- UMMA issuer: S_0(j+1), S_1(j+1), P_0 V(j), P_1 V(j) ----
       constexpr uint32_t id_s = idesc_attn<F16>(128, BN, false);
       constexpr uint32_t id_o = idesc_attn<F16>(128, HD, true);
-      auto issue_s = [&](int t, int j) {
-        const int s = j % C::STAGES;
+      const uint32_t q_base = smem_u32(sQ + t * C::Q_BYTES);
+      const uint32_t k_base = smem_u32(sK), v_base = smem_u32(sV);
+      const uint32_t s_tm = tmem + t * BN, p_tm = tmem + C::P_COL + t * (BN / 2);
+      const uint32_t o_tm = tmem + C::O_COL + t * HD;
+      auto issue_s = [&](int j) {
+        const uint32_t kst = k_base + (j % C::STAGES) * C::KV_BYTES;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
           const int cb = kk >> 2, w = kk & 3;
-          const uint64_t ad = sdesc_k_sw128(smem_u32(sQ + t * C::Q_BYTES + cb * (C::BM * 128) + w * 32));
-          const uint64_t bd = sdesc_k_sw128(smem_u32(sK + s * C::KV_BYTES + cb * (BN * 128) + w * 32));
-          umma_f16(tmem + t * BN, ad, bd, id_s, kk > 0 ? 1u : 0u);
+          umma_f16(s_tm, sdesc_k_sw128(q_base + cb * (C::BM * 128) + w * 32),
+                   sdesc_k_sw128(kst + cb * (BN * 128) + w * 32), id_s, kk > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[t]);
       };
-      auto issue_pv = [&](int t, int j) {
+      auto issue_pv = [&](int j) {
         const int s = j % C::STAGES;
+        const uint32_t vst = v_base + s * C::KV_BYTES;
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const int pcb = kk >> 2, w = kk & 3;
-          const uint64_t ad = sdesc_k_sw128(smem_u32(sP + t * C::P_BYTES + pcb * (C::BM * 128) + w * 32));
-          const uint64_t bd = sdesc_mn_sw128(smem_u32(sV + s * C::KV_BYTES + kk * 16 * 128), BN * 128);
-          umma_f16(tmem + C::O_COL + t * HD, ad, bd, id_o, (j > 0 || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < BN / 16; ++kk)
+          umma_f16_ts(o_tm, p_tm + kk * 8, sdesc_mn_sw128(vst + kk * 16 * 128, BN * 128), id_o,
+                      (j > 0 || kk > 0) ? 1u : 0u);
         umma_commit(&p_free[t]);
+        umma_commit(&kv_empty[s]);
       };
       bool ok = wait_bar(&k_full[0], 0, status, abort_flag);
       if (ok) {
         tc_fence_after();
-        issue_s(0, 0);
-        issue_s(1, 0);
+        issue_s(0);
       }
       for (int j = 0; ok && j < T; ++j) {
-        const int s = j % C::STAGES;
         const uint32_t ph = j & 1;
         if (j + 1 < T) {
-          // the next S of each tile runs while the softmax exponentiates S(j)
+          // the next S runs while the softmax exponentiates S(j)
           if (!wait_bar(&k_full[(j + 1) % C::STAGES], ((j + 1) / C::STAGES) & 1, status, abort_flag)) break;
-          if (!wait_bar(&s_free[0], ph, status, abort_flag)) break;
+          if (!wait_bar(&s_free[t], ph, status, abort_flag)) break;
           tc_fence_after();
-          issue_s(0, j + 1);
-          if (!wait_bar(&s_free[1], ph, status, abort_flag)) break;
-          tc_fence_after();
-          issue_s(1, j + 1);
+          issue_s(j + 1);
         }
-        if (!wait_bar(&v_full[s], (j / C::STAGES) & 1, status, abort_flag)) break;
-        if (!wait_bar(&p_full[0], ph, status, abort_flag)) break;
+        if (!wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag)) break;
+        if (!wait_bar(&p_full[t], ph, status, abort_flag)) break;
         tc_fence_after();
-        issue_pv(0, j);
-        if (!wait_bar(&p_full[1], ph, status, abort_flag)) break;
-        tc_fence_after();
-        issue_pv(1, j);
-        umma_commit(&kv_empty[s]);
+        issue_pv(j);
       }
     }
   } else {
     // ---- softmax: thread = row of Q tile qt, all BN columns ----
     const uint32_t trow = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-    const uint32_t s_col = qt * BN, o_col = C::O_COL + qt * HD;
-    uint8_t* prow = sP + qt * C::P_BYTES + row * 128;
+    const uint32_t s_col = qt * BN, p_col = C::P_COL + qt * (BN / 2), o_col = C::O_COL + qt * HD;
     float m_ref = -INFINITY, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < T && ok; ++j) {
@@ -363,15 +412,33 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
           if (!(key <= row_pos && key < k_end)) v[i] = -INFINITY;
         }
       }
-      float mx[8];
+      float mx[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = v[i];
+      for (int a = 0; a < 4; ++a) mx[a] = fmaxf(v[2 * a], v[2 * a + 1]);
 #pragma unroll
-      for (int i = 8; i < BN; ++i) mx[i & 7] = fmaxf(mx[i & 7], v[i]);
-      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * scale_log2;
+      for (int i = 8; i < BN; i += 8) {
+#pragma unroll
+        for (int a = 0; a < 4; ++a) mx[a] = fmax3(mx[a], v[i + 2 * a], v[i + 2 * a + 1]);
+      }
+      const float tmax = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]) * scale_log2;
       const float m_new = fmaxf(m_ref, tmax);
       const bool need = m_new > m_ref + 8.0f;
+      const float m_old = m_ref;
+      if (need) m_ref = m_new;
+      const float nbase = m_ref == -INFINITY ? 0.0f : -m_ref;
+      // P(j) goes to registers first, so the exponentials run while P(j-1) V(j-1)
+      // still reads the P buffer
+      uint32_t pk[BN / 2];
+      const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nb2 = f2_pack(nbase, nbase);
+      uint64_t ls2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
+#pragma unroll
+      for (int i = 0; i < BN / 2; ++i) {
+        float x0, x1;
+        f2_unpack(f2_fma(f2_pack(v[2 * i], v[2 * i + 1]), sc2, nb2), x0, x1);
+        const float p0 = ex2(x0), p1 = ex2(x1);
+        ls2[i & 1] = f2_add(ls2[i & 1], f2_pack(p0, p1));
+        pk[i] = pack2<F16>(p0, p1);
+      }
       // P(j-1) V(j-1) must be done before O is rebased or P is overwritten
       if (j > 0) {
         ok = wait_bar(&p_free[qt], (j - 1) & 1, status, abort_flag);
@@ -381,10 +448,8 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
           break;
         }
         tc_fence_after();
-      }
-      if (__any_sync(0xffffffffu, need)) {
-        if (j > 0) {
-          const float alpha = need ? ex2(m_ref - m_new) : 1.0f;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = need ? ex2(m_old - m_ref) : 1.0f;
 #pragma unroll 1
           for (int c = 0; c < HD; c += 32) {
             float o[32];
@@ -395,28 +460,19 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(
           }
           l *= alpha;
         }
-        if (need) m_ref = m_new;
       }
-      const float nbase = m_ref == -INFINITY ? 0.0f : -m_ref;
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int u = 0; u < BN / 8; ++u) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p0 = ex2(fmaf(v[8 * u + 2 * e], scale_log2, nbase));
-          const float p1 = ex2(fmaf(v[8 * u + 2 * e + 1], scale_log2, nbase));
-          ls[e] += p0 + p1;
-          pk[e] = pack2<F16>(p0, p1);
-        }
-        // keys [8u, 8u+8) of this row in the swizzled K-major P tile
-        uint8_t* slice = prow + (u >> 3) * (C::BM * 128);
-        *reinterpret_cast<uint4*>(slice + (((u & 7) ^ (row & 7)) << 4)) =
-            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      {
+        float a0, a1, b0, b1;
+        f2_unpack(ls2[0], a0, a1);
+        f2_unpack(ls2[1], b0, b1);
+        l += (a0 + a1) + (b0 + b1);
       }
-      l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      fence_async_smem();  // P visible to the tensor core
-      tc_fence_before();
+      if constexpr (BN == 128) {
+        tmem_st64w_u32(trow + p_col, pk);
+      } else {
+        tmem_st32w_u32(trow + p_col, pk);
+      }
+      tc_fence_before();  // P in TMEM before the issuer's P V
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[qt]);
     }
@@ -521,23 +577,26 @@ EncodeFn encode_fn() {
   return fn;
 }
 
-// The pool as a 2-D tensor of 16-bit elements: [pool_blocks * 2 * hkv * 16 rows][hd],
-// read in boxes of 16 rows x 64 columns with 128-byte swizzle.
-bool make_pool_map(CUtensorMap* map, const void* pool, int64_t pool_blocks, int hkv, int hd) {
+// The pool as a 3-D tensor of 16-bit elements: [pool_blocks][2 * hkv * 16 rows][hd]
+// (K rows of every head, then V rows), read in boxes of `depth` blocks x 16 rows
+// (one head) x 64 columns with 128-byte swizzle.
+bool make_pool_map(CUtensorMap* map, const void* pool, int64_t pool_blocks, int hkv, int hd,
+                   int depth) {
   EncodeFn fn = encode_fn();
   if (!fn) return false;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(hd), static_cast<cuuint64_t>(pool_blocks) * 2 * hkv * 16};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(hd) * 2};
-  cuuint32_t box[2] = {64, 16};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<void*>(pool), dims, strides, box,
+  const cuuint64_t rows = static_cast<cuuint64_t>(2) * hkv * 16;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(hd), rows, static_cast<cuuint64_t>(pool_blocks)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(hd) * 2, rows * hd * 2};
+  cuuint32_t box[3] = {64, 16, static_cast<cuuint32_t>(depth)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, const_cast<void*>(pool), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int HD, bool F16>
 cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
-                      const int32_t* table, int64_t n_logical, const CUtensorMap& map,
+                      const int32_t* table, int64_t n_logical, const void* pool,
                       int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
                       int n_splits, int keys_per_split, int32_t* status, cudaStream_t st) {
   using C = AttnCfg<HD>;
@@ -548,14 +607,18 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   });
   if (attr_err != cudaSuccess) return attr_err;
+  CUtensorMap run_map, blk_map;
+  if (!make_pool_map(&run_map, pool, pool_blocks, hkv, HD, C::BN / 16) ||
+      !make_pool_map(&blk_map, pool, pool_blocks, hkv, HD, 1))
+    return cudaErrorInvalidValue;
   const int group = hq / hkv;
   const int64_t R = n * group;
   dim3 grid(static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta), static_cast<unsigned>(hkv),
             static_cast<unsigned>(n_splits));
   const float scale_log2 =
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
-  attn_tc_kernel<HD, F16><<<grid, 320, C::SMEM, st>>>(
-      q, pos, static_cast<int>(n), hq, hkv, table, n_logical, map, pool_blocks, out, part_o,
+  attn_tc_kernel<HD, F16><<<grid, kThreads, C::SMEM, st>>>(
+      q, pos, static_cast<int>(n), hq, hkv, table, n_logical, run_map, blk_map, pool_blocks, out, part_o,
       part_lse, keys_per_split, n_splits, scale_log2, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || n_splits == 1) return e;
@@ -611,16 +674,14 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
     s = 1;
     per = static_cast<int>((max_keys + 127) / 128 * 128);
   }
-  CUtensorMap map;
-  if (!make_pool_map(&map, pool, pool_blocks, hkv, hd)) return cudaErrorInvalidValue;
   float* part_o = static_cast<float*>(scratch);
   float* part_lse = s > 1 ? part_o + static_cast<int64_t>(s) * n * hq * hd : nullptr;
   (void)kv_dtype;  // the pool is fp16-encoded for both KV types: q, K, P, V are fp16
   if (hd == 64)
-    return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
+    return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
                                part_o, part_lse, s, per, status, st);
   if (hd == 128)
-    return launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, map, pool_blocks, out,
+    return launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
                                 part_o, part_lse, s, per, status, st);
   return cudaErrorInvalidValue;
 }
