@@ -12,7 +12,11 @@
 //   EPI_ADD_F32     out fp32 += C                     (O / down projection + residual)
 //   EPI_SWIGLU_BF16 out fp16 = silu(C_gate) * C_up    (gate/up projection, rows interleaved
 //                                                     in groups of 64, see kSwigluGroup)
-// Rows >= m are computed on whatever the A buffer holds and never stored.
+// writing each 32-row x 128-byte piece to shared memory and out with a TMA
+// store (fp16) or a TMA reduce-add (the fp32 residual: the add happens in L2,
+// one fp32 add per element as in a read-modify-write).  The output tensor map
+// spans exactly m rows and n columns, so rows >= m (computed on whatever the A
+// buffer holds) are clipped by the TMA unit.
 #include <cstdio>
 #include <mutex>
 
@@ -46,7 +50,11 @@ struct PCfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  // epilogue staging: per epilogue warp two 32-row x 128-byte boxes
+  static constexpr int OUT_BOX = 32 * 128;
+  static constexpr int OFF_OUT = STAGES * STAGE_BYTES;
+  static constexpr int OFF_BAR = OFF_OUT + 4 * 2 * OUT_BOX;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 };
 
@@ -76,14 +84,15 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int*
 template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw,
-    void* __restrict__ out, int m, int n, int k, int32_t* status) {
+    const __grid_constant__ CUtensorMap tmo, int m, int n, int k, int32_t* status) {
   using C = PCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint8_t* sOut = smem + C::OFF_OUT;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* empty = full + STAGES;
   uint64_t* acc_full = empty + STAGES;  // [2]
   uint64_t* acc_empty = acc_full + 2;   // [2]
@@ -99,6 +108,7 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tma);
     tma_prefetch_desc(&tmw);
+    tma_prefetch_desc(&tmo);
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
@@ -169,78 +179,100 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
       }
     }
   } else {
-    // ---- epilogue warps 2-5 ----
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    // ---- epilogue warps 2-5: TMEM -> registers -> swizzled staging box -> TMA ----
+    // Warp q owns rows q*32..+31 of the tile (its TMEM lane quarter) and two
+    // 32 x 128-byte staging boxes; lane = row.  Each box goes out as one TMA
+    // store (fp16 outputs) or TMA reduce-add into the fp32 residual stream, so
+    // the epilogue never reads the output and writes whole 128-byte lines.
+    const int q = warp & 3;
+    uint8_t* box0 = sOut + q * 2 * C::OUT_BOX;
+    int nbox = 0;  // boxes issued by this warp (buffer = nbox & 1)
+    // one staging row: 8 16-byte units, unit u at u ^ (row & 7) (128-byte swizzle)
+    auto stage_row = [&](const uint32_t* w) -> uint8_t* {
+      uint8_t* box = box0 + (nbox & 1) * C::OUT_BOX;
+      if (lane == 0 && nbox >= 2) bulk_wait_read<1>();  // the store that last used this box
+      __syncwarp();
+      uint8_t* r = box + lane * 128;
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        *reinterpret_cast<uint4*>(r + ((u ^ (lane & 7)) << 4)) =
+            make_uint4(w[4 * u], w[4 * u + 1], w[4 * u + 2], w[4 * u + 3]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      return box;
+    };
     int local = 0;
+    bool ok = true;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
       const int a = local & 1;
-      bool ok = pwait(&acc_full[a], (local >> 1) & 1, status, abort_flag);
+      ok = ok && pwait(&acc_full[a], (local >> 1) & 1, status, abort_flag);
       __syncwarp();
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
       int mt, nt;
       tile_coords(tile, num_m, num_n, &mt, &nt);
-      const int row = mt * BM + q * 32 + lane;
+      const int y = mt * BM + q * 32;
       const uint32_t trow = tmem + a * BN + (static_cast<uint32_t>(q * 32) << 16);
       const int n0 = nt * BN;
       if constexpr (EPI == EPI_SWIGLU_BF16) {
-        const int nout = n / 2;
 #pragma unroll 1
         for (int g = 0; g < BN / (2 * kSwigluGroup); ++g) {
-#pragma unroll 1
+          uint32_t pk[32];
+#pragma unroll
           for (int c = 0; c < kSwigluGroup; c += 32) {
             float vg[32], vu[32];
             tmem_ld32w(trow + g * 2 * kSwigluGroup + c, vg);
             tmem_ld32w(trow + g * 2 * kSwigluGroup + kSwigluGroup + c, vu);
-            const int col = n0 / 2 + g * kSwigluGroup + c;
-            if (row < m && col < nout) {
-              uint32_t pk[16];
 #pragma unroll
-              for (int i = 0; i < 16; ++i)
-                pk[i] = pack2<true>(silu_f(vg[2 * i]) * vu[2 * i], silu_f(vg[2 * i + 1]) * vu[2 * i + 1]);
-              uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + static_cast<size_t>(row) * nout + col);
-#pragma unroll
-              for (int i = 0; i < 4; ++i) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-            }
+            for (int i = 0; i < 16; ++i)
+              pk[c / 2 + i] = pack2<true>(silu_f(vg[2 * i]) * vu[2 * i], silu_f(vg[2 * i + 1]) * vu[2 * i + 1]);
           }
+          uint8_t* box = stage_row(pk);
+          if (lane == 0) {
+            if (y < m && n0 / 2 + g * kSwigluGroup < n / 2)
+              tma_store_2d(&tmo, box, n0 / 2 + g * kSwigluGroup, y);
+            bulk_commit();
+          }
+          ++nbox;
+        }
+      } else if constexpr (EPI == EPI_STORE_BF16) {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 64) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int h = 0; h < 64; h += 32) {
+            float v[32];
+            tmem_ld32w(trow + c + h, v);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) pk[h / 2 + i] = pack2<true>(v[2 * i], v[2 * i + 1]);
+          }
+          uint8_t* box = stage_row(pk);
+          if (lane == 0) {
+            if (y < m && n0 + c < n) tma_store_2d(&tmo, box, n0 + c, y);
+            bulk_commit();
+          }
+          ++nbox;
         }
       } else {
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
           float v[32];
           tmem_ld32w(trow + c, v);
-          const int col = n0 + c;
-          if (row < m && col < n) {
-            const int cnt = min(32, n - col);  // n is a multiple of 16
-            if constexpr (EPI == EPI_STORE_BF16) {
-              uint32_t pk[16];
-#pragma unroll
-              for (int i = 0; i < 16; ++i) pk[i] = pack2<true>(v[2 * i], v[2 * i + 1]);
-              uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + static_cast<size_t>(row) * n + col);
-#pragma unroll
-              for (int i = 0; i < 4; ++i)
-                if (i * 8 < cnt) o[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-            } else {
-              float4* o = reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<size_t>(row) * n + col);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                if (i * 4 < cnt) {
-                  float4 t = o[i];
-                  t.x += v[4 * i];
-                  t.y += v[4 * i + 1];
-                  t.z += v[4 * i + 2];
-                  t.w += v[4 * i + 3];
-                  o[i] = t;
-                }
-              }
-            }
+          uint8_t* box = stage_row(reinterpret_cast<const uint32_t*>(v));
+          if (lane == 0) {
+            if (y < m && n0 + c < n) tma_reduce_add_2d(&tmo, box, n0 + c, y);
+            bulk_commit();
           }
+          ++nbox;
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[a]);
     }
+    // every store has finished reading shared memory and reached global memory
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -249,29 +281,6 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     __syncwarp();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
-}
-
-template <int BN, int STAGES, int EPI>
-cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void* out, int64_t m,
-                              int64_t n, int64_t k, int32_t* status, cudaStream_t st) {
-  using C = PCfg<BN, STAGES>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  static int sms = 0;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_persistent_kernel<BN, STAGES, EPI>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-    int dev = 0;
-    if (attr_err == cudaSuccess) attr_err = cudaGetDevice(&dev);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  });
-  if (attr_err != cudaSuccess) return attr_err;
-  const int64_t tiles = ((m + BM - 1) / BM) * ((n + BN - 1) / BN);
-  const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
-  gemm_persistent_kernel<BN, STAGES, EPI><<<grid, 192, C::SMEM, st>>>(
-      ta, tw, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
-  return cudaGetLastError();
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -291,6 +300,49 @@ EncodeFn encode_fn() {
       fn = reinterpret_cast<EncodeFn>(p);
   });
   return fn;
+}
+
+// Output [rows][cols] (fp16, or fp32 for the residual stream) in boxes of
+// 32 rows x 128 bytes with 128-byte swizzle, matching the epilogue's staging.
+bool make_out_map(CUtensorMap* map, void* base, uint64_t rows, uint64_t cols, bool f32) {
+  EncodeFn fn = encode_fn();
+  if (!fn) return false;
+  const uint64_t esz = f32 ? 4 : 2;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * esz};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(128 / esz), 32};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base,
+            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int STAGES, int EPI>
+cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void* out, int64_t m,
+                              int64_t n, int64_t k, int32_t* status, cudaStream_t st) {
+  using C = PCfg<BN, STAGES>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  static int sms = 0;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(gemm_persistent_kernel<BN, STAGES, EPI>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    int dev = 0;
+    if (attr_err == cudaSuccess) attr_err = cudaGetDevice(&dev);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  CUtensorMap tmo;
+  const bool f32 = EPI == EPI_ADD_F32;
+  if (!make_out_map(&tmo, out, static_cast<uint64_t>(m),
+                    static_cast<uint64_t>(EPI == EPI_SWIGLU_BF16 ? n / 2 : n), f32))
+    return cudaErrorInvalidValue;
+  const int64_t tiles = ((m + BM - 1) / BM) * ((n + BN - 1) / BN);
+  const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
+  gemm_persistent_kernel<BN, STAGES, EPI><<<grid, 192, C::SMEM, st>>>(
+      ta, tw, tmo, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
+  return cudaGetLastError();
 }
 
 }  // namespace

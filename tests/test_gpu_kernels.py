@@ -84,6 +84,30 @@ def test_gemm_swiglu(mm, f, kk):
     assert np.all(err <= 2.0 ** -9 * np.abs(ref) + 2e-5 * np.max(np.abs(ref)))
 
 
+@pytest.mark.parametrize("epi", [0, 1, 2])
+@pytest.mark.parametrize("mm,nn", [(5, 128), (300, 384), (1000, 2048)])
+def test_gemm_writes_only_its_rows(epi, mm, nn):
+    """The epilogue's TMA stores are clipped at m rows: guard rows after the
+    output keep their sentinel, every row before it is written."""
+    torch = _torch()
+    kk = 128
+    a = _act16(9, (mm, kk))
+    _, wh = bf16_weights_exact_in_f16(_rand_bf16(10, (nn, kk), sigma=0.05))
+    ncol = nn // 2 if epi == 2 else nn
+    guard = 40
+    if epi == 1:
+        buf = torch.full((mm + guard, ncol), 7.0, dtype=torch.float32, device="cuda")
+    else:
+        buf = torch.full((mm + guard, ncol), 0x1234, dtype=torch.int16, device="cuda")
+    w = m.mzc_k_swiglu_pack(wh[: nn // 2], wh[nn // 2:]) if epi == 2 else wh
+    m.mzc_k_gemm(bf16_dev(a), bf16_dev(w), buf[:mm], mm, nn, kk, epi)
+    torch.cuda.synchronize()
+    host = buf.cpu().numpy()
+    sentinel = 7.0 if epi == 1 else 0x1234
+    assert np.all(host[mm:] == sentinel)
+    assert not np.any(np.all(host[:mm] == sentinel, axis=1))
+
+
 # ---- RMSNorm, embedding, LM head --------------------------------------------
 
 @pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072)])
