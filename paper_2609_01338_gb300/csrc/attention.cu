@@ -205,10 +205,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
   volatile int* abort_flag = &s_abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int g = blockIdx.y;
+  // grid: x = KV head, y = row tile counted from the last (the longest key
+  // ranges are dispatched first, so the shortest fill the tail of the grid)
+  const int g = blockIdx.x;
   const int group = hq / hkv;
   const int R = n * group;
-  const int r0 = blockIdx.x * kRowsPerCta;
+  const int r0 = (gridDim.y - 1 - blockIdx.y) * kRowsPerCta;
   const int split = blockIdx.z;
 
   if (tid == 0) {
@@ -412,15 +414,17 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
           if (!(key <= row_pos && key < k_end)) v[i] = -INFINITY;
         }
       }
-      float mx[4];
+      float mx[8];
 #pragma unroll
-      for (int a = 0; a < 4; ++a) mx[a] = fmaxf(v[2 * a], v[2 * a + 1]);
+      for (int a = 0; a < 8; ++a) mx[a] = fmaxf(v[2 * a], v[2 * a + 1]);
 #pragma unroll
-      for (int i = 8; i < BN; i += 8) {
+      for (int i = 16; i < BN; i += 16) {
 #pragma unroll
-        for (int a = 0; a < 4; ++a) mx[a] = fmax3(mx[a], v[i + 2 * a], v[i + 2 * a + 1]);
+        for (int a = 0; a < 8; ++a) mx[a] = fmax3(mx[a], v[i + 2 * a], v[i + 2 * a + 1]);
       }
-      const float tmax = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]) * scale_log2;
+      const float tmax =
+          fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) *
+          scale_log2;
       const float m_new = fmaxf(m_ref, tmax);
       const bool need = m_new > m_ref + 8.0f;
       const float m_old = m_ref;
@@ -613,8 +617,9 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
     return cudaErrorInvalidValue;
   const int group = hq / hkv;
   const int64_t R = n * group;
-  dim3 grid(static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta), static_cast<unsigned>(hkv),
-            static_cast<unsigned>(n_splits));
+  const int64_t row_tiles = (R + kRowsPerCta - 1) / kRowsPerCta;
+  if (row_tiles > 65535) return cudaErrorInvalidValue;
+  dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(row_tiles), static_cast<unsigned>(n_splits));
   const float scale_log2 =
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
   attn_tc_kernel<HD, F16><<<grid, kThreads, C::SMEM, st>>>(
