@@ -17,9 +17,11 @@
 //     into the tile's TMEM accumulator with P_t read from TMEM (A operand) and
 //     V from shared memory as an MN-major operand in its stored layout;
 //   - warps 0-3 and 4-7 are the softmax warpgroups of the two Q tiles, one
-//     thread per row: the whole S row comes out of TMEM (the S buffer is
-//     released right away, so the next S runs on the tensor cores during the
-//     exponentials), is masked by the row's position on diagonal tiles,
+//     thread per row: the whole S row comes out of TMEM together with its
+//     maximum (tcgen05.ld.red; the S buffer is released right away, so the
+//     next S runs on the tensor cores during the exponentials), is masked by
+//     the row's position on diagonal tiles (their maximum is then reduced in
+//     registers),
 //     exponentiated in base 2 against a running reference maximum into fp16
 //     registers, and written as P into its TMEM columns once the previous P V
 //     has released them.  O is rescaled in TMEM only when the maximum grows by
@@ -401,30 +403,38 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
       }
       tc_fence_after();
       float v[BN];
+      float hmax = -INFINITY;  // the row's maximum, reduced by the TMEM loads
 #pragma unroll
-      for (int c = 0; c < BN; c += 64) tmem_ld64w(trow + s_col + c, v + c);
+      for (int c = 0; c < BN; c += 64) {
+        float h;
+        tmem_ld64w_max(trow + s_col + c, v + c, h);
+        hmax = fmaxf(hmax, h);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_free[qt]);
       const bool full = __all_sync(0xffffffffu, (kb + BN - 1 <= row_pos) && (kb + BN <= k_end));
-      if (!full) {
+      float tmax;
+      if (full) {
+        tmax = hmax * scale_log2;
+      } else {
+        // diagonal or ragged tile: mask, then reduce in registers
 #pragma unroll
         for (int i = 0; i < BN; ++i) {
           const int key = kb + i;
           if (!(key <= row_pos && key < k_end)) v[i] = -INFINITY;
         }
+        float mx[8];
+#pragma unroll
+        for (int a = 0; a < 8; ++a) mx[a] = fmaxf(v[2 * a], v[2 * a + 1]);
+#pragma unroll
+        for (int i = 16; i < BN; i += 16) {
+#pragma unroll
+          for (int a = 0; a < 8; ++a) mx[a] = fmax3(mx[a], v[i + 2 * a], v[i + 2 * a + 1]);
+        }
+        tmax = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) *
+               scale_log2;
       }
-      float mx[8];
-#pragma unroll
-      for (int a = 0; a < 8; ++a) mx[a] = fmaxf(v[2 * a], v[2 * a + 1]);
-#pragma unroll
-      for (int i = 16; i < BN; i += 16) {
-#pragma unroll
-        for (int a = 0; a < 8; ++a) mx[a] = fmax3(mx[a], v[i + 2 * a], v[i + 2 * a + 1]);
-      }
-      const float tmax =
-          fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) *
-          scale_log2;
       const float m_new = fmaxf(m_ref, tmax);
       const bool need = m_new > m_ref + 8.0f;
       const float m_old = m_ref;
