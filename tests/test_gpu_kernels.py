@@ -110,7 +110,7 @@ def test_gemm_writes_only_its_rows(epi, mm, nn):
 
 # ---- RMSNorm, embedding, LM head --------------------------------------------
 
-@pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072)])
+@pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072), (5, 320), (3, 4608), (9, 4096)])
 def test_rmsnorm(n, d):
     torch = _torch()
     rng = np.random.default_rng(n)
