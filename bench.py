@@ -457,18 +457,20 @@ def run_sweep(r, args, rank):
     for frac in r.sc["fractions"]:
         for pol in r.sc["policies"]:
             vals, comp, copy = [], [], []
-            m.mzc_set_kernel_timing(r.c, 0)
+            # per-kernel events only in the last warm-up step (they would
+            # otherwise add to the timed steps)
+            ks = {}
             for i in range(args.warmup + args.steps):
-                if i == args.warmup:
-                    m.mzc_set_kernel_timing(r.c, -1)
+                m.mzc_set_kernel_timing(r.c, -1 if i == args.warmup - 1 else 0)
                 r.evict(pol, frac)
                 d, h, st, times = r.step()
+                if i == args.warmup - 1:
+                    ks = {nm: round(m.mzc_kernel_stats(r.c, j).ms, 3)
+                          for j, nm in enumerate(m.KERNEL_CLASS_NAMES)}
                 if i >= args.warmup:
                     vals.append(d)
                     comp.append(float(times[0]))
                     copy.append(float(times[1]))
-            ks = {nm: round(m.mzc_kernel_stats(r.c, j).ms / args.steps, 3)
-                  for j, nm in enumerate(m.KERNEL_CLASS_NAMES)}
             m.mzc_set_kernel_timing(r.c, 0)
             pt = {"fraction": frac, "policy": pol, "ttft_ms": round(statistics.median(vals), 3),
                   "p10": round(float(np.percentile(vals, 10)), 3),

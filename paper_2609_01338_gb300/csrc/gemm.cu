@@ -361,9 +361,31 @@ bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 }
 
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue) {
-  (void)n;
-  if (m > 512) return 256;                        // persistent 128 x 256 tiles
-  return epilogue == EPI_SWIGLU_BF16 ? 128 : 64;  // persistent narrow tiles, deep ring
+  if (m > 512) return 256;  // tensor-bound: 128 x 256 tiles
+  // Weight-streaming bound: the tile width with the fewest waves over the SMs
+  // and, among those, the most tiles (the most SMs pulling weight bytes).
+  // SwiGLU tiles hold whole 128-row gate/up groups.
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 1;
+  }
+  const int64_t mt = (m + BM - 1) / BM;
+  uint32_t best = 256;
+  int64_t best_waves = 0, best_tiles = 0;
+  for (uint32_t bn : {256u, 128u, 64u}) {
+    if (epilogue == EPI_SWIGLU_BF16 && bn < 128) continue;
+    const int64_t tiles = mt * ((n + bn - 1) / bn);
+    const int64_t waves = (tiles + sms - 1) / sms;
+    if (best_tiles == 0 || waves < best_waves || (waves == best_waves && tiles > best_tiles)) {
+      best = bn;
+      best_waves = waves;
+      best_tiles = tiles;
+    }
+  }
+  return best;
 }
 
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) {
@@ -371,14 +393,15 @@ bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) 
          make_tmap_f16(&gw->box256, base, n, k, 256);
 }
 
-// Tile choice: above 512 rows the GEMM is tensor-bound and takes 128 x 256
-// tiles; at or below it is bound by streaming the weights, so it takes narrow
-// tiles (more CTAs pulling weight bytes) and a deeper ring (more bytes in
-// flight per SM).  The W map passed always has the box the kernel expects.
+// Tile choice (gemm_box_n): above 512 rows the GEMM is tensor-bound and takes
+// 128 x 256 tiles with a 4-stage ring; at or below it streams the weights and
+// takes the width that keeps the most SMs busy in the fewest waves, with a
+// deeper ring for the narrower tiles.  The W map passed has the matching box.
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
   if (m <= 0) return cudaSuccess;
-  if (m > 512) {
+  const uint32_t bn = gemm_box_n(m, n, epilogue);
+  if (bn == 256) {
     switch (epilogue) {
       case EPI_STORE_BF16:
         return launch_persistent<256, 4, EPI_STORE_BF16>(ta, w.box256, out, m, n, k, status, st);
@@ -390,13 +413,23 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
         return cudaErrorInvalidValue;
     }
   }
+  if (bn == 128) {
+    switch (epilogue) {
+      case EPI_STORE_BF16:
+        return launch_persistent<128, 6, EPI_STORE_BF16>(ta, w.box128, out, m, n, k, status, st);
+      case EPI_ADD_F32:
+        return launch_persistent<128, 6, EPI_ADD_F32>(ta, w.box128, out, m, n, k, status, st);
+      case EPI_SWIGLU_BF16:
+        return launch_persistent<128, 6, EPI_SWIGLU_BF16>(ta, w.box128, out, m, n, k, status, st);
+      default:
+        return cudaErrorInvalidValue;
+    }
+  }
   switch (epilogue) {
     case EPI_STORE_BF16:
       return launch_persistent<64, 8, EPI_STORE_BF16>(ta, w.box64, out, m, n, k, status, st);
     case EPI_ADD_F32:
       return launch_persistent<64, 8, EPI_ADD_F32>(ta, w.box64, out, m, n, k, status, st);
-    case EPI_SWIGLU_BF16:
-      return launch_persistent<128, 6, EPI_SWIGLU_BF16>(ta, w.box128, out, m, n, k, status, st);
     default:
       return cudaErrorInvalidValue;
   }

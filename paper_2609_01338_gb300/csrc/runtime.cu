@@ -600,25 +600,27 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
 
 // Per-layer algorithmic sizes of a shape.
 struct CostModelShape {
-  double layer_weight_bytes, linear_flops_row, attn_flops_pair;
+  double layer_weight_bytes, linear_flops_row, attn_flops_pair, qkv_frac;
   explicit CostModelShape(const mzc_model_shape& s) {
     const double d = s.d_model, hq = s.n_q_heads, hkv = s.n_kv_heads, hd = s.head_dim, f = s.ffn_dim;
     const double params = d * (hq + 2 * hkv) * hd + hq * hd * d + 3.0 * d * f;
     layer_weight_bytes = 2.0 * params;
     linear_flops_row = 2.0 * params;
     attn_flops_pair = 4.0 * hd * hq;
+    qkv_frac = d * (hq + 2 * hkv) * hd / params;
   }
 };
 
 // Per-unit cost model of the two restore paths (Sec. 4.3: per-unit times
 // from offline profiling, total time linear in the number of units).
-// Copy: evicted blocks x bytes / host-link rate.  Compute of the fused rows
-// (recomputed tail + prompt), per layer: the projections interpolated from
-// their measured times at 128 / 512 / 2048 rows, attention pairs at the
-// measured rates of recompute-like and prompt-like rows, per-row
+// Copy: evicted blocks x bytes / host-link rate, layer after layer.  Compute
+// of the fused rows (recomputed tail + prompt), per layer: the projections
+// interpolated from their measured times at 128 / 512 / 2048 rows, attention
+// pairs at the measured rates of recompute-like and prompt-like rows, per-row
 // memory-bound kernels and a fixed per-layer cost.  The two paths overlap
-// layer by layer, so a step takes the longer of the two, plus the part of the
-// last layer that runs after its copy has landed.
+// layer by layer: the part of a layer before the attention that reads copied
+// keys (QKV projection, rotary/KV write, attention of the recomputed rows)
+// never waits; the rest starts once that layer's copy has landed.
 struct CostModel : CostModelShape {
   mzc_model_shape s;
   mzc_profile p;
@@ -635,23 +637,31 @@ struct CostModel : CostModelShape {
     else us = p.gemm_us_512 + (rows - 512) * (p.gemm_us_2048 - p.gemm_us_512) / 1536.0;
     return us * 1e-6;
   }
-  double layer_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
+  // one layer's compute, split at the wait for copied keys: *pre never waits
+  double layer_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt, double* pre = nullptr) const {
     const double rows = static_cast<double>(s1 - p0 + n_prompt);
+    if (pre) *pre = 0.0;
     if (rows <= 0) return 0.0;
     auto tri = [](double a, double b) { return (b * (b + 1) - a * (a + 1)) / 2.0; };
     const double rec_pairs = tri(static_cast<double>(p0), static_cast<double>(s1));
     const double prm_pairs = tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
-    const double attn = rec_pairs * attn_flops_pair / (p.attn_tflops * 1e12) +
-                        static_cast<double>(s1 - p0) * p.attn_row_ns * 1e-9 +
-                        prm_pairs * attn_flops_pair / (p.attn_prompt_tflops * 1e12);
-    return gemm_s(rows) + attn + rows * p.row_ns * 1e-9 + p.layer_us * 1e-6;
+    const double rec_attn = rec_pairs * attn_flops_pair / (p.attn_tflops * 1e12) +
+                            static_cast<double>(s1 - p0) * p.attn_row_ns * 1e-9;
+    const double prm_attn = prm_pairs * attn_flops_pair / (p.attn_prompt_tflops * 1e12);
+    const double g = gemm_s(rows), rw = rows * p.row_ns * 1e-9, fixed = p.layer_us * 1e-6;
+    if (pre) *pre = g * qkv_frac + rec_attn + rw * (2.0 / 3.0) + fixed * 0.5;
+    return g + rec_attn + prm_attn + rw + fixed;
   }
   // predicted TTFT when [p0, s1) is recomputed and [s1, n_ctx) copied
   double ttft_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
-    const double layer = layer_s(p0, s1, n_ctx, n_prompt);
-    const double compute = s.n_layers * layer;
+    double pre = 0.0;
+    const double layer = layer_s(p0, s1, n_ctx, n_prompt, &pre);
     const double copy = copy_s(n_ctx - s1);
-    return copy > 0.0 ? std::max(compute, copy + 0.75 * layer) : compute;
+    if (copy <= 0.0) return s.n_layers * layer;
+    const double per_copy = copy / s.n_layers;
+    double t = 0.0;
+    for (int l = 0; l < s.n_layers; ++l) t = std::max(t + pre, (l + 1) * per_copy) + (layer - pre);
+    return t;
   }
 };
 
@@ -1070,8 +1080,9 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
     }
   }
   // memory-bound kernels per row (two RMSNorms and the rotary/KV write,
-  // approximated by three norms over 1024 rows) and the fixed per-layer cost
-  // (the same launches at one row)
+  // approximated by three norms): the per-row slope between a quarter and all
+  // of up to 8192 rows (both large enough to stream), and the fixed per-layer
+  // cost from the same launches at one row
   {
     auto norms = [&](int64_t rows) -> cudaError_t {
       cudaError_t e = cudaSuccess;
@@ -1080,19 +1091,22 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
                                 ctx->d_h, ctx->cs);
       return e;
     };
-    float ms1 = 0.0f, msn = 0.0f;
-    const int64_t rows = std::min<int64_t>(ctx->max_rows, 1024);
-    for (int pass = 0; pass < 2; ++pass) {
-      const int64_t r = pass == 0 ? 1 : rows;
-      CK(norms(r));
+    const int64_t rows = std::min<int64_t>(ctx->max_rows, 8192);
+    const int64_t sizes[3] = {1, std::max<int64_t>(1, rows / 4), rows};
+    float ms[3] = {0.0f, 0.0f, 0.0f};
+    for (int pass = 0; pass < 3; ++pass) {
+      CK(norms(sizes[pass]));
       CK(cudaEventRecord(a, ctx->cs));
-      for (int i = 0; i < 20; ++i) CK(norms(r));
+      for (int i = 0; i < 20; ++i) CK(norms(sizes[pass]));
       CK(cudaEventRecord(b, ctx->cs));
       CK(cudaEventSynchronize(b));
-      CK(cudaEventElapsedTime(pass == 0 ? &ms1 : &msn, a, b));
+      CK(cudaEventElapsedTime(&ms[pass], a, b));
     }
-    p.layer_us = ms1 * 1e3 / 20.0 * (8.0 / 3.0);  // ~8 launches per layer
-    p.row_ns = std::max(0.0, (static_cast<double>(msn) - ms1) * 1e6 / 20.0 / static_cast<double>(rows));
+    p.layer_us = ms[0] * 1e3 / 20.0 * (8.0 / 3.0);  // ~8 launches per layer
+    p.row_ns = sizes[2] > sizes[1]
+                   ? std::max(0.0, (static_cast<double>(ms[2]) - ms[1]) * 1e6 / 20.0 /
+                                       static_cast<double>(sizes[2] - sizes[1]))
+                   : 0.0;
   }
   CK(cudaEventDestroy(a));
   CK(cudaEventDestroy(b));

@@ -171,19 +171,24 @@ def _prof(h2d=200.0):
 
 def test_hybrid_split_bruteforce_and_limits():
     """The solver returns the block-aligned split minimising the documented
-    cost (per layer: projections interpolated from their 128/512/2048-row
-    times, recompute attention pairs at their rate plus a per-row cost, prompt
-    attention pairs at their rate, per-row and
-    per-layer costs; TTFT = max(compute, copy + 0.75 layer)), and stays at
-    copy-only unless that saves at least 5%."""
+    cost, and stays at copy-only unless that saves at least 5%.  Per layer:
+    projections interpolated from their 128/512/2048-row times, recompute
+    attention pairs at their rate plus a per-row cost, prompt attention pairs
+    at their rate, per-row and per-layer costs.  The layer's part before the
+    attention over copied keys (the QKV share of the projections, the
+    recompute attention, 2/3 of the per-row and 1/2 of the per-layer cost)
+    never waits; the rest of layer l starts once copy l (copy / L each, in
+    layer order) has landed."""
     prof = _prof()
     sh = W.THREE_B
 
     def cost(p, s, n, P, pr=prof):
-        d, hq, hkv, hd, L = (sh[k] for k in ("d_model", "n_q_heads", "n_kv_heads", "head_dim",
-                                               "n_layers"))
+        d, hq, hkv, hd, L, f = (sh[k] for k in ("d_model", "n_q_heads", "n_kv_heads", "head_dim",
+                                                  "n_layers", "ffn_dim"))
+        params = d * (hq + 2 * hkv) * hd + hq * hd * d + 3 * d * f
+        qkv_frac = d * (hq + 2 * hkv) * hd / params
         rows = s - p + P
-        layer = 0.0
+        layer = pre = 0.0
         if rows > 0:
             if rows <= 128:
                 g = pr.gemm_us_128
@@ -191,14 +196,21 @@ def test_hybrid_split_bruteforce_and_limits():
                 g = pr.gemm_us_128 + (rows - 128) * (pr.gemm_us_512 - pr.gemm_us_128) / 384
             else:
                 g = pr.gemm_us_512 + (rows - 512) * (pr.gemm_us_2048 - pr.gemm_us_512) / 1536
+            g *= 1e-6
             rec = sum(range(p + 1, s + 1))
             prm = sum(range(n + 1, n + P + 1))
-            layer = (g * 1e-6 + rec * 4 * hd * hq / (pr.attn_tflops * 1e12) + (s - p) * pr.attn_row_ns * 1e-9
-                     + prm * 4 * hd * hq / (pr.attn_prompt_tflops * 1e12)
-                     + rows * pr.row_ns * 1e-9 + pr.layer_us * 1e-6)
+            rec_attn = rec * 4 * hd * hq / (pr.attn_tflops * 1e12) + (s - p) * pr.attn_row_ns * 1e-9
+            rw = rows * pr.row_ns * 1e-9
+            layer = (g + rec_attn + prm * 4 * hd * hq / (pr.attn_prompt_tflops * 1e12) + rw
+                     + pr.layer_us * 1e-6)
+            pre = g * qkv_frac + rec_attn + rw * 2 / 3 + pr.layer_us * 1e-6 / 2
         copy = -(-(n - s) // 16) * L * 2 * hkv * 16 * hd * 2 / (pr.h2d_gbs * 1e9)
-        comp = L * layer
-        return max(comp, copy + 0.75 * layer) if copy > 0 else comp
+        if copy <= 0:
+            return L * layer
+        t = 0.0
+        for l in range(L):
+            t = max(t + pre, (l + 1) * copy / L) + (layer - pre)
+        return t
 
     for p, n, P in ((16384, 32768, 128), (0, 4096, 0), (31744, 32768, 512), (1000 // 16 * 16, 1000, 3),
                     (0, 32768, 128)):
