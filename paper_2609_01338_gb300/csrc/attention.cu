@@ -46,28 +46,37 @@ namespace mzc {
 
 namespace {
 
-constexpr int kRowsPerCta = 256;  // two Q tiles of 128 rows
-constexpr int kThreads = 352;     // 8 softmax warps, TMA producer, 2 UMMA issuers
 
 template <int HD>
 struct AttnCfg {
   static constexpr int BM = 128;                  // rows per Q tile (TMEM lanes)
   static constexpr int BN = HD == 64 ? 128 : 64;  // keys per tile
+  // Q tiles per CTA (both share every K/V tile) and CTAs per SM.  One tile
+  // per CTA with two CTAs per SM (2-stage ring) measured 32% slower at head
+  // dim 64: each CTA fetches its own K/V and the shallow ring exposes latency.
+  static constexpr int NQ = 2;
+  static constexpr int CTAS_PER_SM = 1;
+  static constexpr int ROWS = NQ * BM;
+  // warps: 4 NQ softmax, then the TMA producer, then NQ UMMA issuers
+  static constexpr int PRODUCER_WARP = 4 * NQ;
+  static constexpr int THREADS = (5 * NQ + 1) * 32;
   static constexpr int STAGES = HD == 64 ? 5 : 4;
   static constexpr int CB = HD / 64;              // 64-column slices of the head dim
   static constexpr int Q_BYTES = BM * HD * 2;     // one Q tile
   static constexpr int KV_BYTES = BN * HD * 2;    // K or V of one key tile
-  static constexpr int OFF_K = 2 * Q_BYTES;
+  static constexpr int OFF_K = NQ * Q_BYTES;
   static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;  // + barriers + alignment slack
   // TMEM columns: S of tile t at t*BN (fp32), P of tile t at P_COL + t*BN/2
   // (fp16 pairs), O of tile t at O_COL + t*HD (fp32)
-  static constexpr uint32_t P_COL = 2 * BN;
-  static constexpr uint32_t O_COL = 3 * BN;
-  static constexpr uint32_t TMEM_COLS = 512;
-  static_assert(O_COL + 2 * HD <= TMEM_COLS, "S, P and O of both tiles fit in TMEM");
-  static_assert(SMEM <= 232448, "shared memory per CTA");
+  static constexpr uint32_t P_COL = NQ * BN;
+  static constexpr uint32_t O_COL = NQ * BN + NQ * BN / 2;
+  static constexpr uint32_t TMEM_COLS = NQ == 2 ? 512 : 256;
+  static_assert(O_COL + NQ * HD <= TMEM_COLS, "S, P and O of every tile fit in TMEM");
+  static_assert(TMEM_COLS * CTAS_PER_SM <= 512, "TMEM of the CTAs sharing an SM");
+  static_assert(3 * STAGES * 8 + 4 * NQ * 8 <= 256, "barriers");
+  static_assert((SMEM + 1024) * CTAS_PER_SM <= 233472, "shared memory of the CTAs sharing an SM");
 };
 
 // kind::f16 instruction descriptor: fp32 D, A/B fp16 (or bf16), A K-major,
@@ -178,7 +187,7 @@ __device__ __forceinline__ void tmem_st_row(uint32_t taddr, const float* v) {
 // TMEM owner, warps 9 and 10 issue the UMMAs of Q tiles 0 and 1.  Both Q tiles
 // share every K/V tile.
 template <int HD, bool F16>
-__global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
+__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM) attn_tc_kernel(
     const uint16_t* __restrict__ q, const int32_t* __restrict__ pos, int n, int hq, int hkv,
     const int32_t* __restrict__ table, int64_t n_logical,
     const __grid_constant__ CUtensorMap pool_run, const __grid_constant__ CUtensorMap pool_blk,
@@ -190,17 +199,17 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sQ = smem;  // [2 tiles]
+  uint8_t* sQ = smem;  // [NQ tiles]
   uint8_t* sK = smem + C::OFF_K;
   uint8_t* sV = smem + C::OFF_V;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* k_full = bars;                    // [STAGES]
   uint64_t* v_full = bars + C::STAGES;        // [STAGES]
   uint64_t* kv_empty = bars + 2 * C::STAGES;  // [STAGES]
-  uint64_t* s_full = bars + 3 * C::STAGES;    // [2 tiles] S(j) in TMEM
-  uint64_t* s_free = s_full + 2;              // [2 tiles] S(j) read into registers
-  uint64_t* p_full = s_free + 2;              // [2 tiles] P(j) in TMEM
-  uint64_t* p_free = p_full + 2;              // [2 tiles] P(j) V(j) done
+  uint64_t* s_full = bars + 3 * C::STAGES;    // [NQ tiles] S(j) in TMEM
+  uint64_t* s_free = s_full + C::NQ;          // [NQ tiles] S(j) read into registers
+  uint64_t* p_full = s_free + C::NQ;          // [NQ tiles] P(j) in TMEM
+  uint64_t* p_free = p_full + C::NQ;          // [NQ tiles] P(j) V(j) done
   __shared__ uint32_t s_tmem;
   __shared__ int s_maxpos;
   __shared__ int s_abort;
@@ -212,16 +221,16 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
   const int g = blockIdx.x;
   const int group = hq / hkv;
   const int R = n * group;
-  const int r0 = (gridDim.y - 1 - blockIdx.y) * kRowsPerCta;
+  const int r0 = (gridDim.y - 1 - blockIdx.y) * C::ROWS;
   const int split = blockIdx.z;
 
   if (tid == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
-      mbar_init(&kv_empty[s], 2);  // both Q tiles' P V done
+      mbar_init(&kv_empty[s], C::NQ);  // every Q tile's P V done
     }
-    for (int t = 0; t < 2; ++t) {
+    for (int t = 0; t < C::NQ; ++t) {
       mbar_init(&s_full[t], 1);
       mbar_init(&s_free[t], 4);  // one arrival per softmax warp of the tile
       mbar_init(&p_full[t], 4);
@@ -233,14 +242,14 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
     tma_prefetch_desc(&pool_run);
     tma_prefetch_desc(&pool_blk);
   }
-  if (warp == 8) tmem_alloc(&s_tmem, C::TMEM_COLS);
+  if (warp == C::PRODUCER_WARP) tmem_alloc(&s_tmem, C::TMEM_COLS);
 
   // softmax threads: tile and row; the Q tiles in the UMMA K-major layout
-  const int qt = tid >> 7;  // Q tile of warps 0-7
+  const int qt = tid >> 7;  // Q tile of the softmax warps
   const int row = tid & 127;
   const int rr = r0 + qt * C::BM + row;
   int row_pos = -1;
-  if (warp < 8) {
+  if (warp < C::PRODUCER_WARP) {
     const int t = rr / group, h = g * group + rr % group;
     if (rr < R) row_pos = pos[t];
     uint8_t* q_tile = sQ + qt * C::Q_BYTES;
@@ -255,8 +264,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
     cp_async_commit();
   }
   __syncthreads();
-  if (warp < 8 && row_pos >= 0) atomicMax(&s_maxpos, row_pos);
-  if (warp < 8) {
+  if (warp < C::PRODUCER_WARP && row_pos >= 0) atomicMax(&s_maxpos, row_pos);
+  if (warp < C::PRODUCER_WARP) {
     cp_async_wait<0>();
     fence_async_smem();  // Q (generic-proxy writes) visible to the tensor core
   }
@@ -269,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
   const int k_end = min(kv_len, k_begin + keys_per_split);
   const int T = k_end > k_begin ? (k_end - k_begin + BN - 1) / BN : 0;
 
-  if (warp == 8) {
+  if (warp == C::PRODUCER_WARP) {
     if (T > 0) {
       // ---- TMA producer (whole warp): lane b looks up block b of a key tile,
       // one tile ahead of its use, so the table reads overlap the copies ----
@@ -336,9 +345,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
         }
       }
     }
-  } else if (warp >= 9) {
+  } else if (warp > C::PRODUCER_WARP) {
     // ---- UMMA issuers, one per Q tile t: S_t(j+1), then P_t V(j) ----
-    const int t = warp - 9;
+    const int t = warp - C::PRODUCER_WARP - 1;
     if (lane == 0 && T > 0) {
       constexpr uint32_t id_s = idesc_attn<F16>(128, BN, false);
       constexpr uint32_t id_o = idesc_attn<F16>(128, HD, true);
@@ -535,7 +544,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == C::PRODUCER_WARP) {
     __syncwarp();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
@@ -627,12 +636,12 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
     return cudaErrorInvalidValue;
   const int group = hq / hkv;
   const int64_t R = n * group;
-  const int64_t row_tiles = (R + kRowsPerCta - 1) / kRowsPerCta;
+  const int64_t row_tiles = (R + C::ROWS - 1) / C::ROWS;
   if (row_tiles > 65535) return cudaErrorInvalidValue;
   dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(row_tiles), static_cast<unsigned>(n_splits));
   const float scale_log2 =
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
-  attn_tc_kernel<HD, F16><<<grid, kThreads, C::SMEM, st>>>(
+  attn_tc_kernel<HD, F16><<<grid, C::THREADS, C::SMEM, st>>>(
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, run_map, blk_map, pool_blocks, out, part_o,
       part_lse, keys_per_split, n_splits, scale_log2, status);
   cudaError_t e = cudaGetLastError();
@@ -645,19 +654,21 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
 
 }  // namespace
 
-void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int num_sms,
+void attention_split(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys, int num_sms,
                      int* n_splits, int* keys_per_split) {
-  const int64_t ctas = ((n * (hq / hkv) + kRowsPerCta - 1) / kRowsPerCta) * hkv;
+  const int rows_per_cta = hd == 64 ? AttnCfg<64>::ROWS : AttnCfg<128>::ROWS;
+  const int slots = num_sms * (hd == 64 ? AttnCfg<64>::CTAS_PER_SM : AttnCfg<128>::CTAS_PER_SM);
+  const int64_t ctas = ((n * (hq / hkv) + rows_per_cta - 1) / rows_per_cta) * hkv;
   int s = 1;
-  if (ctas < num_sms && max_keys > 1024) {
-    // one CTA per SM: pick the split count whose waves are fullest (ties -> more
-    // splits), with at least 512 keys per split
+  if (ctas < slots && max_keys > 1024) {
+    // fewer CTAs than resident slots: pick the split count whose waves are
+    // fullest (ties -> more splits), with at least 512 keys per split
     const int64_t max_s = std::min<int64_t>(64, (max_keys + 511) / 512);
     double best = 0.0;
     for (int64_t c = 1; c <= max_s; ++c) {
       const int64_t total = ctas * c;
-      const int64_t waves = (total + num_sms - 1) / num_sms;
-      const double eff = static_cast<double>(total) / static_cast<double>(waves * num_sms);
+      const int64_t waves = (total + slots - 1) / slots;
+      const double eff = static_cast<double>(total) / static_cast<double>(waves * slots);
       if (eff >= best - 1e-9) {
         best = eff;
         s = static_cast<int>(c);
@@ -684,7 +695,7 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
                              int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   int s = 1, per = 0;
-  attention_split(n, hq, hkv, max_keys, num_sms, &s, &per);
+  attention_split(n, hq, hkv, hd, max_keys, num_sms, &s, &per);
   if (s > 1 && (scratch == nullptr || scratch_bytes < attention_scratch_bytes(n, hq, hd, s))) {
     s = 1;
     per = static_cast<int>((max_keys + 127) / 128 * 128);

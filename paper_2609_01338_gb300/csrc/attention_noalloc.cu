@@ -44,7 +44,7 @@ cudaError_t noalloc_scratch(void** out) {
 int64_t attention_noalloc_need(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys,
                                int num_sms) {
   int s = 1, per = 0;
-  attention_split(n, hq, hkv, max_keys, num_sms, &s, &per);
+  attention_split(n, hq, hkv, hd, max_keys, num_sms, &s, &per);
   return attention_scratch_bytes(n, hq, hd, s);
 }
 

@@ -43,7 +43,7 @@ cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_
                                  int32_t* status, cudaStream_t st);
 // Split-KV plan: how many key splits a launch of n rows over at most
 // max_keys keys uses, and the keys per split (a multiple of 64).
-void attention_split(int64_t n, int32_t hq, int32_t hkv, int64_t max_keys, int num_sms,
+void attention_split(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys, int num_sms,
                      int* n_splits, int* keys_per_split);
 int64_t attention_scratch_bytes(int64_t n, int32_t hq, int32_t hd, int n_splits);
 cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,

@@ -332,7 +332,7 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   int64_t scratch = 0;
   for (int64_t n = 1; n <= std::min<int64_t>(R, 8192); ++n) {
     int sp = 1, per = 0;
-    mzc::attention_split(n, s.n_q_heads, s.n_kv_heads, s.max_ctx, ctx->num_sms, &sp, &per);
+    mzc::attention_split(n, s.n_q_heads, s.n_kv_heads, s.head_dim, s.max_ctx, ctx->num_sms, &sp, &per);
     scratch = std::max(scratch, mzc::attention_scratch_bytes(n, s.n_q_heads, s.head_dim, sp));
   }
   ctx->scratch_bytes = scratch;
@@ -519,7 +519,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       double fl, by;
       attn_work(c0 + r0, nr, &fl, &by);
       int sp = 1, per = 0;
-      mzc::attention_split(nr, s.n_q_heads, s.n_kv_heads, mk, ctx->num_sms, &sp, &per);
+      mzc::attention_split(nr, s.n_q_heads, s.n_kv_heads, s.head_dim, mk, ctx->num_sms, &sp, &per);
       const bool fits = sp == 1 || ctx->scratch_bytes >= mzc::attention_scratch_bytes(nr, s.n_q_heads, s.head_dim, sp);
       return klaunch(ctx, MZC_K_ATTENTION, fl, by, (sp > 1 && fits) ? 2 : 1, [&] {
         return mzc::launch_attention(ctx->d_q + r0 * hq * hd, cpos + r0, nr, s.n_q_heads, s.n_kv_heads,
@@ -1184,7 +1184,7 @@ mzc_status mzc_k_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_t 
 int64_t mzc_k_attention_scratch_bytes(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys) {
   if (n <= 0 || hkv <= 0) return 0;
   int sp = 1, per = 0;
-  mzc::attention_split(n, hq, hkv, max_keys, sm_count(), &sp, &per);
+  mzc::attention_split(n, hq, hkv, hd, max_keys, sm_count(), &sp, &per);
   return mzc::attention_scratch_bytes(n, hq, hd, sp);
 }
 
