@@ -80,6 +80,8 @@ def lib():
             L.orc_round_kv_array.argtypes = [vp, i64, i32, vp]
             L.orc_f32_to_f16_array.argtypes = [vp, i64, vp]
             L.orc_f32_to_bf16_array.argtypes = [vp, i64, vp]
+            L.orc_q8_encode.argtypes = [vp, i64, vp, vp, vp]
+            L.orc_q8_decode.argtypes = [vp, vp, vp, i64, vp]
             L.orc_num_threads.restype = ctypes.c_int
             _lib = L
     return _lib
@@ -228,3 +230,55 @@ def to_bf16_bits(x):
     x = _f32(x); y = np.empty(x.shape, dtype=np.uint16)
     lib().orc_f32_to_bf16_array(_p(x), x.size, _p(y))
     return y
+
+
+# ---- 8-bit swap codec (oracle.c: orc_q8_encode / orc_q8_decode) -------------
+
+Q8_GROUP = 64
+
+
+def q8_encode(x):
+    """Groups of 64 along the last axis -> (codes uint8, min fp32, step fp32)."""
+    x = _f32(x)
+    assert x.shape[-1] % Q8_GROUP == 0
+    g = x.size // Q8_GROUP
+    codes = np.empty(x.shape, np.uint8)
+    mn = np.empty(x.shape[:-1] + (x.shape[-1] // Q8_GROUP,), np.float32)
+    st = np.empty_like(mn)
+    lib().orc_q8_encode(_p(x), g, _p(codes), _p(mn), _p(st))
+    return codes, mn, st
+
+
+def q8_decode(codes, mn, step):
+    codes = np.ascontiguousarray(codes, np.uint8)
+    mn, step = _f32(mn), _f32(step)
+    out = np.empty(codes.shape, np.float32)
+    lib().orc_q8_decode(_p(codes), _p(mn), _p(step), codes.size // Q8_GROUP, _p(out))
+    return out
+
+
+def q8_block_bytes(hkv: int, hd: int) -> int:
+    """Compressed size of one KV block: the codes, then (min, step) per group."""
+    e = 2 * hkv * 16 * hd
+    return e + 8 * (e // Q8_GROUP)
+
+
+def q8_encode_blocks(blocks_f16_bits):
+    """KV blocks [n][2*hkv*16*hd] of fp16 bits -> compressed bytes [n][q8_block_bytes]:
+    the codes in the block's element order, then fp32 (min, step) pairs in group order."""
+    b = np.ascontiguousarray(blocks_f16_bits, np.uint16)
+    n, e = b.shape
+    x = b.view(np.float16).astype(np.float32).reshape(n, e // Q8_GROUP, Q8_GROUP)
+    codes, mn, st = q8_encode(x)
+    params = np.stack([mn, st], axis=-1).astype(np.float32).reshape(n, -1)
+    return np.concatenate([codes.reshape(n, e), params.view(np.uint8)], axis=1)
+
+
+def q8_decode_blocks(comp, e: int, kv_dtype: int):
+    """Compressed blocks -> fp16 bits [n][e] of the values rounded to the KV type."""
+    c = np.ascontiguousarray(comp, np.uint8)
+    n = c.shape[0]
+    codes = c[:, :e].reshape(n, e // Q8_GROUP, Q8_GROUP)
+    params = np.ascontiguousarray(c[:, e:]).view(np.float32).reshape(n, e // Q8_GROUP, 2)
+    y = q8_decode(codes, params[..., 0], params[..., 1]).reshape(n, e)
+    return to_f16_bits(round_kv(y, kv_dtype))

@@ -364,6 +364,49 @@ void orc_f32_to_bf16_array(const float* x, int64_t n, uint16_t* y) {
   for (int64_t i = 0; i < n; ++i) y[i] = orc_f32_to_bf16(x[i]);
 }
 
+/* ---- 8-bit swap codec ------------------------------------------------------
+ * The paper keeps swapped KV compressed, with 8-bit quantization as the
+ * default codec (Sec. 5), and notes that it is idempotent: compressing the
+ * decompressed values again gives the same result (Sec. 6.5).  The format is
+ * not given; reading used here: asymmetric min/max quantization over groups
+ * of 64 consecutive values (one group = 64 head_dim entries of one K or V
+ * row), fp32 minimum and step, step = (max - min) / 255,
+ *   code  = round-half-even((x - min) / step), clamped to [0, 255]
+ *           (0 for every value of a constant group, step == 0),
+ *   value = code * step + min   (two fp32 roundings, no fused multiply-add).
+ */
+void orc_q8_encode(const float* x, int64_t n_groups, uint8_t* codes, float* mn_out,
+                   float* step_out) {
+  for (int64_t g = 0; g < n_groups; ++g) {
+    const float* v = x + g * 64;
+    float mn = v[0], mx = v[0];
+    for (int i = 1; i < 64; ++i) {
+      if (v[i] < mn) mn = v[i];
+      if (v[i] > mx) mx = v[i];
+    }
+    const float step = (mx - mn) / 255.0f;
+    for (int i = 0; i < 64; ++i) {
+      uint8_t c = 0;
+      if (step > 0.0f) {
+        const float q = rintf((v[i] - mn) / step);
+        c = q <= 0.0f ? 0 : (q >= 255.0f ? 255 : (uint8_t)q);
+      }
+      codes[g * 64 + i] = c;
+    }
+    mn_out[g] = mn;
+    step_out[g] = step;
+  }
+}
+
+void orc_q8_decode(const uint8_t* codes, const float* mn, const float* step, int64_t n_groups,
+                   float* out) {
+  for (int64_t g = 0; g < n_groups; ++g)
+    for (int i = 0; i < 64; ++i) {
+      const float prod = (float)codes[g * 64 + i] * step[g];
+      out[g * 64 + i] = prod + mn[g];
+    }
+}
+
 int orc_num_threads(void) {
 #ifdef _OPENMP
   extern int omp_get_max_threads(void);
