@@ -50,6 +50,7 @@ typedef enum {
 } mzc_status;
 
 enum { MZC_KV_BF16 = 0, MZC_KV_FP16 = 1 };
+enum { MZC_CODEC_NONE = 0, MZC_CODEC_Q8 = 1 };
 /* eviction modes: COPY = swap to pinned host (restored by copy); DROP =
  * discard (restored by recompute); AUTO = split by the ctx's policy. */
 enum { MZC_COPY = 0, MZC_DROP = 1, MZC_AUTO = 2 };
@@ -75,6 +76,9 @@ typedef struct {
   int32_t overlap;          /* 1 = zero-wait overlap of restore and prefill; 0 = restore
                                completes before prefill starts (ablation) */
   int32_t device;           /* CUDA device ordinal */
+  int32_t swap_codec;       /* MZC_CODEC_NONE: COPY swaps blocks as stored; MZC_CODEC_Q8:
+                               8-bit quantized (mzc_k_q8_encode; about 0.56 of the bytes),
+                               decoded into the pool on restore */
 } mzc_options;
 
 /* Weights, host memory, bf16 bit patterns, row-major [out_features][in_features]
@@ -161,7 +165,10 @@ mzc_status mzc_prefill(mzc_ctx *ctx, const int32_t *tokens, int64_t n, float *lo
  * all layers, with the dropped positions forming one contiguous range;
  * MZC_AUTO splits [tok_begin, context_tokens) into a recomputed front and a
  * copied back by the ctx's policy (mzc_set_policy).  Every block in range
- * must be RESIDENT (else MZC_ERR_STATE, nothing changes).  Synchronous. */
+ * must be RESIDENT (else MZC_ERR_STATE, nothing changes).  With the
+ * MZC_CODEC_Q8 option, copied blocks are quantized on the device before the
+ * D2H copy, and restored blocks hold the decoded values (lossy; repeated
+ * swaps give the same values again).  Synchronous. */
 mzc_status mzc_evict(mzc_ctx *ctx, int32_t layer_begin, int32_t layer_end, int64_t tok_begin,
                      int64_t tok_end, int32_t mode);
 /* Fine-grained COPY eviction of n scattered (layer[i], logical_block[i]). */
@@ -373,6 +380,26 @@ mzc_status mzc_k_attention_noalloc(const uint16_t *q, const int32_t *pos, int64_
                                    int64_t n_logical, const void *pool, int64_t pool_blocks,
                                    int32_t kv_dtype, uint16_t *out, int64_t max_keys,
                                    int32_t *status, void *stream);
+
+/* 8-bit swap codec (the paper's default KV compression, Sec. 5; idempotent,
+ * Sec. 6.5).  Per group of 64 consecutive values of a KV block (64 head_dim
+ * entries of one K or V row): fp32 min and step = (max - min) / 255,
+ * code = round-half-even((x - min) / step) clamped to [0, 255] (0 for a
+ * constant group), decoded value = code * step + min (two fp32 roundings),
+ * rounded to kv_dtype and stored fp16-encoded.  A compressed block is the
+ * block_elems codes in the block's element order followed by block_elems/64
+ * fp32 (min, step) pairs: mzc_q8_block_bytes(hkv, hd) bytes, where
+ * block_elems = 2 * hkv * 16 * hd.
+ * encode: pool (device, fp16-encoded blocks) blocks phys[i] (device int32
+ * [n]) -> out (device) [n][mzc_q8_block_bytes].
+ * decode: in (device) [n][...] -> pool blocks phys[i], or phys_begin + i when
+ * phys is NULL. */
+int64_t mzc_q8_block_bytes(int32_t hkv, int32_t hd);
+mzc_status mzc_k_q8_encode(const void *pool, const int32_t *phys, int64_t n, int32_t hkv,
+                           int32_t hd, void *out, void *stream);
+mzc_status mzc_k_q8_decode(const void *in, int64_t n, int32_t hkv, int32_t hd,
+                           const int32_t *phys, int64_t phys_begin, int32_t kv_dtype, void *pool,
+                           void *stream);
 
 /* logits fp32 [vocab] = RMSNorm(x_row) * g  W^T, x_row fp32 [d], W bf16 [vocab][d]. */
 mzc_status mzc_k_lm_head(const float *x_row, const float *g, int32_t d, float eps,

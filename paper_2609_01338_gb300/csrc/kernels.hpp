@@ -32,6 +32,14 @@ uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st);
 
+// 8-bit swap codec (codec.cu).  block_elems = 2 * hkv * 16 * hd.
+int64_t q8_block_bytes(int64_t block_elems);
+cudaError_t launch_q8_encode(const void* pool, const int32_t* phys, int64_t n_blocks,
+                             int64_t block_elems, void* out, cudaStream_t st);
+cudaError_t launch_q8_decode(const void* in, int64_t n_blocks, int64_t block_elems,
+                             const int32_t* phys, int64_t phys_begin, int32_t kv_dtype, void* pool,
+                             cudaStream_t st);
+
 cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
                          int64_t vocab, float* x, int32_t* status, cudaStream_t st);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,

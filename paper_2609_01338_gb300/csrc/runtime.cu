@@ -93,6 +93,13 @@ struct mzc_ctx {
   int32_t* h_list = nullptr;
   uint8_t* h_staging = nullptr;  // pinned, one layer of blocks (reads)
   std::vector<cudaEvent_t> ev_kv, ev_w;
+  // swap codec: compressed slots; restores land in a staging buffer (two,
+  // alternating by layer) and a decode stream writes the pool
+  int32_t codec = MZC_CODEC_NONE;
+  int64_t slot_bytes = 0;
+  cudaStream_t ds = nullptr;
+  std::vector<cudaEvent_t> ev_h2d, ev_dec;
+  uint8_t* d_rstage[2] = {nullptr, nullptr};
   cudaEvent_t ev_t0 = nullptr, ev_t1 = nullptr, ev_c0 = nullptr, ev_c1 = nullptr,
               ev_l0 = nullptr, ev_l1 = nullptr;
   bool restore_issued = false, lm_timed = false, ttft_from_copy = false;
@@ -137,12 +144,14 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
   cudaSetDevice(ctx->opt.device);
   if (ctx->cs) cudaStreamSynchronize(ctx->cs);
   if (ctx->xs) cudaStreamSynchronize(ctx->xs);
+  if (ctx->ds) cudaStreamSynchronize(ctx->ds);
   for (auto& L : ctx->layers)
     if (L.host_master) cudaFreeHost(L.host_master);
   void* dev[] = {ctx->d_weights, ctx->d_embed, ctx->d_lm,      ctx->d_fnorm,   ctx->d_pool,
                  ctx->d_cos,     ctx->d_sin,   ctx->d_x,       ctx->d_h,       ctx->d_qkv,
                  ctx->d_q,       ctx->d_attn,  ctx->d_act,     ctx->d_meta,    ctx->d_logits,
-                 ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list};
+                 ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list,
+                 ctx->d_rstage[0], ctx->d_rstage[1]};
   for (void* p : dev)
     if (p) cudaFree(p);
   void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging};
@@ -151,11 +160,14 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
   for (auto e : ctx->ev_pool) cudaEventDestroy(e);
   for (auto e : ctx->ev_kv) cudaEventDestroy(e);
   for (auto e : ctx->ev_w) cudaEventDestroy(e);
+  for (auto e : ctx->ev_h2d) cudaEventDestroy(e);
+  for (auto e : ctx->ev_dec) cudaEventDestroy(e);
   cudaEvent_t evs[] = {ctx->ev_t0, ctx->ev_t1, ctx->ev_c0, ctx->ev_c1, ctx->ev_l0, ctx->ev_l1};
   for (auto e : evs)
     if (e) cudaEventDestroy(e);
   if (ctx->cs) cudaStreamDestroy(ctx->cs);
   if (ctx->xs) cudaStreamDestroy(ctx->xs);
+  if (ctx->ds) cudaStreamDestroy(ctx->ds);
   delete ctx;
   return MZC_OK;
 }
@@ -214,7 +226,14 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   if (s.d_model % 64 != 0) return ctx->fail(MZC_ERR_INVALID, "d_model must be a multiple of 64");
   if ((static_cast<int64_t>(s.n_q_heads) * s.head_dim) % 64 != 0)
     return ctx->fail(MZC_ERR_INVALID, "n_q_heads*head_dim must be a multiple of 64");
-  mzc_status ss = ctx->st.init(s, ctx->opt.pool_blocks, ctx->opt.host_store_bytes);
+  if (ctx->opt.swap_codec != MZC_CODEC_NONE && ctx->opt.swap_codec != MZC_CODEC_Q8)
+    return ctx->fail(MZC_ERR_INVALID, "unknown swap_codec");
+  ctx->codec = ctx->opt.swap_codec;
+  {
+    const int64_t block_elems = 2LL * s.n_kv_heads * 16 * s.head_dim;
+    ctx->slot_bytes = ctx->codec == MZC_CODEC_Q8 ? mzc::q8_block_bytes(block_elems) : 2 * block_elems;
+  }
+  mzc_status ss = ctx->st.init(s, ctx->opt.pool_blocks, ctx->opt.host_store_bytes, ctx->slot_bytes);
   if (ss != MZC_OK) return ctx->fail(ss, ctx->st.error());
   if (!weights || !weights->embed || !weights->lm_head || !weights->final_norm || !weights->layers)
     return ctx->fail(MZC_ERR_INVALID, "weights are incomplete");
@@ -231,6 +250,15 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
 
   CK(cudaStreamCreateWithFlags(&ctx->cs, cudaStreamNonBlocking));
   CK(cudaStreamCreateWithFlags(&ctx->xs, cudaStreamNonBlocking));
+  if (ctx->codec != MZC_CODEC_NONE) {
+    CK(cudaStreamCreateWithFlags(&ctx->ds, cudaStreamNonBlocking));
+    ctx->ev_h2d.assign(L, nullptr);
+    ctx->ev_dec.assign(L, nullptr);
+    for (int64_t l = 0; l < L; ++l) {
+      CK(cudaEventCreateWithFlags(&ctx->ev_h2d[l], cudaEventDisableTiming));
+      CK(cudaEventCreateWithFlags(&ctx->ev_dec[l], cudaEventDisableTiming));
+    }
+  }
   ctx->ev_kv.assign(L, nullptr);
   ctx->ev_w.assign(L, nullptr);
   for (int64_t l = 0; l < L; ++l) {
@@ -340,6 +368,8 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   CK(cudaMalloc(&ctx->d_status, 4));
   CK(cudaMemset(ctx->d_status, 0, 4));
   CK(cudaMalloc(&ctx->d_staging, ctx->nblk * ctx->block_bytes));
+  if (ctx->codec != MZC_CODEC_NONE)
+    for (auto& b : ctx->d_rstage) CK(cudaMalloc(&b, ctx->nblk * ctx->slot_bytes));
   CK(cudaMalloc(&ctx->d_list, L * ctx->nblk * 4));
   CK(cudaHostAlloc(&ctx->h_list, L * ctx->nblk * 4, cudaHostAllocDefault));
   CK(cudaHostAlloc(&ctx->h_staging, ctx->nblk * ctx->block_bytes, cudaHostAllocDefault));
@@ -361,8 +391,11 @@ mzc_status copy_out(mzc_ctx* ctx, const std::vector<mzc::EvictMove>& moves) {
   int64_t at = 0;
   for (auto& mv : moves) {
     const int64_t nb = static_cast<int64_t>(mv.phys.size());
-    CK(mzc::launch_gather_blocks(ctx->d_pool, ctx->d_list + at, nb, ctx->block_bytes, ctx->d_staging, ctx->cs));
-    CK(cudaMemcpyAsync(ctx->h_store + mv.host_off, ctx->d_staging, nb * ctx->block_bytes,
+    if (ctx->codec == MZC_CODEC_Q8)
+      CK(mzc::launch_q8_encode(ctx->d_pool, ctx->d_list + at, nb, ctx->block_bytes / 2, ctx->d_staging, ctx->cs));
+    else
+      CK(mzc::launch_gather_blocks(ctx->d_pool, ctx->d_list + at, nb, ctx->block_bytes, ctx->d_staging, ctx->cs));
+    CK(cudaMemcpyAsync(ctx->h_store + mv.host_off, ctx->d_staging, nb * ctx->slot_bytes,
                        cudaMemcpyDeviceToHost, ctx->cs));
     at += nb;
   }
@@ -709,7 +742,11 @@ mzc_status mzc_evict(mzc_ctx* ctx, int32_t l0, int32_t l1, int64_t t0, int64_t t
     int64_t split = n_ctx;
     if (ctx->policy == MZC_POLICY_COPY) split = p;
     else if (ctx->policy == MZC_POLICY_HYBRID) {
-      mzc_status e = mzc_plan_split(&ctx->shape, &ctx->prof, p, n_ctx, 0, &split);
+      // the model prices a copied block at its stored size over the link; a
+      // compressed store moves slot_bytes per block
+      mzc_profile pr = ctx->prof;
+      pr.h2d_gbs *= static_cast<double>(ctx->block_bytes) / static_cast<double>(ctx->slot_bytes);
+      mzc_status e = mzc_plan_split(&ctx->shape, &pr, p, n_ctx, 0, &split);
       if (e != MZC_OK) return ctx->fail(e, "hybrid split failed");
     }
     if (split > p) {
@@ -785,15 +822,48 @@ mzc_status mzc_restore_async(mzc_ctx* ctx) {
       ++wi;
     }
     CK(cudaEventRecord(ctx->ev_w[l], xs));
+    if (ctx->codec == MZC_CODEC_NONE) {
+      while (ri < runs.size() && runs[ri].layer == l) {
+        const mzc_copy_run& r = runs[ri++];
+        const int64_t nb = static_cast<int64_t>(r.n_blocks) * ctx->block_bytes;
+        CK(cudaMemcpyAsync(ctx->d_pool + r.phys_begin * ctx->block_bytes, ctx->h_store + r.host_off,
+                           nb, cudaMemcpyHostToDevice, xs));
+        bytes += nb;
+        ++copies;
+      }
+      CK(cudaEventRecord(ctx->ev_kv[l], xs));
+      continue;
+    }
+    // compressed: the layer's runs land packed in staging buffer l % 2 (free
+    // once layer l - 2 is decoded), then the decode stream writes the pool
+    const size_t r0 = ri;
+    uint8_t* stage = ctx->d_rstage[l & 1];
+    if (l >= 2) CK(cudaStreamWaitEvent(xs, ctx->ev_dec[l - 2], 0));
+    int64_t at = 0;
     while (ri < runs.size() && runs[ri].layer == l) {
       const mzc_copy_run& r = runs[ri++];
-      const int64_t nb = static_cast<int64_t>(r.n_blocks) * ctx->block_bytes;
-      CK(cudaMemcpyAsync(ctx->d_pool + r.phys_begin * ctx->block_bytes, ctx->h_store + r.host_off,
-                         nb, cudaMemcpyHostToDevice, xs));
+      const int64_t nb = static_cast<int64_t>(r.n_blocks) * ctx->slot_bytes;
+      CK(cudaMemcpyAsync(stage + at, ctx->h_store + r.host_off, nb, cudaMemcpyHostToDevice, xs));
+      at += nb;
       bytes += nb;
       ++copies;
     }
-    CK(cudaEventRecord(ctx->ev_kv[l], xs));
+    CK(cudaEventRecord(ctx->ev_h2d[l], xs));
+    CK(cudaStreamWaitEvent(ctx->ds, ctx->ev_h2d[l], 0));
+    at = 0;
+    for (size_t k = r0; k < ri; ++k) {
+      const mzc_copy_run& r = runs[k];
+      CK(mzc::launch_q8_decode(stage + at, r.n_blocks, ctx->block_bytes / 2, nullptr, r.phys_begin,
+                               ctx->shape.kv_dtype, ctx->d_pool, ctx->ds));
+      at += static_cast<int64_t>(r.n_blocks) * ctx->slot_bytes;
+    }
+    CK(cudaEventRecord(ctx->ev_dec[l], ctx->ds));
+    CK(cudaEventRecord(ctx->ev_kv[l], ctx->ds));
+  }
+  if (ctx->codec != MZC_CODEC_NONE) {
+    // the copy stream's end event covers the decodes
+    CK(cudaEventRecord(ctx->ev_dec[0], ctx->ds));
+    CK(cudaStreamWaitEvent(xs, ctx->ev_dec[0], 0));
   }
   CK(cudaEventRecord(ctx->ev_c1, xs));
   ctx->restore_issued = true;
@@ -1229,6 +1299,26 @@ mzc_status mzc_k_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_
     return MZC_ERR_CUDA;
   }
   return MZC_OK;
+}
+
+int64_t mzc_q8_block_bytes(int32_t hkv, int32_t hd) {
+  if (hkv <= 0 || hd <= 0 || hd % 64 != 0) return 0;
+  return mzc::q8_block_bytes(2LL * hkv * 16 * hd);
+}
+
+mzc_status mzc_k_q8_encode(const void* pool, const int32_t* phys, int64_t n, int32_t hkv, int32_t hd,
+                           void* out, void* stream) {
+  if (!pool || !phys || !out || n < 0 || hkv <= 0 || hd <= 0 || hd % 64 != 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_q8_encode(pool, phys, n, 2LL * hkv * 16 * hd, out, static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_q8_decode(const void* in, int64_t n, int32_t hkv, int32_t hd, const int32_t* phys,
+                           int64_t phys_begin, int32_t kv_dtype, void* pool, void* stream) {
+  if (!in || !pool || n < 0 || hkv <= 0 || hd <= 0 || hd % 64 != 0 || phys_begin < 0 ||
+      (kv_dtype != MZC_KV_BF16 && kv_dtype != MZC_KV_FP16))
+    return MZC_ERR_INVALID;
+  KCK(mzc::launch_q8_decode(in, n, 2LL * hkv * 16 * hd, phys, phys_begin, kv_dtype, pool,
+                            static_cast<cudaStream_t>(stream)));
 }
 
 mzc_status mzc_k_lm_head(const float* x_row, const float* g, int32_t d, float eps,

@@ -75,7 +75,8 @@ void RangeAlloc::release(int64_t start, int64_t n) {
 
 // ---- State --------------------------------------------------------------
 
-mzc_status State::init(const mzc_model_shape& s, int64_t pool_blocks, int64_t host_store_bytes) {
+mzc_status State::init(const mzc_model_shape& s, int64_t pool_blocks, int64_t host_store_bytes,
+                       int64_t slot_bytes) {
   if (s.n_layers <= 0 || s.d_model <= 0 || s.n_q_heads <= 0 || s.n_kv_heads <= 0 ||
       s.head_dim <= 0 || s.ffn_dim <= 0 || s.vocab <= 0 || s.max_ctx <= 0)
     return fail(MZC_ERR_INVALID, "shape fields must be positive");
@@ -87,9 +88,10 @@ mzc_status State::init(const mzc_model_shape& s, int64_t pool_blocks, int64_t ho
   shape_ = s;
   nblk_max_ = ceil_div(s.max_ctx, 16);
   block_bytes_ = 2LL * s.n_kv_heads * 16 * s.head_dim * 2;
+  slot_bytes_ = slot_bytes > 0 ? slot_bytes : block_bytes_;
   pool_blocks_ = pool_blocks > 0 ? pool_blocks : 2LL * s.n_layers * nblk_max_;
   if (pool_blocks_ >= (1LL << 31)) return fail(MZC_ERR_INVALID, "pool_blocks too large");
-  host_bytes_ = host_store_bytes > 0 ? host_store_bytes : (int64_t)s.n_layers * nblk_max_ * block_bytes_;
+  host_bytes_ = host_store_bytes > 0 ? host_store_bytes : (int64_t)s.n_layers * nblk_max_ * slot_bytes_;
   tab_.assign((size_t)s.n_layers * nblk_max_, BlockEntry{});
   regions_.clear();
   w_state_.assign(s.n_layers, MZC_RESIDENT);
@@ -104,7 +106,7 @@ mzc_status State::init(const mzc_model_shape& s, int64_t pool_blocks, int64_t ho
 void State::drop_region_slot(int32_t r) {
   Region& R = regions_[r];
   if (--R.live == 0) {
-    host_.release(R.host_off, (int64_t)R.n_slots * block_bytes_);
+    host_.release(R.host_off, (int64_t)R.n_slots * slot_bytes_);
     R.n_slots = 0;
   }
 }
@@ -145,7 +147,7 @@ mzc_status State::evict_range(int32_t l0, int32_t l1, int64_t t0, int64_t t1, in
     return MZC_OK;
   }
   // COPY: one packed region per layer, blocks in logical order.
-  const int64_t per_layer = (b1 - b0) * block_bytes_;
+  const int64_t per_layer = (b1 - b0) * slot_bytes_;
   std::vector<int64_t> offs;
   for (int32_t l = l0; l < l1; ++l) {
     int64_t off = host_.alloc_contig(per_layer);
@@ -202,10 +204,10 @@ mzc_status State::evict_blocks(const int32_t* layer, const int64_t* blk, int64_t
   std::vector<int64_t> offs(L, -1);
   for (int32_t l = 0; l < L; ++l) {
     if (per[l].empty()) continue;
-    offs[l] = host_.alloc_contig((int64_t)per[l].size() * block_bytes_);
+    offs[l] = host_.alloc_contig((int64_t)per[l].size() * slot_bytes_);
     if (offs[l] < 0) {
       for (int32_t j = 0; j < l; ++j)
-        if (offs[j] >= 0) host_.release(offs[j], (int64_t)per[j].size() * block_bytes_);
+        if (offs[j] >= 0) host_.release(offs[j], (int64_t)per[j].size() * slot_bytes_);
       return fail(MZC_ERR_OOM, "pinned swap store is full");
     }
   }
@@ -282,12 +284,12 @@ mzc_status State::plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int3
           BlockEntry& e = at(l, blocks[bi]);
           e.st = MZC_INFLIGHT;
           e.phys = (int32_t)(rg.first + j);
-          int64_t off = R.host_off + (int64_t)e.idx * block_bytes_;
+          int64_t off = R.host_off + (int64_t)e.idx * slot_bytes_;
           // extend the previous run when host and device are both contiguous
           if (runs && !runs->empty()) {
             mzc_copy_run& pr = runs->back();
             if (pr.layer == l && pr.phys_begin + pr.n_blocks == e.phys &&
-                pr.host_off + (int64_t)pr.n_blocks * block_bytes_ == off) {
+                pr.host_off + (int64_t)pr.n_blocks * slot_bytes_ == off) {
               pr.n_blocks += 1;
               continue;
             }

@@ -72,12 +72,16 @@ struct PrefillPlan {
 
 class State {
  public:
-  mzc_status init(const mzc_model_shape& s, int64_t pool_blocks, int64_t host_store_bytes);
+  // slot_bytes: pinned-store bytes per swapped block (0 = block_bytes, the
+  // block as stored; less when the swap codec compresses it)
+  mzc_status init(const mzc_model_shape& s, int64_t pool_blocks, int64_t host_store_bytes,
+                  int64_t slot_bytes = 0);
 
   const mzc_model_shape& shape() const { return shape_; }
   int64_t n_ctx() const { return n_ctx_; }
   int64_t nblk_max() const { return nblk_max_; }
   int64_t block_bytes() const { return block_bytes_; }
+  int64_t slot_bytes() const { return slot_bytes_; }
   int64_t pool_blocks() const { return pool_blocks_; }
   int64_t host_store_bytes() const { return host_bytes_; }
   const std::string& error() const { return err_; }
@@ -130,7 +134,7 @@ class State {
   void drop_region_slot(int32_t r);
 
   mzc_model_shape shape_{};
-  int64_t nblk_max_ = 0, block_bytes_ = 0, pool_blocks_ = 0, host_bytes_ = 0;
+  int64_t nblk_max_ = 0, block_bytes_ = 0, slot_bytes_ = 0, pool_blocks_ = 0, host_bytes_ = 0;
   int64_t n_ctx_ = 0;
   std::vector<BlockEntry> tab_;
   std::vector<Region> regions_;

@@ -17,6 +17,7 @@ _lib = None
 MZC_OK, MZC_ERR_INVALID, MZC_ERR_RANGE, MZC_ERR_STATE = 0, 1, 2, 3
 MZC_ERR_OOM, MZC_ERR_CUDA, MZC_ERR_TIMEOUT, MZC_ERR_DEVICE = 4, 5, 6, 7
 MZC_KV_BF16, MZC_KV_FP16 = 0, 1
+MZC_CODEC_NONE, MZC_CODEC_Q8 = 0, 1
 MZC_COPY, MZC_DROP, MZC_AUTO = 0, 1, 2
 MZC_POLICY_COPY, MZC_POLICY_RECOMPUTE, MZC_POLICY_HYBRID = 0, 1, 2
 MZC_RESIDENT, MZC_SWAPPED, MZC_DROPPED, MZC_INFLIGHT, MZC_EMPTY = 0, 1, 2, 3, 4
@@ -36,7 +37,7 @@ class mzc_model_shape(ctypes.Structure):
 
 class mzc_options(ctypes.Structure):
     _fields_ = [("pool_blocks", c_i64), ("max_rows", c_i64), ("host_store_bytes", c_i64),
-                ("overlap", c_i32), ("device", c_i32)]
+                ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32)]
 
 
 class mzc_layer_weights(ctypes.Structure):
@@ -121,10 +122,13 @@ _SIGS = {
     "mzc_k_attention_noalloc": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64,
                                 c_i32, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
+    "mzc_k_q8_encode": [c_vp, c_vp, c_i64, c_i32, c_i32, c_vp, c_vp],
+    "mzc_k_q8_decode": [c_vp, c_i64, c_i32, c_i32, c_vp, c_i64, c_i32, c_vp, c_vp],
     "mzc_k_embed": [c_vp, c_i64, c_vp, c_i32, c_i64, c_vp, c_vp, c_vp],
 }
 _RESTYPES = {"mzc_last_error": (ctypes.c_char_p, [c_vp]),
-             "mzc_k_attention_scratch_bytes": (c_i64, [c_i64, c_i32, c_i32, c_i32, c_i64])}
+             "mzc_k_attention_scratch_bytes": (c_i64, [c_i64, c_i32, c_i32, c_i32, c_i64]),
+             "mzc_q8_block_bytes": (c_i64, [c_i32, c_i32])}
 
 
 def lib_path() -> str:
@@ -213,9 +217,9 @@ def make_weights(weights: dict):
 # ---- ctx entry points (same names as the C ABI) -------------------------
 
 def mzc_create(shape: dict, weights: dict, pool_blocks=0, max_rows=0, host_store_bytes=0,
-               overlap=1, device=0):
+               overlap=1, device=0, swap_codec=MZC_CODEC_NONE):
     sh = make_shape(shape)
-    opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device)
+    opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec)
     w, keep = make_weights(weights)
     out = c_vp()
     _call("mzc_create", ctypes.byref(sh), ctypes.byref(opt), ctypes.byref(w), ctypes.byref(out))
@@ -413,3 +417,16 @@ def mzc_k_lm_head(x_row, g, d, eps, w, vocab, logits, stream=None):
 
 def mzc_k_embed(tokens, n, embed, d, vocab, x, status, stream=None):
     return _call("mzc_k_embed", _ptr(tokens), n, _ptr(embed), d, vocab, _ptr(x), _ptr(status), stream)
+
+
+def mzc_q8_block_bytes(hkv, hd) -> int:
+    return load().mzc_q8_block_bytes(hkv, hd)
+
+
+def mzc_k_q8_encode(pool, phys, n, hkv, hd, out, stream=None):
+    return _call("mzc_k_q8_encode", _ptr(pool), _ptr(phys), n, hkv, hd, _ptr(out), stream)
+
+
+def mzc_k_q8_decode(inp, n, hkv, hd, phys, phys_begin, kv_dtype, pool, stream=None):
+    return _call("mzc_k_q8_decode", _ptr(inp), n, hkv, hd, _ptr(phys), phys_begin, kv_dtype,
+                 _ptr(pool), stream)

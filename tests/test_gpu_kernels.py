@@ -108,6 +108,42 @@ def test_gemm_writes_only_its_rows(epi, mm, nn):
     assert not np.any(np.all(host[:mm] == sentinel, axis=1))
 
 
+# ---- 8-bit swap codec ------------------------------------------------------------
+
+@pytest.mark.parametrize("hkv,hd,kvd", [(2, 64, 1), (8, 128, 0), (8, 64, 1)])
+def test_q8_codec_matches_oracle(hkv, hd, kvd):
+    """Encoded bytes (codes and fp32 min/step) and decoded fp16 bits equal the
+    oracle's, through a block list and into a contiguous run."""
+    torch = _torch()
+    e = 2 * hkv * 16 * hd
+    nb = 12
+    rng = np.random.default_rng(hd + hkv)
+    vals = (rng.standard_normal((nb, e)) * np.exp(rng.uniform(-3, 2, (nb, 1)))).astype(np.float32)
+    bits = oracle.to_f16_bits(oracle.round_kv(vals, kvd))  # as the pool stores values
+    bits[3, :64] = bits[3, 0]                                 # a constant group
+    pool = torch.from_numpy(bits.view(np.int16)).cuda()
+    phys = np.array([7, 2, 11, 3, 0], np.int32)
+    cb = m.mzc_q8_block_bytes(hkv, hd)
+    assert cb == oracle.q8_block_bytes(hkv, hd)
+    comp = torch.zeros((len(phys), cb), dtype=torch.uint8, device="cuda")
+    m.mzc_k_q8_encode(pool, i32_dev(phys), len(phys), hkv, hd, comp)
+    torch.cuda.synchronize()
+    ref = oracle.q8_encode_blocks(bits[phys])
+    assert np.array_equal(comp.cpu().numpy(), ref)
+    dec = oracle.q8_decode_blocks(ref, e, kvd)
+    out = torch.zeros((nb, e), dtype=torch.int16, device="cuda")
+    dst = np.array([1, 9, 4, 10, 6], np.int32)
+    m.mzc_k_q8_decode(comp, len(phys), hkv, hd, i32_dev(dst), 0, kvd, out)
+    run = torch.zeros((nb, e), dtype=torch.int16, device="cuda")
+    m.mzc_k_q8_decode(comp, 3, hkv, hd, None, 5, kvd, run)
+    torch.cuda.synchronize()
+    got, got_run = to_np_u16(out), to_np_u16(run)
+    assert np.array_equal(got[dst], dec)
+    assert np.array_equal(got_run[5:8], dec[:3])
+    untouched = np.setdiff1d(np.arange(nb), dst)
+    assert not got[untouched].any() and not got_run[:5].any() and not got_run[8:].any()
+
+
 # ---- RMSNorm, embedding, LM head --------------------------------------------
 
 @pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072), (5, 320), (3, 4608), (9, 4096)])
