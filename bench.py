@@ -134,7 +134,7 @@ class Runner:
     """Owns one ctx on one GPU and knows how to put the evicted state at rest
     (untimed) and run one timed restore + prefill."""
 
-    def __init__(self, name, sc, device):
+    def __init__(self, name, sc, device, codec=0):
         import synth
         import paper_2609_01338_gb300 as m
         self.m, self.name, self.sc = m, name, sc
@@ -147,7 +147,7 @@ class Runner:
         self.prompt = synth.tokens(synth.SEED_PROMPT, 0, sc["prompt"], sh["vocab"])
         max_rows = min(sh["max_ctx"], 16384 + 1024)
         t = time.time()
-        self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device)
+        self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device, swap_codec=codec)
         self.t_create = time.time() - t
         t = time.time()
         m.mzc_prefill(self.c, self.ctx_tokens)  # long contexts run in causal chunks
@@ -198,7 +198,7 @@ class Runner:
                 m.mzc_evict(self.c, 0, L, p, N, m.MZC_DROP)
                 self.rec = (p, N - p)
             else:
-                s = m.mzc_plan_split(self.shape, self.profile, p, N, self.sc["prompt"])
+                s = m.mzc_plan_split_ctx(self.c, p, self.sc["prompt"])
                 if s > p:
                     m.mzc_evict(self.c, 0, L, p, s, m.MZC_DROP)
                     self.rec = (p, s - p)
@@ -305,6 +305,8 @@ def main():
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
     ap.add_argument("--policies", default=None, help="comma list overriding the sweep's policies")
+    ap.add_argument("--codec", default="none", choices=["none", "q8"],
+                    help="swap codec of the pinned store: none, or 8-bit groups (q8)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mzc":
         args.warmup = 3
@@ -336,7 +338,7 @@ def main():
     __graft_entry__.build()
     import paper_2609_01338_gb300 as m
 
-    r = Runner(name, sc, local)
+    r = Runner(name, sc, local, codec=1 if args.codec == "q8" else 0)
     if name == "3b_sweep":
         r.profile = m.mzc_profile_measure(r.c)
         run_sweep(r, args, rank)
@@ -419,7 +421,7 @@ def main():
         "ms_per_step": round(statistics.mean(dev), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": {"workload": _describe(name, sc),
+        "config": {"workload": _describe(name, sc), "swap_codec": args.codec,
                    "l2": "inputs larger than L2 (weights + KV >> 129 MB)",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "timed": "restore + recompute + prompt prefill + logits D2H per step; eviction between steps untimed"},
@@ -486,7 +488,7 @@ def run_sweep(r, args, rank):
         best = {}
         for p in pts:
             best.setdefault(p["fraction"], {})[p["policy"]] = p["ttft_ms"]
-        print(json.dumps({"metric": METRIC, "workload": _describe("3b_sweep", r.sc),
+        print(json.dumps({"metric": METRIC, "workload": _describe("3b_sweep", r.sc), "swap_codec": args.codec,
                           "profile": {k: getattr(r.profile, k) for k, _ in r.profile._fields_},
                           "sweep": best, "points": pts}), flush=True)
 

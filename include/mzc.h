@@ -195,15 +195,20 @@ mzc_status mzc_recompute_tail(mzc_ctx *ctx, int64_t p, int64_t n);
 mzc_status mzc_set_policy(mzc_ctx *ctx, int32_t policy, const mzc_profile *profile);
 
 /* Hybrid split (pure host arithmetic): for an evicted tail [p, n_ctx) and a
- * prompt of n_prompt tokens, the block-aligned s in [p, n_ctx] at which the
- * recompute of [p, s) (fused with the prompt) and the copy of [s, n_ctx)
- * finish together, i.e. that minimises the predicted
- * max(T_compute(p, s), T_copy(s, n_ctx) + last-layer tail) under the
- * profile's linear per-unit costs (Sec. 4.3, split in inverse proportion to
- * per-unit times).  Returns s = p (copy only) unless the split is predicted
- * to be at least 3% faster. */
+ * prompt of n_prompt tokens, the block-aligned s in [p, n_ctx] such that
+ * recomputing [p, s) (fused with the prompt) while [s, n_ctx) is copied
+ * minimises the predicted TTFT (Sec. 4.3: the two paths balanced by their
+ * profiled per-unit times).  The prediction runs the paths layer by layer:
+ * a layer's QKV projection, rotary/KV write and attention of recomputed rows
+ * never wait; the rest of layer l starts once layer l's copy (copy time / L
+ * each, in layer order) has landed.  Returns s = p (copy only) unless the
+ * split is predicted to be at least 5% faster. */
 mzc_status mzc_plan_split(const mzc_model_shape *shape, const mzc_profile *profile, int64_t p,
                           int64_t n_ctx, int64_t n_prompt, int64_t *s_out);
+/* The same split for this ctx's context, with its profile (mzc_set_policy or
+ * mzc_profile_measure) and its swap codec: a compressed store moves
+ * mzc_q8_block_bytes per block over the link. */
+mzc_status mzc_plan_split_ctx(mzc_ctx *ctx, int64_t p, int64_t n_prompt, int64_t *s_out);
 
 /* Measures the per-unit profile on this ctx's device (the paper's one-time
  * offline profiling, Sec. 4.3): timed host->device copies from the pinned

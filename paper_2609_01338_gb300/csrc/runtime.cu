@@ -742,11 +742,7 @@ mzc_status mzc_evict(mzc_ctx* ctx, int32_t l0, int32_t l1, int64_t t0, int64_t t
     int64_t split = n_ctx;
     if (ctx->policy == MZC_POLICY_COPY) split = p;
     else if (ctx->policy == MZC_POLICY_HYBRID) {
-      // the model prices a copied block at its stored size over the link; a
-      // compressed store moves slot_bytes per block
-      mzc_profile pr = ctx->prof;
-      pr.h2d_gbs *= static_cast<double>(ctx->block_bytes) / static_cast<double>(ctx->slot_bytes);
-      mzc_status e = mzc_plan_split(&ctx->shape, &pr, p, n_ctx, 0, &split);
+      mzc_status e = mzc_plan_split_ctx(ctx, p, 0, &split);
       if (e != MZC_OK) return ctx->fail(e, "hybrid split failed");
     }
     if (split > p) {
@@ -912,6 +908,16 @@ mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profi
   if (best_t > 0.95 * copy_only) best = p;
   *s_out = best;
   return MZC_OK;
+}
+
+mzc_status mzc_plan_split_ctx(mzc_ctx* ctx, int64_t p, int64_t n_prompt, int64_t* s_out) {
+  if (!ctx || !s_out) return MZC_ERR_INVALID;
+  // the model prices a copied block at its stored size over the link; a
+  // compressed store moves slot_bytes per block
+  mzc_profile pr = ctx->prof;
+  pr.h2d_gbs *= static_cast<double>(ctx->block_bytes) / static_cast<double>(ctx->slot_bytes);
+  mzc_status e = mzc_plan_split(&ctx->shape, &pr, p, ctx->st.n_ctx(), n_prompt, s_out);
+  return e == MZC_OK ? e : ctx->fail(e, "hybrid split failed");
 }
 
 mzc_status mzc_truncate(mzc_ctx* ctx, int64_t n_ctx) {

@@ -122,6 +122,7 @@ _SIGS = {
     "mzc_k_attention_noalloc": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64,
                                 c_i32, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
+    "mzc_plan_split_ctx": [c_vp, c_i64, c_i64, c_vp],
     "mzc_k_q8_encode": [c_vp, c_vp, c_i64, c_i32, c_i32, c_vp, c_vp],
     "mzc_k_q8_decode": [c_vp, c_i64, c_i32, c_i32, c_vp, c_i64, c_i32, c_vp, c_vp],
     "mzc_k_embed": [c_vp, c_i64, c_vp, c_i32, c_i64, c_vp, c_vp, c_vp],
@@ -269,6 +270,12 @@ def mzc_plan_split(shape: dict, profile: mzc_profile | None, p, n_ctx, n_prompt)
     out = c_i64()
     _call("mzc_plan_split", ctypes.byref(sh), ctypes.byref(profile) if profile else None, p,
           n_ctx, n_prompt, ctypes.byref(out))
+    return out.value
+
+
+def mzc_plan_split_ctx(ctx, p, n_prompt) -> int:
+    out = c_i64()
+    _call("mzc_plan_split_ctx", ctx, p, n_prompt, ctypes.byref(out), ctx=ctx)
     return out.value
 
 
