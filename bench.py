@@ -300,7 +300,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="mzc", choices=["mzc", "reference"])
     ap.add_argument("--workload", default="1b_recompute",
-                    choices=["1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed", "3b_sweep"])
+                    choices=["1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed", "3b_sweep",
+                             "3b_order"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
@@ -342,6 +343,10 @@ def main():
     if name == "3b_sweep":
         r.profile = m.mzc_profile_measure(r.c)
         run_sweep(r, args, rank)
+        r.close()
+        return
+    if name == "3b_order":
+        run_order(r, args, rank)
         r.close()
         return
     # warm-up; the last warm-up step times every kernel class to find the
@@ -491,6 +496,44 @@ def run_sweep(r, args, rank):
         print(json.dumps({"metric": METRIC, "workload": _describe("3b_sweep", r.sc), "swap_codec": args.codec,
                           "profile": {k: getattr(r.profile, k) for k, _ in r.profile._fields_},
                           "sweep": best, "points": pts}), flush=True)
+
+
+def run_order(r, args, rank):
+    """Eviction-order ablation (Sec. 6.3, Fig. 12b): the same number of whole
+    layers (weights and every KV block) swapped out backward-out, forward-out or
+    at random, restored forward-in while the prompt runs."""
+    import synth
+    m, L, N = r.m, r.shape["n_layers"], r.N
+    res, pts = {}, []
+    for frac in r.sc["fractions"]:
+        k = int(round(frac * L))
+        for order in r.sc["orders"]:
+            if order == "backward":
+                draws = [list(range(L - k, L))]
+            elif order == "forward":
+                draws = [list(range(k))]
+            else:
+                draws = [sorted(synth.permutation(synth.SEED_EVICT, 10 + d, L)[:k].tolist())
+                         for d in range(r.sc["random_draws"])]
+            vals = []
+            for layers in draws:
+                for i in range(args.warmup + args.steps):
+                    for l in layers:
+                        m.mzc_evict_weights(r.c, l, l + 1)
+                        m.mzc_evict(r.c, l, l + 1, 0, N, m.MZC_COPY)
+                    d, h, st, times = r.step()
+                    if i >= args.warmup:
+                        vals.append(d)
+            pt = {"fraction": frac, "order": order, "layers_per_draw": k, "draws": len(draws),
+                  "ttft_ms": round(statistics.median(vals), 3),
+                  "p10": round(float(np.percentile(vals, 10)), 3),
+                  "p90": round(float(np.percentile(vals, 90)), 3)}
+            pts.append(pt)
+            res.setdefault(frac, {})[order] = pt["ttft_ms"]
+            print(json.dumps(pt), file=sys.stderr, flush=True)
+    if rank == 0:
+        print(json.dumps({"metric": "TTFT ms by eviction order", "workload": _describe("3b_order", r.sc),
+                          "swap_codec": args.codec, "order": res, "points": pts}), flush=True)
 
 
 if __name__ == "__main__":

@@ -45,6 +45,12 @@ SCENARIOS = {
     # 3B sweep: evicted fraction of the token tail x {copy, recompute, hybrid}, 128-token prompt
     "3b_sweep": dict(model=THREE_B, context=32768, fractions=(0.0, 0.10, 0.25, 0.50, 0.75, 1.0),
                      policies=("copy", "recompute", "hybrid"), prompt=128),
+    # 3B eviction-order ablation (Sec. 6.3): a fraction of the layers (weights and
+    # every KV block) swapped to pinned host, chosen backward-out (last layers),
+    # forward-out (first layers) or random-out (seeded, several draws); restore
+    # forward-in, 128-token prompt
+    "3b_order": dict(model=THREE_B, context=32768, fractions=(0.25, 0.50),
+                     orders=("backward", "forward", "random"), random_draws=5, prompt=128),
 }
 
 
