@@ -162,26 +162,6 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-template <int N>
-__device__ __forceinline__ void tmem_ld_row(uint32_t taddr, float* v) {
-  if constexpr (N == 64) {
-    tmem_ld64w(taddr, v);
-  } else {
-    static_assert(N == 32, "row slices of 32 or 64 columns");
-    tmem_ld32w(taddr, v);
-  }
-}
-
-template <int N>
-__device__ __forceinline__ void tmem_st_row(uint32_t taddr, const float* v) {
-  if constexpr (N == 64) {
-    tmem_st64w(taddr, v);
-  } else {
-    static_assert(N == 32, "row slices of 32 or 64 columns");
-    tmem_st32w(taddr, v);
-  }
-}
-
 // Threads: warps 0-3 and 4-7 are the softmax warpgroups of Q tiles 0 and 1
 // (thread = row of its tile, whole rows of S), warp 8 is the TMA producer and
 // TMEM owner, warps 9 and 10 issue the UMMAs of Q tiles 0 and 1.  Both Q tiles
