@@ -301,7 +301,7 @@ def main():
     ap.add_argument("--impl", default="mzc", choices=["mzc", "reference"])
     ap.add_argument("--workload", default="1b_recompute",
                     choices=["1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed", "3b_sweep",
-                             "3b_order"])
+                             "3b_order", "1b_decode", "3b_decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
@@ -347,6 +347,10 @@ def main():
         return
     if name == "3b_order":
         run_order(r, args, rank)
+        r.close()
+        return
+    if name.endswith("_decode"):
+        run_decode(r, args, rank)
         r.close()
         return
     # warm-up; the last warm-up step times every kernel class to find the
@@ -534,6 +538,37 @@ def run_order(r, args, rank):
     if rank == 0:
         print(json.dumps({"metric": "TTFT ms by eviction order", "workload": _describe("3b_order", r.sc),
                           "swap_codec": args.codec, "order": res, "points": pts}), flush=True)
+
+
+def run_decode(r, args, rank):
+    """Decode after the first token: greedy single-token steps over the
+    resident context (each step is a one-row prefill through the same path)."""
+    m, sh = r.m, r.shape
+    tok = np.array([int(r.prompt[0])], np.int32)
+    vals = []
+    for i in range(args.warmup + args.steps):
+        m.mzc_prefill(r.c, tok, r.logits)
+        t = m.mzc_last_times(r.c)
+        tok = np.array([int(np.argmax(r.logits))], np.int32)
+        if i >= args.warmup:
+            vals.append(float(t[3]))
+    # one more step with every kernel class timed (not part of the median)
+    m.mzc_set_kernel_timing(r.c, -1)
+    m.mzc_prefill(r.c, tok, r.logits)
+    ks = {nm: round(m.mzc_kernel_stats(r.c, j).ms, 4) for j, nm in enumerate(m.KERNEL_CLASS_NAMES)}
+    m.mzc_set_kernel_timing(r.c, 0)
+    m.mzc_truncate(r.c, r.N)
+    ms = statistics.median(vals)
+    d, hq, hkv, hd, L = (sh[k] for k in ("d_model", "n_q_heads", "n_kv_heads", "head_dim", "n_layers"))
+    params = L * (d * (hq + 2 * hkv) * hd + hq * hd * d + 3 * d * sh["ffn_dim"]) + sh["vocab"] * d
+    kv = L * r.N * 2 * hkv * hd * 2
+    bytes_step = 2 * params + kv
+    if rank == 0:
+        print(json.dumps({"metric": "decode ms per token", "workload": _describe(r.name, r.sc),
+                          "value": round(ms, 3), "unit": "ms", "tokens_per_s": round(1e3 / ms, 1),
+                          "bytes_per_token": int(bytes_step),
+                          "hbm_gbs": round(bytes_step / (ms * 1e-3) / 1e9, 1),
+                          "kernel_ms_per_token": ks}), flush=True)
 
 
 if __name__ == "__main__":

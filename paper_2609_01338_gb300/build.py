@@ -18,8 +18,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmzc.so")
 
-CU_SOURCES = ["gemm.cu", "attention.cu", "attention_noalloc.cu", "elementwise.cu", "codec.cu",
-              "runtime.cu"]
+CU_SOURCES = ["gemm.cu", "gemv.cu", "attention.cu", "attention_noalloc.cu", "elementwise.cu",
+              "codec.cu", "runtime.cu"]
 CXX_SOURCES = ["state.cpp", "state_api.cpp"]
 HEADERS = ["ptx.cuh", "kernels.hpp", "state.hpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

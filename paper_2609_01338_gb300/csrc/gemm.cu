@@ -389,6 +389,7 @@ uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue) {
 }
 
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) {
+  gw->ptr = static_cast<const uint16_t*>(base);
   return make_tmap_f16(&gw->box64, base, n, k, 64) && make_tmap_f16(&gw->box128, base, n, k, 128) &&
          make_tmap_f16(&gw->box256, base, n, k, 256);
 }
@@ -398,8 +399,11 @@ bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) 
 // takes the width that keeps the most SMs busy in the fewest waves, with a
 // deeper ring for the narrower tiles.  The W map passed has the matching box.
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
-                        int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
+                        int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
+                        const uint16_t* a_ptr) {
   if (m <= 0) return cudaSuccess;
+  if (a_ptr && w.ptr && m <= kGemvMaxRows)
+    return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, st);
   const uint32_t bn = gemm_box_n(m, n, epilogue);
   if (bn == 256) {
     switch (epilogue) {

@@ -1,0 +1,143 @@
+// Projections of one to four rows (decode steps): out[m][n] = epilogue(sum_k
+// A[m][k] W[n][k]) with the weight matrix streamed once from HBM.  At these
+// row counts the product is bound by the weight bytes; the tensor-core GEMM
+// would pad every row to a 128-row tile and keep only its ring of weight
+// tiles in flight per SM.  Here one warp owns one output row of W (SwiGLU:
+// the gate and up rows of one output column), reads it with 16-byte
+// non-caching loads, several in flight per lane, and reduces with shuffles;
+// the few activation rows come through L1.  fp32 accumulation; the
+// epilogues are the GEMM's (fp16 store, fp32 residual add, SwiGLU).
+#include <cuda_fp16.h>
+
+#include "kernels.hpp"
+
+namespace mzc {
+
+namespace {
+
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ float dot8(const uint4& w, const uint4& a) {
+  const __half2* wh = reinterpret_cast<const __half2*>(&w);
+  const __half2* ah = reinterpret_cast<const __half2*>(&a);
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 wf = __half22float2(wh[i]), af = __half22float2(ah[i]);
+    s = fmaf(wf.x, af.x, s);
+    s = fmaf(wf.y, af.y, s);
+  }
+  return s;
+}
+
+__device__ __forceinline__ float silu_g(float g) { return g / (1.0f + __expf(-g)); }
+
+// R weight rows per warp (2 for SwiGLU), MR activation rows (m <= MR).
+template <int EPI, int MR>
+__global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ a,
+                                                   const uint16_t* __restrict__ w,
+                                                   void* __restrict__ out, int m, int n, int k) {
+  constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
+  const int lane = threadIdx.x & 31;
+  const int j = static_cast<int>((static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5);
+  const int n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
+  if (j >= n_out) return;
+  int rows[R];
+  if constexpr (EPI == EPI_SWIGLU_BF16) {
+    rows[0] = (j / kSwigluGroup) * 2 * kSwigluGroup + j % kSwigluGroup;  // gate
+    rows[1] = rows[0] + kSwigluGroup;                                    // up
+  } else {
+    rows[0] = j;
+  }
+  float acc[R][MR];
+#pragma unroll
+  for (int r = 0; r < R; ++r)
+#pragma unroll
+    for (int i = 0; i < MR; ++i) acc[r][i] = 0.0f;
+  const int chunks = k / 8;  // 16-byte chunks per row
+  constexpr int U = 4;       // chunks in flight per lane and row
+  for (int c0 = lane; c0 < chunks; c0 += 32 * U) {
+    uint4 wv[R][U];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int c = c0 + 32 * u;
+        wv[r][u] = c < chunks ? ld_stream(reinterpret_cast<const uint4*>(w + static_cast<int64_t>(rows[r]) * k) + c)
+                              : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int c = c0 + 32 * u;
+      if (c >= chunks) break;
+#pragma unroll
+      for (int i = 0; i < MR; ++i) {
+        if (i >= m) break;
+        const uint4 av = __ldg(reinterpret_cast<const uint4*>(a + static_cast<int64_t>(i) * k) + c);
+#pragma unroll
+        for (int r = 0; r < R; ++r) acc[r][i] += dot8(wv[r][u], av);
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < R; ++r)
+#pragma unroll
+    for (int i = 0; i < MR; ++i)
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[r][i] += __shfl_xor_sync(0xffffffffu, acc[r][i], o);
+  if (lane != 0) return;
+#pragma unroll
+  for (int i = 0; i < MR; ++i) {
+    if (i >= m) break;
+    if constexpr (EPI == EPI_STORE_BF16) {
+      static_cast<__half*>(out)[static_cast<int64_t>(i) * n + j] = __float2half_rn(acc[0][i]);
+    } else if constexpr (EPI == EPI_ADD_F32) {
+      static_cast<float*>(out)[static_cast<int64_t>(i) * n + j] += acc[0][i];
+    } else {
+      static_cast<__half*>(out)[static_cast<int64_t>(i) * n_out + j] =
+          __float2half_rn(silu_g(acc[0][i]) * acc[1][i]);
+    }
+  }
+}
+
+template <int EPI, int MR>
+cudaError_t launch_mr(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
+                      int64_t k, cudaStream_t st) {
+  const int64_t n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
+  const int64_t threads = n_out * 32;
+  gemv_kernel<EPI, MR><<<static_cast<unsigned>((threads + 255) / 256), 256, 0, st>>>(
+      a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k));
+  return cudaGetLastError();
+}
+
+template <int EPI>
+cudaError_t launch_epi(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
+                       int64_t k, cudaStream_t st) {
+  return m == 1 ? launch_mr<EPI, 1>(a, w, out, m, n, k, st) : launch_mr<EPI, 4>(a, w, out, m, n, k, st);
+}
+
+}  // namespace
+
+cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
+                        int64_t k, int epilogue, cudaStream_t st) {
+  if (m <= 0) return cudaSuccess;
+  if (m > kGemvMaxRows || k % 8 != 0) return cudaErrorInvalidValue;
+  switch (epilogue) {
+    case EPI_STORE_BF16:
+      return launch_epi<EPI_STORE_BF16>(a, w, out, m, n, k, st);
+    case EPI_ADD_F32:
+      return launch_epi<EPI_ADD_F32>(a, w, out, m, n, k, st);
+    case EPI_SWIGLU_BF16:
+      return launch_epi<EPI_SWIGLU_BF16>(a, w, out, m, n, k, st);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace mzc

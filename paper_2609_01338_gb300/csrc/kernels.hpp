@@ -23,6 +23,7 @@ bool make_tmap_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 // pick (box rows 64, 128 and 256).
 struct GemmWeight {
   CUtensorMap box64, box128, box256;
+  const uint16_t* ptr = nullptr;  // W itself, for the few-row GEMV
 };
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 
@@ -30,7 +31,15 @@ bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 // whose box matches the tile width gemm_box_n(m, n, epilogue) selects.
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
-                        int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st);
+                        int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
+                        const uint16_t* a_ptr = nullptr);
+
+// Few-row projections (decode steps; gemv.cu): A fp16 [m][k], W fp16 [n][k],
+// same epilogues as the GEMM; launch_gemm takes this path for m <= kGemvMaxRows
+// when it is given the activation pointer.
+constexpr int kGemvMaxRows = 4;
+cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
+                        int64_t k, int epilogue, cudaStream_t st);
 
 // 8-bit swap codec (codec.cu).  block_elems = 2 * hkv * 16 * hd.
 int64_t q8_block_bytes(int64_t block_elems);

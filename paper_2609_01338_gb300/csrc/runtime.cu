@@ -542,10 +542,14 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
       return mzc::launch_embed(ctok, cr, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
     }));
-    auto gemm = [&](const CUtensorMap& ta, const mzc::GemmWeight& w, void* out, int64_t N, int64_t K, int epi) {
+    auto gemm = [&](const CUtensorMap& ta, const void* a_ptr, const mzc::GemmWeight& w, void* out,
+                    int64_t N, int64_t K, int epi) {
       const double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
       return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
-                     [&] { return mzc::launch_gemm(ta, w, out, cr, N, K, epi, ctx->d_status, cs); });
+                     [&] {
+                       return mzc::launch_gemm(ta, w, out, cr, N, K, epi, ctx->d_status, cs,
+                                               static_cast<const uint16_t*>(a_ptr));
+                     });
     };
     // attention of chunk rows [r0, r0 + nr) (r0 relative to the chunk)
     auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab) {
@@ -570,7 +574,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
         return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
       }));
-      CKP(gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
+      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
       if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
       CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
         return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
@@ -588,12 +592,12 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         if (wait_rec || wait_prm) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
         CKP(attention(0, cr, max_keys, ltab));
       }
-      CKP(gemm(ctx->tm_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
+      CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
       CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
         return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
       }));
-      CKP(gemm(ctx->tm_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
-      CKP(gemm(ctx->tm_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
+      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
+      CKP(gemm(ctx->tm_act, ctx->d_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
     }
     last_rows = cr;
   }
@@ -1231,7 +1235,7 @@ mzc_status mzc_k_gemm(const uint16_t* a, const uint16_t* w, void* out, int64_t m
   if (!mzc::make_tmap_f16(&ta, a, static_cast<uint64_t>(m), static_cast<uint64_t>(k), 128) ||
       !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
     return MZC_ERR_CUDA;
-  KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, nullptr, static_cast<cudaStream_t>(stream)));
+  KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, nullptr, static_cast<cudaStream_t>(stream), a));
 }
 
 mzc_status mzc_k_swiglu_pack(const uint16_t* gate, const uint16_t* up, int64_t f, int64_t d,

@@ -27,8 +27,9 @@ def _rand_bf16(tid, shape, sigma=1.0):
 
 # ---- GEMM (tcgen05 / TMEM / TMA) -------------------------------------------
 
-GEMM_SHAPES = [(1, 64, 64), (7, 80, 72), (128, 256, 512), (130, 384, 320), (300, 1024, 2048),
-               (1000, 512, 256), (4224, 3072, 2048)]
+# m <= 4: the few-row GEMV path; larger m: the tcgen05 GEMM
+GEMM_SHAPES = [(1, 64, 64), (2, 1024, 2048), (4, 3072, 3072), (7, 80, 72), (128, 256, 512),
+               (130, 384, 320), (300, 1024, 2048), (1000, 512, 256), (4224, 3072, 2048)]
 
 
 def _act16(tid, shape):
@@ -50,7 +51,8 @@ def test_gemm_store_f16(mm, nn, kk):
     assert np.all(err <= 2.0 ** -10 * np.abs(ref) + 1e-5 * np.max(np.abs(ref)))
 
 
-@pytest.mark.parametrize("mm,nn,kk", [(5, 64, 128), (200, 256, 768), (4224, 2048, 2048)])
+@pytest.mark.parametrize("mm,nn,kk", [(1, 2048, 8192), (3, 3072, 1024), (5, 64, 128), (200, 256, 768),
+                                     (4224, 2048, 2048)])
 def test_gemm_residual_add(mm, nn, kk):
     torch = _torch()
     a = _act16(3, (mm, kk))
@@ -65,7 +67,8 @@ def test_gemm_residual_add(mm, nn, kk):
     assert np.max(np.abs(got[rows] - ref)) <= 1e-4 * np.max(np.abs(ref))
 
 
-@pytest.mark.parametrize("mm,f,kk", [(3, 128, 256), (260, 384, 512), (70, 704, 256),
+@pytest.mark.parametrize("mm,f,kk", [(1, 1024, 2048), (3, 128, 256), (4, 256, 512), (260, 384, 512),
+                                     (70, 704, 256),
                                      (4224, 1024, 2048)])
 def test_gemm_swiglu(mm, f, kk):
     torch = _torch()
