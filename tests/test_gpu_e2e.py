@@ -282,3 +282,23 @@ def test_q8_swap_overlapped_with_prompt_matches_sync_restore(tiny):
         outs.append(_logits(tiny, c, tiny["prm"]))
         m.mzc_destroy(c)
     assert np.array_equal(outs[0], outs[1])
+
+
+def test_decode_steps_match_oracle(tiny):
+    """Decode after the first token: single-token steps (the few-row GEMV
+    projections, one-row attention) match the oracle's forward of the same
+    row step after step, across a newly allocated KV block."""
+    sh, w = tiny["shape"], tiny["w"]
+    c = _new(tiny)
+    m.mzc_prefill(c, tiny["ctx"])
+    kv = oracle.KVState(sh, sh["max_ctx"])
+    lg_ref = oracle.prefill(sh, w, kv, tiny["ctx"], 0)
+    tok = int(np.argmax(lg_ref))
+    for step in range(20):
+        pos = len(tiny["ctx"]) + step
+        lg = _logits(tiny, c, np.array([tok], np.int32))
+        lg_ref = oracle.forward(sh, w, kv, [tok], [pos])
+        assert np.max(np.abs(lg - lg_ref)) < LOGIT_TOL, step
+        tok = int(np.argmax(lg_ref))
+    assert m.mzc_stats(c).context_tokens == len(tiny["ctx"]) + 20
+    m.mzc_destroy(c)
