@@ -203,12 +203,15 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
   const int R = n * group;
   const int r0 = (gridDim.y - 1 - blockIdx.y) * C::ROWS;
   const int split = blockIdx.z;
+  // Q tiles holding at least one real row: a trailing tile of padding rows
+  // (the last row tile of a short row set) gets no UMMAs and no softmax
+  const int nq = min(C::NQ, (R - r0 + C::BM - 1) / C::BM);
 
   if (tid == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
-      mbar_init(&kv_empty[s], C::NQ);  // every Q tile's P V done
+      mbar_init(&kv_empty[s], nq);  // every active Q tile's P V done
     }
     for (int t = 0; t < C::NQ; ++t) {
       mbar_init(&s_full[t], 1);
@@ -328,7 +331,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
   } else if (warp > C::PRODUCER_WARP) {
     // ---- UMMA issuers, one per Q tile t: S_t(j+1), then P_t V(j) ----
     const int t = warp - C::PRODUCER_WARP - 1;
-    if (lane == 0 && T > 0) {
+    if (lane == 0 && T > 0 && t < nq) {
       constexpr uint32_t id_s = idesc_attn<F16>(128, BN, false);
       constexpr uint32_t id_o = idesc_attn<F16>(128, HD, true);
       const uint32_t q_base = smem_u32(sQ + t * C::Q_BYTES);
@@ -381,7 +384,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     const uint32_t s_col = qt * BN, p_col = C::P_COL + qt * (BN / 2), o_col = C::O_COL + qt * HD;
     float m_ref = -INFINITY, l = 0.0f;
     bool ok = true;
-    for (int j = 0; j < T && ok; ++j) {
+    const int Tq = qt < nq ? T : 0;  // key tiles this Q tile processes
+    for (int j = 0; j < Tq && ok; ++j) {
       const uint32_t ph = j & 1;
       const int kb = k_begin + j * BN;
       ok = wait_bar(&s_full[qt], ph, status, abort_flag);
@@ -481,8 +485,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     }
     // ---- epilogue: O / l ----
     bool have_o = false;
-    if (ok && T > 0) {
-      ok = wait_bar(&p_free[qt], (T - 1) & 1, status, abort_flag);
+    if (ok && Tq > 0) {
+      ok = wait_bar(&p_free[qt], (Tq - 1) & 1, status, abort_flag);
       __syncwarp();
       have_o = __all_sync(0xffffffffu, ok);
       tc_fence_after();
