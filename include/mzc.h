@@ -406,6 +406,16 @@ mzc_status mzc_k_q8_decode(const void *in, int64_t n, int32_t hkv, int32_t hd,
                            const int32_t *phys, int64_t phys_begin, int32_t kv_dtype, void *pool,
                            void *stream);
 
+/* The kernels' pipeline waits are bounded: a wait that runs out records
+ * MZC_ERR_TIMEOUT in the kernel's status word and returns, and the CUDA
+ * context stays usable.  This entry point runs that wait on an mbarrier
+ * nothing arrives on (arrive == 0; or that it arrived on first, arrive != 0)
+ * with a limit of limit_cycles SM clocks; *completed (device int32) is 1 if
+ * the phase completed, 0 if the wait ran out; status (device int32) is set to
+ * MZC_ERR_TIMEOUT when it ran out. */
+mzc_status mzc_k_wait_probe(int32_t arrive, int64_t limit_cycles, int32_t *status,
+                            int32_t *completed, void *stream);
+
 /* logits fp32 [vocab] = RMSNorm(x_row) * g  W^T, x_row fp32 [d], W bf16 [vocab][d]. */
 mzc_status mzc_k_lm_head(const float *x_row, const float *g, int32_t d, float eps,
                          const uint16_t *w, int64_t vocab, float *logits, void *stream);

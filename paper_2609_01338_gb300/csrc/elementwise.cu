@@ -312,6 +312,18 @@ __global__ void poison_blocks_kernel(uint4* __restrict__ pool, const int32_t* __
   for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = v;
 }
 
+// A wait that runs out: one thread waits on an mbarrier that nothing arrives
+// on (or, with arrive != 0, that it arrived on first) through the same bounded
+// wait as every kernel's pipeline waits, with a caller-chosen limit.
+__global__ void wait_probe_kernel(int32_t arrive, int64_t limit_cycles, int32_t* status,
+                                  int32_t* completed) {
+  __shared__ uint64_t bar;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  if (arrive) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&bar)) : "memory");
+  *completed = mbar_wait(&bar, 0, status, limit_cycles) ? 1 : 0;
+}
+
 }  // namespace
 
 cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
@@ -354,6 +366,12 @@ cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float 
   const int grid = num_sms * 4;
   lm_head_kernel<<<grid, 256, static_cast<size_t>(d) * sizeof(float), st>>>(x_row, g, d, eps, w,
                                                                             vocab, logits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_probe(int32_t arrive, int64_t limit_cycles, int32_t* status,
+                              int32_t* completed, cudaStream_t st) {
+  wait_probe_kernel<<<1, 1, 0, st>>>(arrive, limit_cycles, status, completed);
   return cudaGetLastError();
 }
 

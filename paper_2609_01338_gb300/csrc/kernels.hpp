@@ -49,6 +49,9 @@ cudaError_t launch_q8_decode(const void* in, int64_t n_blocks, int64_t block_ele
                              const int32_t* phys, int64_t phys_begin, int32_t kv_dtype, void* pool,
                              cudaStream_t st);
 
+cudaError_t launch_wait_probe(int32_t arrive, int64_t limit_cycles, int32_t* status,
+                              int32_t* completed, cudaStream_t st);
+
 cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
                          int64_t vocab, float* x, int32_t* status, cudaStream_t st);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,

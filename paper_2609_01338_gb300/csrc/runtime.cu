@@ -1311,6 +1311,12 @@ mzc_status mzc_k_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_
   return MZC_OK;
 }
 
+mzc_status mzc_k_wait_probe(int32_t arrive, int64_t limit_cycles, int32_t* status, int32_t* completed,
+                            void* stream) {
+  if (!status || !completed || limit_cycles <= 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_wait_probe(arrive, limit_cycles, status, completed, static_cast<cudaStream_t>(stream)));
+}
+
 int64_t mzc_q8_block_bytes(int32_t hkv, int32_t hd) {
   if (hkv <= 0 || hd <= 0 || hd % 64 != 0) return 0;
   return mzc::q8_block_bytes(2LL * hkv * 16 * hd);

@@ -123,6 +123,7 @@ _SIGS = {
                                 c_i32, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
     "mzc_plan_split_ctx": [c_vp, c_i64, c_i64, c_vp],
+    "mzc_k_wait_probe": [c_i32, c_i64, c_vp, c_vp, c_vp],
     "mzc_k_q8_encode": [c_vp, c_vp, c_i64, c_i32, c_i32, c_vp, c_vp],
     "mzc_k_q8_decode": [c_vp, c_i64, c_i32, c_i32, c_vp, c_i64, c_i32, c_vp, c_vp],
     "mzc_k_embed": [c_vp, c_i64, c_vp, c_i32, c_i64, c_vp, c_vp, c_vp],
@@ -437,3 +438,7 @@ def mzc_k_q8_encode(pool, phys, n, hkv, hd, out, stream=None):
 def mzc_k_q8_decode(inp, n, hkv, hd, phys, phys_begin, kv_dtype, pool, stream=None):
     return _call("mzc_k_q8_decode", _ptr(inp), n, hkv, hd, _ptr(phys), phys_begin, kv_dtype,
                  _ptr(pool), stream)
+
+
+def mzc_k_wait_probe(arrive, limit_cycles, status, completed, stream=None):
+    return _call("mzc_k_wait_probe", arrive, limit_cycles, _ptr(status), _ptr(completed), stream)

@@ -292,3 +292,42 @@ def test_attention_split_kv_long_context(hq, hkv, hd, kvd):
     assert rel_err(got, ref) < 1e-2
     got2, ref2, _ = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=3, use_scratch=False)
     assert rel_err(got2, ref2) < 1e-2
+
+
+def test_bounded_wait_runs_out_and_context_stays_usable():
+    """A pipeline wait that nothing completes runs out after its limit (about
+    half a second here), records MZC_ERR_TIMEOUT, and the next kernels run."""
+    torch = _torch()
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    done = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    m.mzc_k_wait_probe(0, 1_000_000_000, status, done)
+    torch.cuda.synchronize()
+    assert int(done.item()) == 0 and int(status.item()) == m.MZC_ERR_TIMEOUT
+    status.zero_()
+    m.mzc_k_wait_probe(1, 1_000_000_000, status, done)
+    torch.cuda.synchronize()
+    assert int(done.item()) == 1 and int(status.item()) == 0
+    # the context is usable: a GEMM right after is still correct
+    test_gemm_store_f16(128, 256, 512)
+
+
+@pytest.mark.parametrize("bad", [-3, 10_000])
+def test_attention_flags_a_block_table_entry_outside_the_pool(bad):
+    """A block-table entry outside the pool is a device error: the kernel
+    records MZC_ERR_DEVICE and reads an in-pool block instead (no stray
+    address)."""
+    torch = _torch()
+    hq, hkv, hd, ctx = 8, 2, 64, 200
+    n_logical = (ctx + 15) // 16
+    pool_blocks = n_logical + 3
+    table = np.arange(n_logical, dtype=np.int32)
+    table[5] = bad
+    pool = torch.zeros((pool_blocks, 2, hkv, 16, hd), dtype=torch.int16, device="cuda")
+    q = torch.zeros((4, hq, hd), dtype=torch.int16, device="cuda")
+    pos = np.array([150, 160, 170, 199], np.int32)
+    out = torch.zeros_like(q)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    m.mzc_k_attention(q, i32_dev(pos), 4, hq, hkv, hd, i32_dev(table), n_logical, pool, pool_blocks,
+                      1, out, ctx, None, 0, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == m.MZC_ERR_DEVICE
