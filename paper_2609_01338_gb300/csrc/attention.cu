@@ -38,6 +38,7 @@
 #include <climits>
 #include <cmath>
 #include <mutex>
+#include <type_traits>
 
 #include "kernels.hpp"
 #include "ptx.cuh"
@@ -535,6 +536,9 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
 }
 
 // out[row] = sum_s 2^(lse_s - lse_max) o_s / sum_s 2^(lse_s - lse_max); one warp per row.
+// Lane s holds split s's log-sum-exp and weight (n_splits <= 64: two per lane),
+// and the partial rows are read eight splits at a time, so the loads of the
+// splits overlap instead of queueing one after another.
 template <int HD>
 __global__ void attn_combine_kernel(const float* __restrict__ part_o,
                                     const float* __restrict__ part_lse, int64_t rows, int n_splits,
@@ -542,21 +546,45 @@ __global__ void attn_combine_kernel(const float* __restrict__ part_o,
   const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
-  float mx = -INFINITY;
-  for (int s = 0; s < n_splits; ++s) mx = fmaxf(mx, part_lse[s * rows + row]);
+  const float l0 = lane < n_splits ? part_lse[lane * rows + row] : -INFINITY;
+  const float l1 = lane + 32 < n_splits ? part_lse[(lane + 32) * rows + row] : -INFINITY;
+  float mx = fmaxf(l0, l1);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  const float w0 = (l0 == -INFINITY) ? 0.0f : exp2f(l0 - mx);  // mx is finite when any l is
+  const float w1 = (l1 == -INFINITY) ? 0.0f : exp2f(l1 - mx);
+  float wsum = w0 + w1;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, off);
   constexpr int PER = HD / 32;
+  using Vec = typename std::conditional<PER == 4, float4, float2>::type;
   float acc[PER];
 #pragma unroll
   for (int j = 0; j < PER; ++j) acc[j] = 0.0f;
-  float wsum = 0.0f;
-  for (int s = 0; s < n_splits; ++s) {
-    const float l = part_lse[s * rows + row];
-    if (l == -INFINITY) continue;
-    const float w = exp2f(l - mx);
-    wsum += w;
-    const float* src = part_o + (s * rows + row) * HD + lane * PER;
+  // eight splits' rows are loaded before any is used, so their loads overlap;
+  // an empty split has weight 0 and rows of zeros
+  for (int s0 = 0; s0 < n_splits; s0 += 8) {
+    Vec v[8];
+    float w[8];
 #pragma unroll
-    for (int j = 0; j < PER; ++j) acc[j] += w * src[j];
+    for (int j = 0; j < 8; ++j) {
+      const int s = s0 + j;
+      const bool in = s < n_splits;  // uniform over the warp
+      w[j] = in ? __shfl_sync(0xffffffffu, s < 32 ? w0 : w1, s & 31) : 0.0f;
+      if (in) {
+        v[j] = *reinterpret_cast<const Vec*>(part_o + (s * rows + row) * HD + lane * PER);
+      } else {
+        float* z = reinterpret_cast<float*>(&v[j]);
+#pragma unroll
+        for (int e = 0; e < PER; ++e) z[e] = 0.0f;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float* f = reinterpret_cast<const float*>(&v[j]);
+#pragma unroll
+      for (int e = 0; e < PER; ++e) acc[e] = fmaf(w[j], f[e], acc[e]);
+    }
   }
   const float inv = wsum > 0.0f ? 1.0f / wsum : 0.0f;
   uint16_t* dst = out + row * HD + lane * PER;
@@ -640,6 +668,10 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
 
 void attention_split(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys, int num_sms,
                      int* n_splits, int* keys_per_split) {
+  if (attention_decode_applies(n, hq, hkv, hd)) {
+    attention_decode_split(hkv, max_keys, num_sms, n_splits, keys_per_split);
+    return;
+  }
   const int rows_per_cta = hd == 64 ? AttnCfg<64>::ROWS : AttnCfg<128>::ROWS;
   const int slots = num_sms * (hd == 64 ? AttnCfg<64>::CTAS_PER_SM : AttnCfg<128>::CTAS_PER_SM);
   const int64_t ctas = ((n * (hq / hkv) + rows_per_cta - 1) / rows_per_cta) * hkv;
@@ -680,13 +712,26 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   if (n <= 0) return cudaSuccess;
   int s = 1, per = 0;
   attention_split(n, hq, hkv, hd, max_keys, num_sms, &s, &per);
-  if (s > 1 && (scratch == nullptr || scratch_bytes < attention_scratch_bytes(n, hq, hd, s))) {
+  // the combine reads the partials as 8- or 16-byte vectors
+  if (s > 1 && (scratch == nullptr || scratch_bytes < attention_scratch_bytes(n, hq, hd, s) ||
+                reinterpret_cast<uintptr_t>(scratch) % 16 != 0)) {
     s = 1;
-    per = static_cast<int>((max_keys + 127) / 128 * 128);
+    per = static_cast<int>((max_keys + 127) / 128 * 128);  // whole 16-token blocks too
   }
   float* part_o = static_cast<float*>(scratch);
   float* part_lse = s > 1 ? part_o + static_cast<int64_t>(s) * n * hq * hd : nullptr;
   (void)kv_dtype;  // the pool is fp16-encoded for both KV types: q, K, P, V are fp16
+  if (attention_decode_applies(n, hq, hkv, hd)) {
+    cudaError_t e = launch_attention_decode(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks, out,
+                                            part_o, part_lse, s, per, status, st);
+    if (e != cudaSuccess || s == 1) return e;
+    const int64_t rows = n * hq;
+    if (hd == 64)
+      attn_combine_kernel<64><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(part_o, part_lse, rows, s, out);
+    else
+      attn_combine_kernel<128><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(part_o, part_lse, rows, s, out);
+    return cudaGetLastError();
+  }
   if (hd == 64)
     return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
                                part_o, part_lse, s, per, status, st);

@@ -66,6 +66,19 @@ cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_
 void attention_split(int64_t n, int32_t hq, int32_t hkv, int32_t hd, int64_t max_keys, int num_sms,
                      int* n_splits, int* keys_per_split);
 int64_t attention_scratch_bytes(int64_t n, int32_t hq, int32_t hd, int n_splits);
+
+// Decode attention (attention_decode.cu): at most kAttnDecodeMaxRows query rows
+// per KV head (n tokens x hq/hkv heads; one decode token of a model with up to
+// 4 query heads per KV head) take a CUDA-core kernel bound by the K/V read
+// instead of the 128-row tensor tiles; same arguments, split-KV partials and
+// combine as launch_attention, which dispatches to it.
+constexpr int kAttnDecodeMaxRows = 4;
+bool attention_decode_applies(int64_t n, int32_t hq, int32_t hkv, int32_t hd);
+void attention_decode_split(int32_t hkv, int64_t max_keys, int num_sms, int* n_splits, int* keys_per_split);
+cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
+                                    int32_t hd, const int32_t* table, int64_t n_logical, const void* pool,
+                                    int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
+                                    int n_splits, int keys_per_split, int32_t* status, cudaStream_t st);
 cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
                              int32_t hkv, int32_t hd, const int32_t* table, int64_t n_logical,
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,

@@ -294,6 +294,36 @@ def test_attention_split_kv_long_context(hq, hkv, hd, kvd):
     assert rel_err(got2, ref2) < 1e-2
 
 
+@pytest.mark.parametrize("hq,hkv,hd,kvd,n,ctx", [
+    (32, 8, 64, 1, 1, 8197),     # 1B decode token: 4 rows per KV head, split-KV, ragged end
+    (32, 8, 64, 1, 1, 70_000),   # more than 32 blocks per warp pair and split
+    (24, 8, 128, 0, 1, 32768),   # 3B decode token at the 3B context
+    (24, 8, 128, 0, 1, 777),     # ragged last block
+    (4, 2, 64, 0, 2, 530),       # tiny config, two tokens: 4 rows per KV head
+    (8, 8, 128, 1, 3, 100),      # no GQA; fewer blocks than warp pairs
+    (8, 8, 64, 0, 4, 16),        # a single block
+])
+def test_attention_decode_rows(hq, hkv, hd, kvd, n, ctx):
+    """At most 4 query rows per KV head take the decode kernel; with the
+    split-KV scratch and without it (one split)."""
+    pos = np.arange(ctx - n, ctx).astype(np.int32)
+    got, ref, sb = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=n + hd)
+    assert rel_err(got, ref) < 1e-2
+    assert np.mean(np.abs(got - ref)) < 2e-3 * np.max(np.abs(ref))
+    got2, ref2, _ = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=n + hd, use_scratch=False)
+    assert rel_err(got2, ref2) < 1e-2
+
+
+def test_attention_decode_rows_at_scattered_positions():
+    """Rows of one call at far-apart positions each see only their own causal
+    prefix (a row at position 0 attends to one key)."""
+    pos = np.array([0, 17, 2500, 4098], np.int32)
+    got, ref, _ = _attention_case(8, 8, 128, 1, 4099, pos, seed=7)
+    assert rel_err(got, ref) < 1e-2
+    # the row at position 0 is exactly V of key 0 (one weight of 1)
+    assert np.max(np.abs(got[0] - ref[0])) <= 2.0 ** -10 * np.max(np.abs(ref[0])) + 1e-6
+
+
 def test_bounded_wait_runs_out_and_context_stays_usable():
     """A pipeline wait that nothing completes runs out after its limit (about
     half a second here), records MZC_ERR_TIMEOUT, and the next kernels run."""
@@ -312,7 +342,8 @@ def test_bounded_wait_runs_out_and_context_stays_usable():
 
 
 @pytest.mark.parametrize("bad", [-3, 10_000])
-def test_attention_flags_a_block_table_entry_outside_the_pool(bad):
+@pytest.mark.parametrize("n", [4, 1])  # 16 rows per KV head (tensor-core kernel), 4 (decode kernel)
+def test_attention_flags_a_block_table_entry_outside_the_pool(bad, n):
     """A block-table entry outside the pool is a device error: the kernel
     records MZC_ERR_DEVICE and reads an in-pool block instead (no stray
     address)."""
@@ -323,11 +354,11 @@ def test_attention_flags_a_block_table_entry_outside_the_pool(bad):
     table = np.arange(n_logical, dtype=np.int32)
     table[5] = bad
     pool = torch.zeros((pool_blocks, 2, hkv, 16, hd), dtype=torch.int16, device="cuda")
-    q = torch.zeros((4, hq, hd), dtype=torch.int16, device="cuda")
-    pos = np.array([150, 160, 170, 199], np.int32)
+    q = torch.zeros((n, hq, hd), dtype=torch.int16, device="cuda")
+    pos = np.array([150, 160, 170, 199], np.int32)[-n:]
     out = torch.zeros_like(q)
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
-    m.mzc_k_attention(q, i32_dev(pos), 4, hq, hkv, hd, i32_dev(table), n_logical, pool, pool_blocks,
+    m.mzc_k_attention(q, i32_dev(pos), n, hq, hkv, hd, i32_dev(table), n_logical, pool, pool_blocks,
                       1, out, ctx, None, 0, status)
     torch.cuda.synchronize()
     assert int(status.item()) == m.MZC_ERR_DEVICE
