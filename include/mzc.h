@@ -350,8 +350,13 @@ mzc_status mzc_k_rope_kv_write(const uint16_t *qkv, const int32_t *pos, int64_t 
  * (kv_dtype is accepted for symmetry and ignored); row i attends to
  * every position <= pos[i] through block_table; out fp16 [n][hq][hd].
  * max_keys: an upper bound of pos[i] + 1 (sizes the split of long key
- * ranges).  scratch: device buffer of mzc_k_attention_scratch_bytes() bytes
- * for the split-KV partials, or NULL to run without splitting. */
+ * ranges).  scratch: device buffer of mzc_k_attention_scratch_bytes() bytes,
+ * 16-byte aligned, for the split-KV partials, or NULL to run without
+ * splitting (an unaligned or short buffer also runs without splitting).
+ * The pool must be 16-byte aligned (MZC_ERR_INVALID otherwise).  Calls
+ * with at most 4 query rows per KV head (n * hq/hkv <= 4: a decode token)
+ * take a kernel bound by reading K/V once (bulk copies of each block's K
+ * and V rows); larger calls take the tensor-core kernel. */
 mzc_status mzc_k_attention(const uint16_t *q, const int32_t *pos, int64_t n, int32_t hq,
                            int32_t hkv, int32_t hd, const int32_t *block_table, int64_t n_logical,
                            const void *pool, int64_t pool_blocks, int32_t kv_dtype,

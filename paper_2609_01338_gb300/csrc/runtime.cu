@@ -1275,6 +1275,7 @@ mzc_status mzc_k_attention(const uint16_t* q, const int32_t* pos, int64_t n, int
                            void* stream) {
   if (!q || !pos || !block_table || !pool || !out || n < 0 || max_keys <= 0) return MZC_ERR_INVALID;
   if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) return MZC_ERR_INVALID;
+  if (reinterpret_cast<uintptr_t>(pool) % 16 != 0) return MZC_ERR_INVALID;  // TMA and bulk copies
   KCK(mzc::launch_attention(q, pos, n, hq, hkv, hd, block_table, n_logical, pool, pool_blocks,
                             kv_dtype, out, scratch, scratch_bytes, max_keys, sm_count(), status,
                             static_cast<cudaStream_t>(stream)));
@@ -1291,6 +1292,10 @@ mzc_status mzc_k_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_
   }
   if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) {
     g_create_error = "mzc_k_attention_noalloc: unsupported head shape";
+    return MZC_ERR_INVALID;
+  }
+  if (reinterpret_cast<uintptr_t>(pool) % 16 != 0) {
+    g_create_error = "mzc_k_attention_noalloc: pool not 16-byte aligned";
     return MZC_ERR_INVALID;
   }
   const int64_t need = mzc::attention_noalloc_need(n, hq, hkv, hd, max_keys, sm_count());

@@ -226,3 +226,12 @@ def test_hybrid_split_bruteforce_and_limits():
     # a link much faster than compute -> copy everything; much slower -> recompute everything
     assert m.mzc_plan_split(sh, _prof(1e6), 0, 4096, 16) == 0
     assert m.mzc_plan_split(sh, _prof(1e-3), 0, 4096, 16) == 4096
+
+
+def test_attention_rejects_an_unaligned_pool_before_any_launch():
+    """Both attention kernels copy pool rows with 16-byte-aligned TMA / bulk
+    copies: an unaligned pool is refused at the boundary (no GPU needed)."""
+    fake = 1 << 20  # never dereferenced: the call returns before any launch
+    for fn, extra in (("mzc_k_attention", (4096, None, 0)), ("mzc_k_attention_noalloc", (4096,))):
+        args = [fake, fake, 1, 32, 8, 64, fake, 4, fake + 8, 8, 1, fake, *extra, None, None]
+        assert M.status_of(fn, *args) == M.MZC_ERR_INVALID, fn
