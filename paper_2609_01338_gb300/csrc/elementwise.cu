@@ -107,46 +107,51 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restr
 }
 
 // The same RMSNorm, one warp per row with the row held in registers (read
-// once, reduced with shuffles, no block barrier): for d a multiple of 256 up to
-// 32 * 8 * kRowVecs.  Lane c owns the 8-float groups c, c + 32, ...
+// once, reduced with shuffles, no block barrier): for d = 256 * G, G <= 16.
+// Lane c owns the 8-float groups c, c + 32, ...  G is a template constant so
+// a row takes only the registers it needs (more warps per SM in flight).
 constexpr int kRowVecs = 16;  // 8-float groups per lane: d <= 4096
 
-__global__ void __launch_bounds__(256) rmsnorm_warp_kernel(const float* __restrict__ x,
+template <int G>
+__global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_warp_kernel(const float* __restrict__ x,
                                                            const float* __restrict__ g, int64_t n,
-                                                           int d, float eps,
-                                                           uint16_t* __restrict__ y) {
+                                                           float eps, uint16_t* __restrict__ y) {
+  constexpr int d = 256 * G;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (i >= n) return;
-  const int groups = d / 256;  // 8-float groups per lane
   const float4* xr = reinterpret_cast<const float4*>(x + i * d);
-  float4 a[kRowVecs], b[kRowVecs];
+  float4 a[G], b[G];
   float ss = 0.0f;
 #pragma unroll
-  for (int k = 0; k < kRowVecs; ++k) {
-    if (k < groups) {
-      const int c = k * 32 + lane;
-      a[k] = xr[2 * c];
-      b[k] = xr[2 * c + 1];
-      ss += a[k].x * a[k].x + a[k].y * a[k].y + a[k].z * a[k].z + a[k].w * a[k].w +
-            b[k].x * b[k].x + b[k].y * b[k].y + b[k].z * b[k].z + b[k].w * b[k].w;
-    }
+  for (int k = 0; k < G; ++k) {
+    const int c = k * 32 + lane;
+    a[k] = xr[2 * c];
+    b[k] = xr[2 * c + 1];
   }
+#pragma unroll
+  for (int k = 0; k < G; ++k)
+    ss += a[k].x * a[k].x + a[k].y * a[k].y + a[k].z * a[k].z + a[k].w * a[k].w +
+          b[k].x * b[k].x + b[k].y * b[k].y + b[k].z * b[k].z + b[k].w * b[k].w;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   const float r = rsqrtf(ss / static_cast<float>(d) + eps);
   const float4* gr = reinterpret_cast<const float4*>(g);
   uint4* yr = reinterpret_cast<uint4*>(y + i * d);
 #pragma unroll
-  for (int k = 0; k < kRowVecs; ++k) {
-    if (k < groups) {
-      const int c = k * 32 + lane;
-      const float4 ga = gr[2 * c], gb = gr[2 * c + 1];
-      float f[8] = {a[k].x * r * ga.x, a[k].y * r * ga.y, a[k].z * r * ga.z, a[k].w * r * ga.w,
-                    b[k].x * r * gb.x, b[k].y * r * gb.y, b[k].z * r * gb.z, b[k].w * r * gb.w};
-      yr[c] = pack8<true>(f);
-    }
+  for (int k = 0; k < G; ++k) {
+    const int c = k * 32 + lane;
+    const float4 ga = gr[2 * c], gb = gr[2 * c + 1];
+    float f[8] = {a[k].x * r * ga.x, a[k].y * r * ga.y, a[k].z * r * ga.z, a[k].w * r * ga.w,
+                  b[k].x * r * gb.x, b[k].y * r * gb.y, b[k].z * r * gb.z, b[k].w * r * gb.w};
+    yr[c] = pack8<true>(f);
   }
+}
+
+template <int G>
+void launch_rmsnorm_warp(const float* x, const float* g, int64_t n, float eps, uint16_t* y,
+                         cudaStream_t st) {
+  rmsnorm_warp_kernel<G><<<static_cast<unsigned>((n + 7) / 8), 256, 0, st>>>(x, g, n, eps, y);
 }
 
 // Rotary embedding (pairs (i, i + hd/2), angle pos * theta^(-2i/hd) from the
@@ -336,10 +341,32 @@ cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed
 cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
                            uint16_t* y, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  if (d % 256 == 0 && d / 256 <= kRowVecs)
-    rmsnorm_warp_kernel<<<static_cast<unsigned>((n + 7) / 8), 256, 0, st>>>(x, g, n, d, eps, y);
-  else
-    rmsnorm_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(x, g, d, eps, y);
+  switch (d % 256 == 0 ? d / 256 : 0) {
+#define MZC_RMS_CASE(G)                         \
+  case G:                                       \
+    launch_rmsnorm_warp<G>(x, g, n, eps, y, st); \
+    break;
+    MZC_RMS_CASE(1)
+    MZC_RMS_CASE(2)
+    MZC_RMS_CASE(3)
+    MZC_RMS_CASE(4)
+    MZC_RMS_CASE(5)
+    MZC_RMS_CASE(6)
+    MZC_RMS_CASE(7)
+    MZC_RMS_CASE(8)
+    MZC_RMS_CASE(9)
+    MZC_RMS_CASE(10)
+    MZC_RMS_CASE(11)
+    MZC_RMS_CASE(12)
+    MZC_RMS_CASE(13)
+    MZC_RMS_CASE(14)
+    MZC_RMS_CASE(15)
+    MZC_RMS_CASE(16)
+#undef MZC_RMS_CASE
+    default:
+      rmsnorm_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(x, g, d, eps, y);
+  }
+  static_assert(kRowVecs == 16, "warp kernel instances for d = 256 .. 4096");
   return cudaGetLastError();
 }
 
