@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmzc.so")
 
-CU_SOURCES = ["gemm.cu", "gemv.cu", "attention.cu", "attention_decode.cu", "attention_noalloc.cu", "elementwise.cu",
+CU_SOURCES = ["gemm.cu", "gemm_splitk.cu", "gemv.cu", "attention.cu", "attention_decode.cu", "attention_noalloc.cu", "elementwise.cu",
               "codec.cu", "runtime.cu"]
 CXX_SOURCES = ["state.cpp", "state_api.cpp"]
 HEADERS = ["ptx.cuh", "kernels.hpp", "state.hpp"]

@@ -404,6 +404,19 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
   if (m <= 0) return cudaSuccess;
   if (a_ptr && w.ptr && m <= kGemvMaxRows)
     return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, st);
+  if (m <= 256) {
+    // weight-streaming bound with few N tiles: split K over a cluster
+    static int sms = 0;
+    if (sms == 0) {
+      int dev = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (sms <= 0) sms = 1;
+    }
+    bool launched = false;
+    const cudaError_t e = launch_gemm_splitk(ta, w, out, m, n, k, epilogue, sms, status, st, &launched);
+    if (launched || e != cudaSuccess) return e;
+  }
   const uint32_t bn = gemm_box_n(m, n, epilogue);
   if (bn == 256) {
     switch (epilogue) {

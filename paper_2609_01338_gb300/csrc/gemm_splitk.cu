@@ -1,0 +1,389 @@
+// Projections of a few hundred rows (a short prompt), where the GEMM is bound
+// by streaming the weights: C[m][n] = A[m][k] W[n][k]^T with m <= 256.
+//
+// With 128 x BN tiles over N alone, an O or down projection (n = 3072) has
+// 24-48 tiles, so only that many SMs pull weight bytes, and at narrow BN the
+// shared activation tiles make up most of every SM's traffic.  Here the K
+// range is split as well, over the S CTAs of a thread-block cluster
+// (grid = S x N tiles of 128 columns):
+//   - CTA s of the cluster accumulates its k-blocks [s*nkb/S, (s+1)*nkb/S) of
+//     the 128-column tile for all (one or two) 128-row M tiles into TMEM, with
+//     the same TMA ring / single-thread tcgen05.mma / commit pipeline as the
+//     persistent GEMM;
+//   - the epilogue warps copy the fp32 partial to shared memory (the ring is
+//     free by then) and the cluster synchronises;
+//   - CTA s then sums rows [s*RS, (s+1)*RS) of the S partials, read through
+//     distributed shared memory in split order (the same sum on every run),
+//     applies the epilogue (fp16 store, fp32 residual add, SwiGLU) and writes
+//     the rows out; a second cluster barrier keeps every partial alive until
+//     all CTAs have read it.
+// Every thread of every CTA passes both cluster barriers exactly once (no
+// early exit on any path); the pipeline waits are bounded as elsewhere.
+#include <algorithm>
+#include <mutex>
+
+#include "kernels.hpp"
+#include "ptx.cuh"
+
+namespace mzc {
+
+namespace {
+
+constexpr int SBM = 128, SBN = 128, SBK = 64;
+
+template <int MT>
+struct SKCfg {
+  static constexpr int STAGES = MT == 1 ? 6 : 4;
+  static constexpr int A_BYTES = SBM * SBK * 2;  // one M tile's k-block
+  static constexpr int B_BYTES = SBN * SBK * 2;
+  static constexpr int STAGE_BYTES = MT * A_BYTES + B_BYTES;
+  static constexpr int RING = STAGES * STAGE_BYTES;
+  static constexpr int PART_BYTES = MT * SBM * SBN * 4;  // fp32 partial, reuses the ring
+  static constexpr int OFF_BAR = RING;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr uint32_t TMEM_COLS = MT * SBN;
+  static_assert(PART_BYTES <= RING, "the partial fits in the ring");
+  static_assert(2 * STAGES * 8 + 8 <= 256, "barriers");
+};
+
+__device__ __forceinline__ bool skwait(uint64_t* bar, uint32_t parity, int32_t* status, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      set_status(status, kStatusTimeout);
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// address of the same shared-memory location in cluster CTA `rank`
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float silu_s(float g) { return g / (1.0f + __expf(-g)); }
+
+__device__ __forceinline__ uint2 pack4_f16(float a, float b, float c, float d) {
+  return make_uint2(pack2<true>(a, b), pack2<true>(c, d));
+}
+
+// Partial layout: row r (0 .. MT*128) of 32 float4 chunks, chunk c stored at
+// c ^ (r & 7) so that eight lanes writing one chunk of eight rows hit eight
+// different bank groups.
+__device__ __forceinline__ uint32_t part_off(int r, int c) {
+  return static_cast<uint32_t>((r * 32 + (c ^ (r & 7))) * 16);
+}
+
+template <int MT, int EPI>
+__global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
+    const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw, void* __restrict__ out,
+    int m, int n, int k, int32_t* status) {
+  using C = SKCfg<MT>;
+  constexpr int STAGES = C::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* empty = full + STAGES;
+  uint64_t* acc_full = empty + STAGES;
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort;
+  volatile int* abort_flag = &s_abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = static_cast<int>(cluster_size()), s = static_cast<int>(cluster_rank());
+  const int nt = blockIdx.y;
+  const int nkb = (k + SBK - 1) / SBK;
+  const int kb0 = static_cast<int>(static_cast<int64_t>(s) * nkb / S);
+  const int kb1 = static_cast<int>(static_cast<int64_t>(s + 1) * nkb / S);
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tma);
+    tma_prefetch_desc(&tmw);
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    fence_barrier_init();
+    s_abort = 0;
+  }
+  if (warp == 1) tmem_alloc(&s_tmem, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer: the split's k-blocks, every M tile and the W tile ----
+      bool ok = true;
+      int it = 0;
+      for (int kb = kb0; ok && kb < kb1; ++kb, ++it) {
+        const int st = it % STAGES;
+        if (it >= STAGES && !skwait(&empty[st], ((it / STAGES) - 1) & 1, status, abort_flag)) {
+          ok = false;
+          break;
+        }
+        uint8_t* base = smem + st * C::STAGE_BYTES;
+        mbar_arrive_expect_tx(&full[st], C::STAGE_BYTES);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) tma_load_2d(base + mt * C::A_BYTES, &tma, &full[st], kb * SBK, mt * SBM);
+        tma_load_2d(base + MT * C::A_BYTES, &tmw, &full[st], kb * SBK, nt * SBN);
+      }
+      // every fill issued has landed before the ring is reused for the partial
+      for (int i = it - STAGES < 0 ? 0 : it - STAGES; i < it; ++i)
+        skwait(&full[i % STAGES], (i / STAGES) & 1, status, abort_flag);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- UMMA issuer: accumulator of M tile mt at TMEM columns mt*128 ----
+      constexpr uint32_t idesc = idesc_f16_f32(SBM, SBN);
+      bool ok = true;
+      int it = 0;
+      for (int kb = kb0; ok && kb < kb1; ++kb, ++it) {
+        const int st = it % STAGES;
+        if (!skwait(&full[st], (it / STAGES) & 1, status, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t base = smem_u32(smem + st * C::STAGE_BYTES);
+        const uint64_t bd = sdesc_k_sw128(base + MT * C::A_BYTES);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint64_t ad = sdesc_k_sw128(base + mt * C::A_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < SBK / 16; ++kk)
+            umma_f16(tmem + mt * SBN, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0 ? 1u : 0u);
+        }
+        umma_commit(&empty[st]);
+      }
+      umma_commit(acc_full);  // all of this thread's UMMAs (none for an empty split)
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue warps 2-5: TMEM accumulator -> shared-memory partial ----
+    const int q = warp & 3;  // TMEM lane quarter: rows q*32 .. q*32+31 of each M tile
+    bool ok = skwait(acc_full, 0, status, abort_flag);
+    __syncwarp();
+    ok = __all_sync(0xffffffffu, ok);
+    tc_fence_after();
+    const bool have = ok && kb1 > kb0;
+#pragma unroll 1
+    for (int mt = 0; mt < MT; ++mt) {
+      const int r = mt * SBM + q * 32 + lane;
+      const uint32_t trow = tmem + mt * SBN + (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < SBN; c += 32) {
+        float v[32];
+        if (have) {
+          tmem_ld32w(trow + c, v);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          *reinterpret_cast<float4*>(smem + part_off(r, c / 4 + u)) =
+              make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+      }
+    }
+    tc_fence_before();
+  }
+
+  // ---- every partial of the cluster is in shared memory ----
+  cluster_sync_all();
+
+  if (warp >= 2) {
+    // ---- rows [s*RS, (s+1)*RS) summed over the S partials in split order ----
+    const int rows = min(MT * SBM, m);
+    const int RS = (rows + S - 1) / S;
+    const int r_begin = s * RS, r_end = min(rows, r_begin + RS);
+    const int t = threadIdx.x - 64;  // 0 .. 127
+    const uint32_t part = smem_u32(smem);
+    constexpr int CH = EPI == EPI_SWIGLU_BF16 ? 16 : 32;  // float4 chunks handled per row
+    for (int idx = t; idx < (r_end - r_begin) * CH; idx += 128) {
+      const int r = r_begin + idx / CH, c = idx % CH;
+      // all S loads are issued before the sum, which then runs in split order
+      float4 v[8], u[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (j < S) {
+          v[j] = ld_cluster_f4(map_rank(part + part_off(r, c), j));
+          if constexpr (EPI == EPI_SWIGLU_BF16) u[j] = ld_cluster_f4(map_rank(part + part_off(r, c + 16), j));
+        }
+      }
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f), acc2 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (j < S) {
+          acc.x += v[j].x;
+          acc.y += v[j].y;
+          acc.z += v[j].z;
+          acc.w += v[j].w;
+          if constexpr (EPI == EPI_SWIGLU_BF16) {
+            acc2.x += u[j].x;
+            acc2.y += u[j].y;
+            acc2.z += u[j].z;
+            acc2.w += u[j].w;
+          }
+        }
+      }
+      if constexpr (EPI == EPI_STORE_BF16) {
+        const int col = nt * SBN + c * 4;
+        if (col < n)
+          *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * n + col) =
+              pack4_f16(acc.x, acc.y, acc.z, acc.w);
+      } else if constexpr (EPI == EPI_ADD_F32) {
+        const int col = nt * SBN + c * 4;
+        if (col < n) {
+          float4* o = reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<int64_t>(r) * n + col);
+          float4 x = *o;
+          x.x += acc.x;
+          x.y += acc.y;
+          x.z += acc.z;
+          x.w += acc.w;
+          *o = x;
+        }
+      } else {
+        // gate columns 0..63 of the tile pair with up columns 64..127
+        const int col = nt * (SBN / 2) + c * 4;
+        if (col < n / 2)
+          *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * (n / 2) + col) =
+              pack4_f16(silu_s(acc.x) * acc2.x, silu_s(acc.y) * acc2.y, silu_s(acc.z) * acc2.z,
+                        silu_s(acc.w) * acc2.w);
+      }
+    }
+  }
+
+  // ---- no CTA leaves while another may still read its partial ----
+  __syncwarp();
+  cluster_sync_all();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int MT, int EPI>
+cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out, int64_t m, int64_t n, int64_t k,
+                      int S, int32_t* status, cudaStream_t st) {
+  using C = SKCfg<MT>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(gemm_splitk_kernel<MT, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    C::SMEM);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  const int num_n = static_cast<int>((n + SBN - 1) / SBN);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(S), static_cast<unsigned>(num_n), 1);
+  cfg.blockDim = dim3(192, 1, 1);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<MT, EPI>, ta, tw128, out, static_cast<int>(m),
+                            static_cast<int>(n), static_cast<int>(k), status);
+}
+
+// The largest cluster size S <= 8 whose S x num_n CTAs are all resident at
+// once (one wave), from the occupancy query for this kernel; 1 if none.
+template <int MT, int EPI>
+int pick_splits(int num_n, int num_sms) {
+  using C = SKCfg<MT>;
+  static std::once_flag once;
+  static int max_clusters[9] = {};
+  std::call_once(once, [] {
+    if (cudaFuncSetAttribute(gemm_splitk_kernel<MT, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+        cudaSuccess)
+      return;
+    for (int sz = 2; sz <= 8; ++sz) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(static_cast<unsigned>(sz), 1, 1);
+      cfg.blockDim = dim3(192, 1, 1);
+      cfg.dynamicSmemBytes = C::SMEM;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = static_cast<unsigned>(sz);
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int count = 0;
+      if (cudaOccupancyMaxActiveClusters(&count, gemm_splitk_kernel<MT, EPI>, &cfg) == cudaSuccess)
+        max_clusters[sz] = count;
+    }
+    cudaGetLastError();  // a refused query leaves no error behind
+  });
+  for (int sz = std::min(8, num_sms / std::max(1, num_n)); sz >= 2; --sz)
+    if (max_clusters[sz] >= num_n) return sz;
+  return 1;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m, int64_t n,
+                               int64_t k, int epilogue, int num_sms, int32_t* status, cudaStream_t st,
+                               bool* launched) {
+  *launched = false;
+  if (m <= 0 || m > 2 * SBM || n % SBN != 0 || k % 8 != 0) return cudaSuccess;
+  const int num_n = static_cast<int>(n / SBN);
+  const bool two = m > SBM;
+#define MZC_SK(MTV, EPIV)                                                                   \
+  {                                                                                        \
+    const int S = pick_splits<MTV, EPIV>(num_n, num_sms);                                  \
+    if (S < 2) return cudaSuccess;                                                         \
+    *launched = true;                                                                      \
+    return launch_sk<MTV, EPIV>(ta, w.box128, out, m, n, k, S, status, st);                \
+  }
+  switch (epilogue) {
+    case EPI_STORE_BF16:
+      if (two) MZC_SK(2, EPI_STORE_BF16) else MZC_SK(1, EPI_STORE_BF16)
+    case EPI_ADD_F32:
+      if (two) MZC_SK(2, EPI_ADD_F32) else MZC_SK(1, EPI_ADD_F32)
+    case EPI_SWIGLU_BF16:
+      if (two) MZC_SK(2, EPI_SWIGLU_BF16) else MZC_SK(1, EPI_SWIGLU_BF16)
+    default:
+      return cudaErrorInvalidValue;
+  }
+#undef MZC_SK
+}
+
+}  // namespace mzc

@@ -25,6 +25,12 @@ struct GemmWeight {
   CUtensorMap box64, box128, box256;
   const uint16_t* ptr = nullptr;  // W itself, for the few-row GEMV
 };
+// Split-K GEMM over a thread-block cluster for m <= 256 (gemm_splitk.cu):
+// launched (and *launched set) when n is a multiple of 128 and a cluster size
+// of at least 2 fits the grid in one wave; otherwise nothing is launched.
+cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const struct GemmWeight& w, void* out, int64_t m,
+                               int64_t n, int64_t k, int epilogue, int num_sms, int32_t* status,
+                               cudaStream_t st, bool* launched);
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 
 // C = A W^T; A map [>= m][k] with box rows 128.  The W map used is the one

@@ -87,6 +87,42 @@ def test_gemm_swiglu(mm, f, kk):
     assert np.all(err <= 2.0 ** -9 * np.abs(ref) + 2e-5 * np.max(np.abs(ref)))
 
 
+@pytest.mark.parametrize("mm,nn,kk,epi", [(128, 3072, 8192, 1), (128, 5120, 3072, 0), (256, 3072, 3072, 1),
+                                         (200, 2048, 4096, 2), (37, 1024, 1000, 0), (9, 128, 64, 1)])
+def test_gemm_split_k_over_a_cluster(mm, nn, kk, epi):
+    """m <= 256 with few 128-column tiles: the K range is split over the CTAs
+    of a cluster and the partials summed in split order through distributed
+    shared memory; the result matches the oracle and repeats bit for bit."""
+    torch = _torch()
+    a = _act16(11, (mm, kk))
+    wb, wh = bf16_weights_exact_in_f16(_rand_bf16(12, (nn, kk), sigma=0.05))
+    ncol = nn // 2 if epi == 2 else nn
+    x0 = np.random.default_rng(1).standard_normal((mm, ncol)).astype(np.float32)
+    if epi == 2:
+        w = m.mzc_k_swiglu_pack(wh[: nn // 2], wh[nn // 2:])
+        wg, wu = wb[: nn // 2], wb[nn // 2:]
+    else:
+        w = wh
+    outs = []
+    for _ in range(2):
+        out = f32_dev(x0) if epi == 1 else torch.zeros((mm, ncol), dtype=torch.int16, device="cuda")
+        m.mzc_k_gemm(bf16_dev(a), bf16_dev(w), out, mm, nn, kk, epi)
+        torch.cuda.synchronize()
+        outs.append(out.cpu().numpy() if epi == 1 else f16_to_f32(to_np_u16(out)))
+    assert np.array_equal(outs[0], outs[1])
+    got = outs[0]
+    af = f16_to_f32(a)
+    if epi == 0:
+        ref = oracle.linear(af, wb)
+        assert np.all(np.abs(got - ref) <= 2.0 ** -10 * np.abs(ref) + 1e-5 * np.max(np.abs(ref)))
+    elif epi == 1:
+        ref = x0 + oracle.linear(af, wb)
+        assert np.max(np.abs(got - ref)) <= 1e-4 * np.max(np.abs(ref))
+    else:
+        ref = oracle.swiglu(oracle.linear(af, wg), oracle.linear(af, wu))
+        assert np.all(np.abs(got - ref) <= 2.0 ** -9 * np.abs(ref) + 2e-5 * np.max(np.abs(ref)))
+
+
 @pytest.mark.parametrize("epi", [0, 1, 2])
 @pytest.mark.parametrize("mm,nn", [(5, 128), (300, 384), (1000, 2048)])
 def test_gemm_writes_only_its_rows(epi, mm, nn):
