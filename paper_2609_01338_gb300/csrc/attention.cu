@@ -175,6 +175,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     int64_t pool_blocks,
     uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
     int keys_per_split, int n_splits, float scale_log2, int32_t* status) {
+  pdl_enter();
   using C = AttnCfg<HD>;
   constexpr int BN = C::BN;
   extern __shared__ uint8_t smem_raw[];
@@ -543,6 +544,7 @@ template <int HD>
 __global__ void attn_combine_kernel(const float* __restrict__ part_o,
                                     const float* __restrict__ part_lse, int64_t rows, int n_splits,
                                     uint16_t* __restrict__ out) {
+  pdl_enter();
   const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -653,13 +655,13 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
   dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(row_tiles), static_cast<unsigned>(n_splits));
   const float scale_log2 =
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
-  attn_tc_kernel<HD, F16><<<grid, C::THREADS, C::SMEM, st>>>(
+  launch_k(attn_tc_kernel<HD, F16>, dim3(grid), dim3(C::THREADS), C::SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, run_map, blk_map, pool_blocks, out, part_o,
       part_lse, keys_per_split, n_splits, scale_log2, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || n_splits == 1) return e;
   const int64_t rows = n * hq;
-  attn_combine_kernel<HD><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(
+  launch_k(attn_combine_kernel<HD>, dim3(static_cast<unsigned>((rows + 7) / 8)), dim3(256), 0, st,
       part_o, part_lse, rows, n_splits, out);
   return cudaGetLastError();
 }
@@ -727,9 +729,9 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
     if (e != cudaSuccess || s == 1) return e;
     const int64_t rows = n * hq;
     if (hd == 64)
-      attn_combine_kernel<64><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(part_o, part_lse, rows, s, out);
+      launch_k(attn_combine_kernel<64>, dim3(static_cast<unsigned>((rows + 7) / 8)), dim3(256), 0, st, part_o, part_lse, rows, s, out);
     else
-      attn_combine_kernel<128><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(part_o, part_lse, rows, s, out);
+      launch_k(attn_combine_kernel<128>, dim3(static_cast<unsigned>((rows + 7) / 8)), dim3(256), 0, st, part_o, part_lse, rows, s, out);
     return cudaGetLastError();
   }
   if (hd == 64)

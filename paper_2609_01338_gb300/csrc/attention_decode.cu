@@ -113,6 +113,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     int64_t pool_blocks, uint16_t* __restrict__ out, float* __restrict__ part_o,
     float* __restrict__ part_lse, int blocks_per_split, int n_splits, float scale_log2,
     int32_t* status) {
+  pdl_enter();
   using C = DecCfg<HD>;
   constexpr int DPL = C::DPL;
   extern __shared__ uint8_t smem_raw[];
@@ -382,7 +383,7 @@ cudaError_t launch_dec(const uint16_t* q, const int32_t* pos, int64_t n, int32_t
   if (attr_err != cudaSuccess) return attr_err;
   const float scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
   dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(n_splits));
-  attn_decode_kernel<HD, R><<<grid, kDecThreads, SMEM, st>>>(
+  launch_k(attn_decode_kernel<HD, R>, dim3(grid), dim3(kDecThreads), SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, static_cast<const uint16_t*>(pool), pool_blocks,
       out, part_o, part_lse, blocks_per_split, n_splits, scale_log2, status);
   return cudaGetLastError();

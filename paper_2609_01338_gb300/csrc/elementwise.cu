@@ -5,10 +5,20 @@
 #include <algorithm>
 #include <cstdio>
 
+#include <cstdlib>
+
 #include "kernels.hpp"
 #include "ptx.cuh"
 
 namespace mzc {
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = std::getenv("MZC_PDL");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
 
 namespace {
 
@@ -67,6 +77,7 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 // x[i][:] = embed[tokens[i]][:] widened to fp32; one CTA per row.
 __global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t* __restrict__ emb,
                              int d, int64_t vocab, float* __restrict__ x, int32_t* status) {
+  pdl_enter();
   const int64_t i = blockIdx.x;
   const int32_t t = tokens[i];
   if (t < 0 || t >= vocab) {
@@ -86,6 +97,7 @@ __global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t*
 // y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, fp16 out; one CTA per row.
 __global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g, int d,
                                float eps, uint16_t* __restrict__ y) {
+  pdl_enter();
   __shared__ float red[32];
   const int64_t i = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + i * d);
@@ -116,6 +128,7 @@ template <int G>
 __global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_warp_kernel(const float* __restrict__ x,
                                                            const float* __restrict__ g, int64_t n,
                                                            float eps, uint16_t* __restrict__ y) {
+  pdl_enter();
   constexpr int d = 256 * G;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -151,7 +164,7 @@ __global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_w
 template <int G>
 void launch_rmsnorm_warp(const float* x, const float* g, int64_t n, float eps, uint16_t* y,
                          cudaStream_t st) {
-  rmsnorm_warp_kernel<G><<<static_cast<unsigned>((n + 7) / 8), 256, 0, st>>>(x, g, n, eps, y);
+  launch_k(rmsnorm_warp_kernel<G>, dim3(static_cast<unsigned>((n + 7) / 8)), dim3(256), 0, st, x, g, n, eps, y);
 }
 
 // Rotary embedding (pairs (i, i + hd/2), angle pos * theta^(-2i/hd) from the
@@ -166,6 +179,7 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
                                int64_t n_logical, uint16_t* __restrict__ pool,
                                int64_t pool_blocks, uint16_t* __restrict__ q_out,
                                int32_t* status) {
+  pdl_enter();
   const int64_t i = blockIdx.x;
   const int p = pos[i];
   const int half = hd / 2;
@@ -245,6 +259,7 @@ __global__ void __launch_bounds__(256) lm_head_kernel(const float* __restrict__ 
                                                       const float* __restrict__ g, int d,
                                                       float eps, const uint16_t* __restrict__ w,
                                                       int64_t vocab, float* __restrict__ logits) {
+  pdl_enter();
   extern __shared__ float sh[];
   __shared__ float red[32];
   float ss = 0.0f;
@@ -296,6 +311,7 @@ __global__ void __launch_bounds__(256) lm_head_kernel(const float* __restrict__ 
 // dst[i] = src[i] for n 16-byte words; src may be mapped pinned host memory,
 // read over the host link by the SMs (no copy engine involved).
 __global__ void copy16_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst, int64_t n) {
+  pdl_enter();
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
     dst[i] = src[i];
@@ -334,7 +350,7 @@ __global__ void wait_probe_kernel(int32_t arrive, int64_t limit_cycles, int32_t*
 cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
                          int64_t vocab, float* x, int32_t* status, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  embed_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(tokens, embed, d, vocab, x, status);
+  launch_k(embed_kernel, dim3(static_cast<unsigned>(n)), dim3(256), 0, st, tokens, embed, d, vocab, x, status);
   return cudaGetLastError();
 }
 
@@ -364,7 +380,7 @@ cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d,
     MZC_RMS_CASE(16)
 #undef MZC_RMS_CASE
     default:
-      rmsnorm_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(x, g, d, eps, y);
+      launch_k(rmsnorm_kernel, dim3(static_cast<unsigned>(n)), dim3(256), 0, st, x, g, d, eps, y);
   }
   static_assert(kRowVecs == 16, "warp kernel instances for d = 256 .. 4096");
   return cudaGetLastError();
@@ -377,11 +393,11 @@ cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_
                                  int32_t* status, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   if (kv_dtype == 1)
-    rope_kv_kernel<true><<<static_cast<unsigned>(n), 128, 0, st>>>(
+    launch_k(rope_kv_kernel<true>, dim3(static_cast<unsigned>(n)), dim3(128), 0, st,
         qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
         pool_blocks, q_out, status);
   else
-    rope_kv_kernel<false><<<static_cast<unsigned>(n), 128, 0, st>>>(
+    launch_k(rope_kv_kernel<false>, dim3(static_cast<unsigned>(n)), dim3(128), 0, st,
         qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
         pool_blocks, q_out, status);
   return cudaGetLastError();
@@ -391,7 +407,7 @@ cudaError_t launch_lm_head(const float* x_row, const float* g, int32_t d, float 
                            const uint16_t* w, int64_t vocab, float* logits, int num_sms,
                            cudaStream_t st) {
   const int grid = num_sms * 4;
-  lm_head_kernel<<<grid, 256, static_cast<size_t>(d) * sizeof(float), st>>>(x_row, g, d, eps, w,
+  launch_k(lm_head_kernel, dim3(grid), dim3(256), static_cast<size_t>(d) * sizeof(float), st, x_row, g, d, eps, w,
                                                                             vocab, logits);
   return cudaGetLastError();
 }
@@ -406,7 +422,7 @@ cudaError_t launch_copy16(const void* src, void* dst, int64_t bytes, cudaStream_
   const int64_t n = (bytes + 15) / 16;
   if (n <= 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((n + 255) / 256, 1024);
-  copy16_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(static_cast<const uint4*>(src),
+  launch_k(copy16_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, static_cast<const uint4*>(src),
                                                                 static_cast<uint4*>(dst), n);
   return cudaGetLastError();
 }

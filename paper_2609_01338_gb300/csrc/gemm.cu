@@ -85,6 +85,7 @@ template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw,
     const __grid_constant__ CUtensorMap tmo, int m, int n, int k, int32_t* status) {
+  pdl_enter();
   using C = PCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -340,7 +341,7 @@ cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void
     return cudaErrorInvalidValue;
   const int64_t tiles = ((m + BM - 1) / BM) * ((n + BN - 1) / BN);
   const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
-  gemm_persistent_kernel<BN, STAGES, EPI><<<grid, 192, C::SMEM, st>>>(
+  launch_k(gemm_persistent_kernel<BN, STAGES, EPI>, dim3(grid), dim3(192), C::SMEM, st,
       ta, tw, tmo, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
   return cudaGetLastError();
 }

@@ -105,6 +105,7 @@ template <int MT, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw, void* __restrict__ out,
     int m, int n, int k, int32_t* status) {
+  pdl_enter();
   using C = SKCfg<MT>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -312,13 +313,15 @@ cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out
   cfg.blockDim = dim3(192, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(S);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<MT, EPI>, ta, tw128, out, static_cast<int>(m),
                             static_cast<int>(n), static_cast<int>(k), status);
 }

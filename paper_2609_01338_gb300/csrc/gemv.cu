@@ -10,6 +10,7 @@
 #include <cuda_fp16.h>
 
 #include "kernels.hpp"
+#include "ptx.cuh"
 
 namespace mzc {
 
@@ -43,6 +44,7 @@ template <int EPI, int MR>
 __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ a,
                                                    const uint16_t* __restrict__ w,
                                                    void* __restrict__ out, int m, int n, int k) {
+  pdl_enter();
   constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
   const int lane = threadIdx.x & 31;
   const int j = static_cast<int>((static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5);
@@ -111,7 +113,7 @@ cudaError_t launch_mr(const uint16_t* a, const uint16_t* w, void* out, int64_t m
                       int64_t k, cudaStream_t st) {
   const int64_t n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
   const int64_t threads = n_out * 32;
-  gemv_kernel<EPI, MR><<<static_cast<unsigned>((threads + 255) / 256), 256, 0, st>>>(
+  launch_k(gemv_kernel<EPI, MR>, dim3(static_cast<unsigned>((threads + 255) / 256)), dim3(256), 0, st,
       a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k));
   return cudaGetLastError();
 }

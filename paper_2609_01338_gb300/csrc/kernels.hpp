@@ -5,8 +5,31 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <utility>
 
 namespace mzc {
+
+// Programmatic dependent launch for the hot-path kernels (on unless the
+// environment sets MZC_PDL=0 when the library loads): the next kernel of a
+// stream is scheduled while the previous one finishes and waits in
+// pdl_enter() for its results, hiding launch and CTA-scheduling latency.
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
 

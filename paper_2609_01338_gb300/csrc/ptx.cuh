@@ -69,6 +69,21 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_
   }
 }
 
+// ---- programmatic dependent launch ----------------------------------------
+// A kernel launched with programmatic stream serialization may start while the
+// previous kernel of its stream still runs; pdl_wait() blocks until that
+// kernel has completed and its writes are visible, and pdl_release() lets the
+// next kernel of the stream be scheduled once every CTA of this one has
+// passed it.  Both are no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_release() { asm volatile("griddepcontrol.launch_dependents;" :::); }
+// Called first in every kernel of the hot path, before it reads or writes
+// anything another kernel touches.
+__device__ __forceinline__ void pdl_enter() {
+  pdl_wait();
+  pdl_release();
+}
+
 // ---- TMA ------------------------------------------------------------------
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
