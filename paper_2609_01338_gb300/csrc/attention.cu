@@ -175,7 +175,6 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     int64_t pool_blocks,
     uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
     int keys_per_split, int n_splits, float scale_log2, int32_t* status) {
-  pdl_enter();
   using C = AttnCfg<HD>;
   constexpr int BN = C::BN;
   extern __shared__ uint8_t smem_raw[];
@@ -228,6 +227,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     tma_prefetch_desc(&pool_blk);
   }
   if (warp == C::PRODUCER_WARP) tmem_alloc(&s_tmem, C::TMEM_COLS);
+  // the prologue above touches no memory another kernel writes
+  pdl_enter();
 
   // softmax threads: tile and row; the Q tiles in the UMMA K-major layout
   const int qt = tid >> 7;  // Q tile of the softmax warps

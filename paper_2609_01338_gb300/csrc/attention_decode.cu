@@ -113,7 +113,6 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     int64_t pool_blocks, uint16_t* __restrict__ out, float* __restrict__ part_o,
     float* __restrict__ part_lse, int blocks_per_split, int n_splits, float scale_log2,
     int32_t* status) {
-  pdl_enter();
   using C = DecCfg<HD>;
   constexpr int DPL = C::DPL;
   extern __shared__ uint8_t smem_raw[];
@@ -139,6 +138,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     }
     fence_barrier_init();
   }
+  // the prologue above touches no memory another kernel writes
+  pdl_enter();
   __syncthreads();
   if (tid < n) atomicMax(&s_maxpos, pos[tid]);
   // this lane's head-dim columns of every q row, and every row's position

@@ -85,7 +85,6 @@ template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw,
     const __grid_constant__ CUtensorMap tmo, int m, int n, int k, int32_t* status) {
-  pdl_enter();
   using C = PCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -125,6 +124,8 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the prologue above touches no memory another kernel writes
+  pdl_enter();
   const uint32_t tmem = s_tmem;
 
   if (warp == 0) {

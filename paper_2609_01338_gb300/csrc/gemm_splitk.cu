@@ -105,7 +105,6 @@ template <int MT, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw, void* __restrict__ out,
     int m, int n, int k, int32_t* status) {
-  pdl_enter();
   using C = SKCfg<MT>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -140,6 +139,8 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the prologue above touches no memory another kernel writes
+  pdl_enter();
   const uint32_t tmem = s_tmem;
 
   if (warp == 0) {
