@@ -302,3 +302,43 @@ def test_decode_steps_match_oracle(tiny):
         tok = int(np.argmax(lg_ref))
     assert m.mzc_stats(c).context_tokens == len(tiny["ctx"]) + 20
     m.mzc_destroy(c)
+
+
+_PDL_SCRIPT = r"""
+import sys
+import numpy as np
+import paper_2609_01338_gb300 as m
+import synth
+from synth import workloads as W
+sh = W.TINY
+w = synth.model_weights(sh)
+ctx = synth.tokens(synth.SEED_CONTEXT, 0, 512, sh["vocab"])
+prm = synth.tokens(synth.SEED_PROMPT, 0, 32, sh["vocab"])
+c = m.mzc_create(sh, w)
+outs = []
+for toks in (ctx, prm, prm[:1], prm[1:2], prm[2:4]):  # 512, 32, then 1, 1 and 2 rows
+    lg = np.empty(sh["vocab"], np.float32)
+    m.mzc_prefill(c, toks, lg)
+    outs.append(lg)
+m.mzc_destroy(c)
+np.save(sys.argv[1], np.stack(outs))
+"""
+
+
+def test_programmatic_dependent_launch_changes_no_bit(tmp_path):
+    """The same prefill and decode steps with programmatic dependent launch
+    off and on (a fresh process each: the switch is read at load) give
+    bit-identical logits, so no kernel touches memory before its wait."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    got = []
+    for v in ("0", "1"):
+        out = tmp_path / f"pdl{v}.npy"
+        env = dict(os.environ, MZC_PDL=v, PYTHONPATH=root + os.pathsep + os.environ.get("PYTHONPATH", ""))
+        subprocess.run([sys.executable, "-c", _PDL_SCRIPT, str(out)], cwd=root, env=env, check=True,
+                       timeout=600)
+        got.append(np.load(out))
+    assert got[0].shape == (5, W.TINY["vocab"])
+    assert np.array_equal(got[0], got[1])
