@@ -201,13 +201,18 @@ mzc_status mzc_set_policy(mzc_ctx *ctx, int32_t policy, const mzc_profile *profi
  * profiled per-unit times).  The prediction runs the paths layer by layer:
  * a layer's QKV projection, rotary/KV write and attention of recomputed rows
  * never wait; the rest of layer l starts once layer l's copy (copy time / L
- * each, in layer order) has landed.  Returns s = p (copy only) unless the
- * split is predicted to be at least 5% faster. */
+ * each, in layer order) has landed.  Attention of recomputed rows runs at a
+ * rate reached linearly from the prompt rate (128 rows) to the recompute rate
+ * (2048 rows).  Only splits whose per-layer compute stays within 95% of the
+ * per-layer copy are taken, and s = p (copy only) is returned unless the best
+ * split is predicted to be at least 1% faster. */
 mzc_status mzc_plan_split(const mzc_model_shape *shape, const mzc_profile *profile, int64_t p,
                           int64_t n_ctx, int64_t n_prompt, int64_t *s_out);
 /* The same split for this ctx's context, with its profile (mzc_set_policy or
  * mzc_profile_measure) and its swap codec: a compressed store moves
- * mzc_q8_block_bytes per block over the link. */
+ * mzc_q8_block_bytes per block over the link, and (its decode kernels share
+ * the SMs with the recompute) splits only for a predicted gain of 5%, with no
+ * per-layer compute bound. */
 mzc_status mzc_plan_split_ctx(mzc_ctx *ctx, int64_t p, int64_t n_prompt, int64_t *s_out);
 
 /* Measures the per-unit profile on this ctx's device (the paper's one-time

@@ -653,8 +653,9 @@ struct CostModelShape {
 // Copy: evicted blocks x bytes / host-link rate, layer after layer.  Compute
 // of the fused rows (recomputed tail + prompt), per layer: the projections
 // interpolated from their measured times at 128 / 512 / 2048 rows, attention
-// pairs at the measured rates of recompute-like and prompt-like rows, per-row
-// memory-bound kernels and a fixed per-layer cost.  The two paths overlap
+// pairs at the measured rates of recompute-like and prompt-like rows (the
+// recompute rate reached linearly from the prompt rate between 128 and 2048
+// recomputed rows), per-row memory-bound kernels and a fixed per-layer cost.  The two paths overlap
 // layer by layer: the part of a layer before the attention that reads copied
 // keys (QKV projection, rotary/KV write, attention of the recomputed rows)
 // never waits; the rest starts once that layer's copy has landed.
@@ -682,8 +683,12 @@ struct CostModel : CostModelShape {
     auto tri = [](double a, double b) { return (b * (b + 1) - a * (a + 1)) / 2.0; };
     const double rec_pairs = tri(static_cast<double>(p0), static_cast<double>(s1));
     const double prm_pairs = tri(static_cast<double>(n_ctx), static_cast<double>(n_ctx + n_prompt));
-    const double rec_attn = rec_pairs * attn_flops_pair / (p.attn_tflops * 1e12) +
-                            static_cast<double>(s1 - p0) * p.attn_row_ns * 1e-9;
+    // a few hundred recomputed rows fill few CTAs and run near the prompt
+    // rate; the recompute rate holds from 2048 rows on
+    const double nrec = static_cast<double>(s1 - p0);
+    const double w = std::min(1.0, std::max(0.0, (nrec - 128.0) / 1920.0));
+    const double rec_rate = p.attn_prompt_tflops + (p.attn_tflops - p.attn_prompt_tflops) * w;
+    const double rec_attn = rec_pairs * attn_flops_pair / (rec_rate * 1e12) + nrec * p.attn_row_ns * 1e-9;
     const double prm_attn = prm_pairs * attn_flops_pair / (p.attn_prompt_tflops * 1e12);
     const double g = gemm_s(rows), rw = rows * p.row_ns * 1e-9, fixed = p.layer_us * 1e-6;
     if (pre) *pre = g * qkv_frac + rec_attn + rw * (2.0 / 3.0) + fixed * 0.5;
@@ -886,8 +891,19 @@ mzc_status mzc_set_policy(mzc_ctx* ctx, int32_t policy, const mzc_profile* profi
   return MZC_OK;
 }
 
-mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profile, int64_t p,
-                          int64_t n_ctx, int64_t n_prompt, int64_t* s_out) {
+}  // extern "C"
+
+namespace {
+
+// The split s minimising the predicted TTFT among the block boundaries from p
+// and n_ctx itself.  A split other than copy-only (s = p) must be predicted
+// min_gain faster, and, when headroom < 1, keep the compute of a layer within
+// headroom x the copy time of a layer: the layer-by-layer overlap then stays
+// bound by the link, whose rate the model knows best, and an underestimate of
+// the compute cannot turn the step compute-bound.
+mzc_status plan_split_impl(const mzc_model_shape* shape, const mzc_profile* profile, int64_t p,
+                           int64_t n_ctx, int64_t n_prompt, double min_gain, double headroom,
+                           int64_t* s_out) {
   if (!shape || !s_out || p < 0 || n_ctx < p || n_prompt < 0) return MZC_ERR_INVALID;
   const mzc_profile prof = profile ? *profile : default_profile();
   if (prof.h2d_gbs <= 0 || prof.gemm_us_128 <= 0 || prof.gemm_us_512 <= 0 || prof.gemm_us_2048 <= 0 ||
@@ -895,32 +911,49 @@ mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profi
       prof.layer_us < 0)
     return MZC_ERR_INVALID;
   CostModel cm(*shape, prof);
-  // candidates: block boundaries from p, and n_ctx itself; leave copy-only
-  // (s = p) only for a predicted gain of at least 5%
   const double copy_only = cm.ttft_s(p, p, n_ctx, n_prompt);
   int64_t best = p;
   double best_t = copy_only;
   for (int64_t s = p + 16;; s += 16) {
     const int64_t sc = std::min(s, n_ctx);
     const double t = cm.ttft_s(p, sc, n_ctx, n_prompt);
-    if (t < best_t) {
+    bool fits = true;
+    if (headroom < 1.0 && sc < n_ctx)
+      fits = cm.layer_s(p, sc, n_ctx, n_prompt) <= headroom * cm.copy_s(n_ctx - sc) / shape->n_layers;
+    if (fits && t < best_t) {
       best_t = t;
       best = sc;
     }
     if (sc >= n_ctx) break;
   }
-  if (best_t > 0.95 * copy_only) best = p;
+  if (best_t > (1.0 - min_gain) * copy_only) best = p;
   *s_out = best;
   return MZC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+// Raw store: a 1% predicted gain with every layer's compute within 95% of
+// its copy (3B sweep: copy-only was kept at f <= 0.25 and beaten at f = 0.75
+// and 1; a 1% margin without the headroom made f = 0.5 slower).
+mzc_status mzc_plan_split(const mzc_model_shape* shape, const mzc_profile* profile, int64_t p,
+                          int64_t n_ctx, int64_t n_prompt, int64_t* s_out) {
+  return plan_split_impl(shape, profile, p, n_ctx, n_prompt, 0.01, 0.95, s_out);
 }
 
 mzc_status mzc_plan_split_ctx(mzc_ctx* ctx, int64_t p, int64_t n_prompt, int64_t* s_out) {
   if (!ctx || !s_out) return MZC_ERR_INVALID;
   // the model prices a copied block at its stored size over the link; a
-  // compressed store moves slot_bytes per block
+  // compressed store moves slot_bytes per block.  Its decode kernels share the
+  // SMs with the recompute, which the model does not price, so a compressed
+  // store splits only for a predicted gain of 5%.
   mzc_profile pr = ctx->prof;
   pr.h2d_gbs *= static_cast<double>(ctx->block_bytes) / static_cast<double>(ctx->slot_bytes);
-  mzc_status e = mzc_plan_split(&ctx->shape, &pr, p, ctx->st.n_ctx(), n_prompt, s_out);
+  const bool raw = ctx->codec == MZC_CODEC_NONE;
+  mzc_status e = plan_split_impl(&ctx->shape, &pr, p, ctx->st.n_ctx(), n_prompt, raw ? 0.01 : 0.05,
+                                 raw ? 0.95 : 1.0, s_out);
   return e == MZC_OK ? e : ctx->fail(e, "hybrid split failed");
 }
 
