@@ -387,12 +387,7 @@ def main():
     ks = {nm: m.mzc_kernel_stats(r.c, i) for i, nm in enumerate(m.KERNEL_CLASS_NAMES)}
     m.mzc_set_kernel_timing(r.c, 0)
 
-    v = statistics.median(dev)
-    e2e = statistics.median(host)
-    if dist:
-        t = torch.tensor([v, e2e], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        v, e2e = float(t[0]), float(t[1])
+    v, e2e = max_over_ranks([statistics.median(dev), statistics.median(host)], dist, "cuda")
 
     peaks, src = _peaks()
     launches = sum(k.launches for k in ks.values())
@@ -460,6 +455,17 @@ def main():
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+def max_over_ranks(vals, dist, device):
+    """Each value's maximum over the ranks (replicas: the job's TTFT is its
+    slowest replica's); the values unchanged on a single process."""
+    if dist is None:
+        return [float(x) for x in vals]
+    import torch
+    t = torch.tensor([float(x) for x in vals], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
 
 
 def run_sweep(r, args, rank):
