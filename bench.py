@@ -42,13 +42,16 @@ sys.path.insert(0, ROOT)
 METRIC = "TTFT ms vs evicted fraction (1 GB300); recompute tok/s; % BF16 tensor peak"
 
 
-def _traffic(kernel_class):
+def _traffic(kernel_class, workload):
     """Per-launch DRAM bytes from the committed ncu capture, or None when the
-    kernel's source changed since the counters were taken."""
+    capture was of another workload or the kernel's source changed since the
+    counters were taken."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
             t = json.load(f)[kernel_class]
+        if t.get("workload") != workload:
+            return None
         src = open(os.path.join(ROOT, t["source"]), "rb").read()
         if hashlib.sha256(src).hexdigest()[:16] != t["source_sha"]:
             return None
@@ -396,18 +399,22 @@ def main():
     if not args.no_kernel_timing:
         k = ks[dom]
         per = k.launches if k.launches else 1
-        if dom in ("gemm", "attention"):
+        # the bound follows the launches' arithmetic intensity: below the ridge
+        # (sustained FLOP/s over HBM bytes/s) a contraction streams its operands
+        ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+        tensor_bound = dom in ("gemm", "attention") and (k.bytes <= 0 or k.flops / k.bytes >= ridge)
+        if tensor_bound:
             ach = k.flops / (k.ms * 1e-3) / 1e12
             peak = peaks["bf16_tflops_sustained"]
             roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 2), "peak": peak,
-                    "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom),
+                    "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom, name),
                     "peak_source": f"{src} bf16 sustained (fp16 operands: nominal fp16/bf16 ratio 1.0)",
                     "avg_launch_ms": round(k.ms / per, 4), "flops_per_launch": k.flops / per}
         else:
             ach = k.bytes / (k.ms * 1e-3) / 1e9
             peak = peaks["hbm_gbs"]
             roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": peak,
-                    "unit": "GB/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom),
+                    "unit": "GB/s", "frac": round(ach / peak, 4), "traffic": _traffic(dom, name),
                     "peak_source": f"{src} HBM copy", "avg_launch_ms": round(k.ms / per, 4),
                     "bytes_per_launch": k.bytes / per}
     rows = stats.rows_last
