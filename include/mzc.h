@@ -325,7 +325,12 @@ mzc_status mzc_k_rmsnorm(const float *x, const float *g, int64_t n, int32_t d, f
  *   1: out fp32 [m][n] += C                       (residual add)
  *   2: out fp16 [m][n/2] = silu(C_gate) * C_up     (SwiGLU; W's rows must be in
  *      the interleaved order mzc_k_swiglu_pack produces)
- * k must be a multiple of 8; n a multiple of 16 (epilogue 2: of 128). */
+ * k must be a multiple of 8; n a multiple of 16 (epilogue 2: of 128).
+ * Kernel by m: up to 4 rows a GEMV streaming W (K split over two warps for
+ * rows of 6 KB and more); up to 256 rows, when n is a multiple of 128, the K
+ * range split over a thread-block cluster with the partials summed in a
+ * fixed order; otherwise the persistent tcgen05 GEMM.  Each path gives the
+ * same bits on every run. */
 mzc_status mzc_k_gemm(const uint16_t *a, const uint16_t *w, void *out, int64_t m, int64_t n,
                       int64_t k, int32_t epilogue, void *stream);
 /* Host helper: interleaves gate [f][d] and up [f][d] into the [2f][d] row
