@@ -8,6 +8,11 @@ layers for recompute; restore moves every swapped block to INFLIGHT; a
 completed prefill makes in-flight and recomputed blocks RESIDENT and appends
 the prompt.  Physical block numbers are not modelled (any valid, distinct
 assignment is correct); the tests check them for validity only.
+
+Pinned by tests/test_oracle_state_pins.py: literal tables and status codes
+worked out by hand from the rules above (outward rounding, one contiguous
+all-layer DROP range, double eviction, prefill over dropped or swapped
+blocks, recompute range, truncation inside a dropped range).
 """
 from __future__ import annotations
 
