@@ -25,8 +25,11 @@
  *   - Token ranges are in absolute positions of the context; KV blocks are
  *     block_tokens (16) consecutive positions of one layer.
  *   - KV storage: K/V values are rounded to the shape's kv_dtype (bf16 or
- *     fp16) and held in fp16 encoding in either case (every normal-range bf16
- *     value is exactly an fp16 value), so attention reads one format.
+ *     fp16) and held in fp16 encoding in either case, so attention reads one
+ *     format.  For a bf16 KV type the encoding is exact only inside fp16's
+ *     range: zero and magnitudes in [2^-14, 65504].  A bf16 K/V value below
+ *     2^-14 keeps only fp16-subnormal precision, and one above 65504 does not
+ *     fit at all.
  */
 #ifndef MZC_H
 #define MZC_H
@@ -216,8 +219,15 @@ mzc_status mzc_plan_split(const mzc_model_shape *shape, const mzc_profile *profi
 mzc_status mzc_plan_split_ctx(mzc_ctx *ctx, int64_t p, int64_t n_prompt, int64_t *s_out);
 
 /* Measures the per-unit profile on this ctx's device (the paper's one-time
- * offline profiling, Sec. 4.3): timed host->device copies from the pinned
- * store, and the ctx's own GEMM and attention kernels on scratch. */
+ * offline profiling, Sec. 4.3, which must leave the memory state as it was):
+ *   - the host link: timed pinned host -> device copies into device memory
+ *     that holds no live KV (the longest run of free pool blocks, poisoned
+ *     again afterwards like every freed block, or the ctx's staging buffer);
+ *   - the ctx's own GEMM, attention and RMSNorm kernels on its activation
+ *     buffers (which hold nothing live between prefills); the attention reads
+ *     the resident context's blocks and writes none.
+ * Resident KV blocks, block tables and residency are unchanged.  Errors:
+ * MZC_ERR_STATE while a restore is in flight or a recompute is pending. */
 mzc_status mzc_profile_measure(mzc_ctx *ctx, mzc_profile *out);
 
 /* Shrinks the context to n_ctx positions (frees the blocks past it). */

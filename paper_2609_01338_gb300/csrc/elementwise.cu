@@ -325,10 +325,12 @@ __global__ void gather_blocks_kernel(const uint4* __restrict__ pool, const int32
   for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = src[c];
 }
 
+// Block b of the list (phys non-null) or of the run phys_begin + b (phys null).
 __global__ void poison_blocks_kernel(uint4* __restrict__ pool, const int32_t* __restrict__ phys,
-                                     int64_t chunks_per_block, uint32_t pattern2) {
+                                     int64_t phys_begin, int64_t chunks_per_block, uint32_t pattern2) {
   const int64_t b = blockIdx.x;
-  uint4* d = pool + static_cast<int64_t>(phys[b]) * chunks_per_block;
+  const int64_t pb = phys ? static_cast<int64_t>(phys[b]) : phys_begin + b;
+  uint4* d = pool + pb * chunks_per_block;
   const uint4 v = make_uint4(pattern2, pattern2, pattern2, pattern2);
   for (int64_t c = threadIdx.x; c < chunks_per_block; c += blockDim.x) d[c] = v;
 }
@@ -443,8 +445,18 @@ cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int
   // before its restore lands shows up in the results
   (void)kv_dtype;
   const uint32_t v16 = 0x7BFFu;  // the pool is fp16-encoded for both KV types
-  poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), phys,
+  poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), phys, 0,
                                                                   block_bytes / 16, v16 | (v16 << 16));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_poison_run(void* pool, int64_t phys_begin, int64_t n, int64_t block_bytes,
+                              cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  const uint32_t v16 = 0x7BFFu;
+  poison_blocks_kernel<<<static_cast<unsigned>(n), 256, 0, st>>>(static_cast<uint4*>(pool), nullptr,
+                                                                  phys_begin, block_bytes / 16,
+                                                                  v16 | (v16 << 16));
   return cudaGetLastError();
 }
 

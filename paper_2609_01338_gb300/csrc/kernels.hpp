@@ -135,5 +135,8 @@ cudaError_t launch_gather_blocks(const void* pool, const int32_t* phys, int64_t 
 // Fills blocks phys[i] with the largest finite value of the KV type.
 cudaError_t launch_poison_blocks(void* pool, const int32_t* phys, int64_t n, int64_t block_bytes,
                                  int32_t kv_dtype, cudaStream_t st);
+// Poisons the contiguous physical blocks [phys_begin, phys_begin + n).
+cudaError_t launch_poison_run(void* pool, int64_t phys_begin, int64_t n, int64_t block_bytes,
+                              cudaStream_t st);
 
 }  // namespace mzc

@@ -1091,27 +1091,41 @@ const char* mzc_last_error(mzc_ctx* ctx) {
 
 mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
   if (!ctx || !out) return MZC_ERR_INVALID;
+  if (ctx->st.restore_in_flight() || ctx->st.recompute_pending())
+    return ctx->fail(MZC_ERR_STATE, "profiling needs a ctx with no restore or recompute pending");
   CK(cudaSetDevice(ctx->opt.device));
   mzc_profile p = ctx->prof;
   cudaEvent_t a, b;
   CK(cudaEventCreate(&a));
   CK(cudaEventCreate(&b));
   float ms = 0.0f;
-  // host link: 256 MiB (or the store) pinned -> device, on the copy stream
+  // Host link: timed pinned -> device copies on the copy stream, into device
+  // memory that holds no live KV -- the longest run of free pool blocks, which
+  // is poisoned again afterwards like every freed block, or the ctx's staging
+  // buffer, whichever is larger.  Resident blocks are never written.
   {
-    const int64_t bytes = std::min<int64_t>(256LL << 20, ctx->st.pool_blocks() * ctx->block_bytes);
+    int64_t run0 = 0;
+    const int64_t run_n = ctx->st.largest_free_pool_run(&run0);
+    const int64_t staging = ctx->nblk * ctx->block_bytes;
+    const bool use_pool = run_n * ctx->block_bytes > staging;
+    uint8_t* dst = use_pool ? ctx->d_pool + run0 * ctx->block_bytes : ctx->d_staging;
+    const int64_t bytes = std::min<int64_t>(256LL << 20, use_pool ? run_n * ctx->block_bytes : staging);
+    // about 1 GiB in all (4 to 64 copies), so small buffers still time steadily
+    const int reps = static_cast<int>(std::min<int64_t>(64, std::max<int64_t>(4, (1LL << 30) / bytes)));
     uint8_t* h = nullptr;
     CK(cudaHostAlloc(&h, bytes, cudaHostAllocDefault));
     std::memset(h, 1, bytes);
-    CK(cudaMemcpyAsync(ctx->d_pool, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
+    CK(cudaMemcpyAsync(dst, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
     CK(cudaEventRecord(a, ctx->xs));
-    for (int i = 0; i < 4; ++i) CK(cudaMemcpyAsync(ctx->d_pool, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
+    for (int i = 0; i < reps; ++i) CK(cudaMemcpyAsync(dst, h, bytes, cudaMemcpyHostToDevice, ctx->xs));
     CK(cudaEventRecord(b, ctx->xs));
     CK(cudaEventSynchronize(b));
     CK(cudaEventElapsedTime(&ms, a, b));
-    p.h2d_gbs = 4.0 * bytes / (ms * 1e-3) / 1e9;
+    p.h2d_gbs = static_cast<double>(reps) * bytes / (ms * 1e-3) / 1e9;
+    if (use_pool)
+      CK(mzc::launch_poison_run(ctx->d_pool, run0, ceil_div(bytes, ctx->block_bytes), ctx->block_bytes, ctx->xs));
+    CK(cudaStreamSynchronize(ctx->xs));
     CK(cudaFreeHost(h));
-    CK(cudaMemset(ctx->d_pool, 0, bytes));
   }
   // A whole layer's four projections on scratch activations at 128, 512 and
   // 2048 rows (capped by max_rows).

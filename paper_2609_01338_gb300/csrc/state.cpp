@@ -53,6 +53,17 @@ std::vector<std::pair<int64_t, int64_t>> RangeAlloc::alloc_runs(int64_t n) {
   return out;
 }
 
+int64_t RangeAlloc::largest_free(int64_t* start) const {
+  int64_t best = 0, at = 0;
+  for (const auto& kv : free_)
+    if (kv.second > best) {
+      best = kv.second;
+      at = kv.first;
+    }
+  if (start) *start = at;
+  return best;
+}
+
 void RangeAlloc::release(int64_t start, int64_t n) {
   if (n <= 0) return;
   free_total_ += n;

@@ -30,6 +30,8 @@ class RangeAlloc {
   // otherwise the lowest-addressed free ranges.  Empty if free_total < n.
   std::vector<std::pair<int64_t, int64_t>> alloc_runs(int64_t n);
   void release(int64_t start, int64_t n);
+  // The longest free range: its length, and its start in *start (0 if none).
+  int64_t largest_free(int64_t* start) const;
 
  private:
   std::map<int64_t, int64_t> free_;  // start -> length
@@ -122,6 +124,8 @@ class State {
   mzc_status truncate(int64_t n_ctx);
 
   int32_t weight_state(int32_t l) const { return w_state_[l]; }
+  // Longest run of free physical blocks (holds no live KV): length, start.
+  int64_t largest_free_pool_run(int64_t* start) const { return pool_.largest_free(start); }
   void counts(mzc_stats_t* out) const;
   // Block table rows [L][nblk_max] (phys or -1) for the device.
   void block_table(std::vector<int32_t>* out) const;
