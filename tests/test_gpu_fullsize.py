@@ -33,21 +33,35 @@ def _ctx(sc):
     return sh, w, c, ctx_tok, prm
 
 
-def _one_row_check(sh, w, c, n_total, row_pos, token, gpu_logits=None):
-    """Oracle forward of one row over the GPU's KV of all other positions;
-    compares that row's K/V per layer and (optionally) the logits."""
-    k, v = m.mzc_read_kv_all(c, n_total, sh)
+def _kv_state(k, v):
     kv = oracle.KVState.__new__(oracle.KVState)
-    kv.k, kv.v, kv.max_ctx = k, v, n_total
+    kv.k, kv.v, kv.max_ctx = k, v, k.shape[1]
+    return kv
+
+
+def _row_check(sh, w, k, v, row_pos, token, gpu_logits=None):
+    """Oracle forward of one row at row_pos over the GPU's K/V of every other
+    position (k, v: [n_layers][n][n_kv_heads][head_dim], as read back, left
+    unchanged); compares that row's K/V per layer and (optionally) the
+    first-token logits."""
+    kv = _kv_state(k, v)
     gpu_k_row, gpu_v_row = k[:, row_pos].copy(), v[:, row_pos].copy()
     kv.k[:, row_pos] = np.nan
     kv.v[:, row_pos] = np.nan
-    lg = oracle.forward(sh, w, kv, [token], [row_pos], logits=gpu_logits is not None)
-    for l in range(sh["n_layers"]):
-        assert rel_err(gpu_k_row[l], kv.k[l, row_pos]) < KV_TOL, l
-        assert rel_err(gpu_v_row[l], kv.v[l, row_pos]) < KV_TOL, l
-    if gpu_logits is not None:
-        assert np.max(np.abs(gpu_logits - lg)) < LOGIT_TOL
+    try:
+        lg = oracle.forward(sh, w, kv, [token], [row_pos], logits=gpu_logits is not None)
+        for l in range(sh["n_layers"]):
+            assert rel_err(gpu_k_row[l], kv.k[l, row_pos]) < KV_TOL, (row_pos, l)
+            assert rel_err(gpu_v_row[l], kv.v[l, row_pos]) < KV_TOL, (row_pos, l)
+        if gpu_logits is not None:
+            assert np.max(np.abs(gpu_logits - lg)) < LOGIT_TOL
+    finally:
+        k[:, row_pos], v[:, row_pos] = gpu_k_row, gpu_v_row
+
+
+def _one_row_check(sh, w, c, n_total, row_pos, token, gpu_logits=None):
+    k, v = m.mzc_read_kv_all(c, n_total, sh)
+    _row_check(sh, w, k, v, row_pos, token, gpu_logits)
     return k, v
 
 
@@ -70,8 +84,10 @@ def test_1b_recompute_full_size():
         assert rel_err(k[l, p:N], k_pre[l, p:N]) < KV_TOL
         assert rel_err(v[l, p:N], v_pre[l, p:N]) < KV_TOL
         assert np.array_equal(k[l, :p], k_pre[l, :p])  # resident prefix untouched
-    # a recomputed row checked one by one against the oracle
-    _one_row_check(sh, w, c, N + P, p + 1234, ctx_tok[p + 1234])
+    # eight recomputed rows, evenly spaced over [p, N) (first and last
+    # included), each checked one by one against the oracle
+    for r in np.linspace(p, N - 1, 8).astype(int):
+        _row_check(sh, w, k, v, int(r), int(ctx_tok[r]))
     m.mzc_destroy(c)
 
 

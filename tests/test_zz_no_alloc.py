@@ -1,22 +1,27 @@
-"""The allocation-free attention entry point against the ordinary one.
+"""The allocation-free attention entry point against the CPU oracle and the
+ordinary entry point.
 
 Some callers cannot allocate device memory when they call: a process whose
 device memory is being reclaimed cannot count on an allocation succeeding at
 request time, a host framework may own all device memory through its own
 allocator, and cudaFree synchronizes the device.  mzc_k_attention_noalloc
 serves them by keeping its split-KV partials in a fixed device array inside
-the library.  This file checks, through the C ABI, that it returns what
-mzc_k_attention returns with caller-allocated scratch (within the attention
-tolerance of the other GPU tests) on two calls in a row with different inputs,
-so the second call cannot lean on the first call's partials, and that a call
-whose partials would not fit in the array is refused without a launch.  It is
-named to be collected last."""
+the library.  This file checks, through the C ABI, on two calls in a row with
+different shapes and inputs (so the second call cannot lean on the first
+call's partials left in the array):
+  - the output against the CPU oracle's attention over the same K/V, q and
+    positions, at the tolerance of the other attention parity tests;
+  - the output against mzc_k_attention with caller-allocated scratch, at the
+    same tolerance;
+and that a call whose partials would not fit in the array is refused without
+a launch.  It is named to be collected last."""
 import numpy as np
 import pytest
 
+import oracle
 import paper_2609_01338_gb300 as m
 import synth
-from tests.gpu_util import f16_to_f32, f32_to_kv_bits, i32_dev, rel_err, to_np_u16
+from tests.gpu_util import f16_to_f32, f32_to_kv_bits, i32_dev, kv_bits_to_f32, rel_err, to_np_u16
 
 pytestmark = pytest.mark.gpu
 
@@ -39,12 +44,14 @@ def _inputs(seed, hq, hkv, hd, kvd, ctx, n):
     pos = np.arange(ctx - n, ctx).astype(np.int32)
     dev = dict(q=torch.from_numpy(q.view(np.int16)).cuda(), pos=i32_dev(pos),
                table=i32_dev(table), pool=torch.from_numpy(pool.view(np.int16)).cuda())
-    return dev, n_logical, pool_blocks
+    # the oracle's attention over the same stored values (fp16-encoded pool)
+    ref = oracle.attention(f16_to_f32(q), pos, kv_bits_to_f32(k), kv_bits_to_f32(v))
+    return dev, n_logical, pool_blocks, ref
 
 
 def _one_call(seed, hq, hkv, hd, kvd, ctx, n):
     import torch
-    dev, n_logical, pool_blocks = _inputs(seed, hq, hkv, hd, kvd, ctx, n)
+    dev, n_logical, pool_blocks, oracle_ref = _inputs(seed, hq, hkv, hd, kvd, ctx, n)
     need = m.mzc_k_attention_scratch_bytes(n, hq, hkv, hd, ctx)
     assert 0 < need <= m.MZC_ATTENTION_NOALLOC_SCRATCH_BYTES  # the split path is exercised
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
@@ -59,6 +66,8 @@ def _one_call(seed, hq, hkv, hd, kvd, ctx, n):
     assert int(status.item()) == 0
     got, want = f16_to_f32(to_np_u16(out)), f16_to_f32(to_np_u16(ref))
     assert np.all(np.isfinite(got))
+    assert rel_err(got, oracle_ref) < ATTN_TOL
+    assert np.mean(np.abs(got - oracle_ref)) < 2e-3 * np.max(np.abs(oracle_ref))
     assert rel_err(got, want) < ATTN_TOL
 
 
