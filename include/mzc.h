@@ -16,8 +16,9 @@
  * Conventions for every call:
  *   - Status codes only; nothing throws or aborts across the ABI.
  *     mzc_last_error() returns a text for the last failing call on a ctx.
- *   - The ctx owns every device buffer, the pinned swap store and its two
- *     CUDA streams.  Pointers passed in are borrowed for the call only
+ *   - The ctx owns every device buffer, the pinned swap store and its CUDA
+ *     streams (unless the caller passes its own compute and copy streams in
+ *     mzc_options).  Pointers passed in are borrowed for the call only
  *     (mzc_create copies the weights).  Host pointers are plain host memory
  *     unless a parameter says "device".
  *   - One ctx per host thread; calls on one ctx must not overlap.  Different
@@ -28,8 +29,11 @@
  *     fp16) and held in fp16 encoding in either case, so attention reads one
  *     format.  For a bf16 KV type the encoding is exact only inside fp16's
  *     range: zero and magnitudes in [2^-14, 65504].  A bf16 K/V value below
- *     2^-14 keeps only fp16-subnormal precision, and one above 65504 does not
- *     fit at all.
+ *     2^-14 keeps only fp16-subnormal precision, and one of 65520 or more
+ *     does not fit at all: the prefill then fails with MZC_ERR_OVERFLOW.
+ *     The activations the projections read (RMSNorm outputs, SwiGLU
+ *     outputs) and the q/k/v projection outputs are fp16 too, with the same
+ *     check.
  */
 #ifndef MZC_H
 #define MZC_H
@@ -49,7 +53,11 @@ typedef enum {
   MZC_ERR_OOM = 4,     /* KV pool, row capacity or pinned store exhausted */
   MZC_ERR_CUDA = 5,    /* a CUDA runtime call failed; the text names it */
   MZC_ERR_TIMEOUT = 6, /* a bounded device wait gave up (kernel status word) */
-  MZC_ERR_DEVICE = 7   /* a device-side bounds check failed (kernel status word) */
+  MZC_ERR_DEVICE = 7,  /* a device-side bounds check failed (kernel status word) */
+  MZC_ERR_OVERFLOW = 8 /* a device-side range check: an fp16 activation (RMSNorm output,
+                          q/k/v projection, SwiGLU output) or fp16-encoded K/V value reached
+                          65520 in magnitude and was stored as infinity (kernel status word);
+                          the results of that call are not to be used */
 } mzc_status;
 
 enum { MZC_KV_BF16 = 0, MZC_KV_FP16 = 1 };
@@ -72,6 +80,20 @@ typedef struct {
   int64_t max_ctx;      /* positions the context may hold */
 } mzc_model_shape;
 
+/* How a layer's attention waits for the KV blocks a restore copies back
+ * (the zero-wait overlap, Sec. 4.4: prefill consumes each unit as soon as it
+ * is restored):
+ *   MZC_WAIT_LAYER_EVENT: on the copy stream's per-layer event, recorded after
+ *     the last copy of that layer (norms, projections and rotary/KV writes of
+ *     the layer run before the wait);
+ *   MZC_WAIT_BLOCK_FLAG: per physical block.  The copy engine writes a block's
+ *     residency flag right after the block's data, and the attention kernels
+ *     wait (bounded) for the flag of each block they are about to read, so a
+ *     layer's attention starts before its last copy lands and runs behind the
+ *     copies.  Not with MZC_CODEC_Q8 (its decode kernels, not the copy
+ *     engine, write the restored blocks). */
+enum { MZC_WAIT_LAYER_EVENT = 0, MZC_WAIT_BLOCK_FLAG = 1 };
+
 typedef struct {
   int64_t pool_blocks;      /* physical KV blocks; 0 = 2 * n_layers * ceil(max_ctx/16) */
   int64_t max_rows;         /* rows per prefill call (recompute + prompt); 0 = max_ctx */
@@ -82,6 +104,19 @@ typedef struct {
   int32_t swap_codec;       /* MZC_CODEC_NONE: COPY swaps blocks as stored; MZC_CODEC_Q8:
                                8-bit quantized (mzc_k_q8_encode; about 0.56 of the bytes),
                                decoded into the pool on restore */
+  int32_t wait_mode;        /* MZC_WAIT_LAYER_EVENT (default) or MZC_WAIT_BLOCK_FLAG */
+  int32_t debug_checks;     /* 1: before each prefill, check the block tables (every
+                               resident or in-flight block maps to its own physical
+                               block inside the pool); during it, synchronize after each
+                               layer and read the device status word, so an error names
+                               the layer where it appeared.  Slower; results unchanged */
+  int32_t reserved;         /* 0 */
+  void *compute_stream;     /* cudaStream_t the prefill kernels run on, owned by the caller
+                               (it must outlive the ctx); NULL = the ctx creates its own.
+                               mzc_prefill synchronizes this stream before it returns */
+  void *copy_stream;        /* cudaStream_t of the restore copies, owned by the caller;
+                               NULL = own.  The same stream as compute_stream is accepted
+                               and serializes restore and prefill (no overlap) */
 } mzc_options;
 
 /* Weights, host memory, bf16 bit patterns, row-major [out_features][in_features]
@@ -384,6 +419,20 @@ mzc_status mzc_k_attention(const uint16_t *q, const int32_t *pos, int64_t n, int
                            int32_t *status, void *stream);
 int64_t mzc_k_attention_scratch_bytes(int64_t n, int32_t hq, int32_t hkv, int32_t hd,
                                       int64_t max_keys);
+/* mzc_k_attention that first waits for residency flags (the per-block wait
+ * of MZC_WAIT_BLOCK_FLAG; Sec. 4.4's zero-wait consumption of restored
+ * units): block_flags is a device int32 array [pool_blocks], non-zero once a
+ * block's data is in the pool; before fetching a block the kernels wait for
+ * its flag, at most flag_wait_cycles SM clocks (0 = the library's default
+ * limit of about 2 s).  A flag that stays zero makes the call record
+ * MZC_ERR_TIMEOUT in *status and return with that block unread (the output
+ * is then undefined); the CUDA context stays usable. */
+mzc_status mzc_k_attention_wait(const uint16_t *q, const int32_t *pos, int64_t n, int32_t hq,
+                                int32_t hkv, int32_t hd, const int32_t *block_table,
+                                int64_t n_logical, const void *pool, int64_t pool_blocks,
+                                int32_t kv_dtype, uint16_t *out, int64_t max_keys, void *scratch,
+                                int64_t scratch_bytes, const int32_t *block_flags,
+                                int64_t flag_wait_cycles, int32_t *status, void *stream);
 
 /* The paper has no counterpart to this entry point: it is a convenience of
  * this library.  Same arguments and result as mzc_k_attention, but the

@@ -83,6 +83,7 @@ def lib():
             L.orc_q8_encode.argtypes = [vp, i64, vp, vp, vp]
             L.orc_q8_decode.argtypes = [vp, vp, vp, i64, vp]
             L.orc_num_threads.restype = ctypes.c_int
+            L.orc_set_num_threads.argtypes = [ctypes.c_int]
             _lib = L
     return _lib
 
@@ -98,6 +99,12 @@ def _f32(a) -> np.ndarray:
 
 def num_threads() -> int:
     return lib().orc_num_threads()
+
+
+def set_num_threads(n: int) -> None:
+    """Thread count of later oracle calls (timing only; results do not depend
+    on it: each row is computed by one thread in a fixed order)."""
+    lib().orc_set_num_threads(int(n))
 
 
 def shape_struct(shape: dict) -> _Shape:

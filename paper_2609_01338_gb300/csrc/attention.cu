@@ -76,7 +76,7 @@ struct AttnCfg {
   static constexpr uint32_t TMEM_COLS = NQ == 2 ? 512 : 256;
   static_assert(O_COL + NQ * HD <= TMEM_COLS, "S, P and O of every tile fit in TMEM");
   static_assert(TMEM_COLS * CTAS_PER_SM <= 512, "TMEM of the CTAs sharing an SM");
-  static_assert(3 * STAGES * 8 + 4 * NQ * 8 <= 256, "barriers");
+  static_assert(3 * STAGES * 8 + 5 * NQ * 8 <= 256, "barriers");
   static_assert((SMEM + 1024) * CTAS_PER_SM <= 233472, "shared memory of the CTAs sharing an SM");
 };
 
@@ -174,7 +174,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     const __grid_constant__ CUtensorMap pool_run, const __grid_constant__ CUtensorMap pool_blk,
     int64_t pool_blocks,
     uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
-    int keys_per_split, int n_splits, float scale_log2, int32_t* status) {
+    int keys_per_split, int n_splits, float scale_log2, int32_t* status,
+    const int32_t* __restrict__ flags, long long flag_wait_cycles) {
   using C = AttnCfg<HD>;
   constexpr int BN = C::BN;
   extern __shared__ uint8_t smem_raw[];
@@ -191,6 +192,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
   uint64_t* s_free = s_full + C::NQ;          // [NQ tiles] S(j) read into registers
   uint64_t* p_full = s_free + C::NQ;          // [NQ tiles] P(j) in TMEM
   uint64_t* p_free = p_full + C::NQ;          // [NQ tiles] P(j) V(j) done
+  uint64_t* drain = p_free + C::NQ;           // [NQ tiles] every UMMA of the tile's issuer done
   __shared__ uint32_t s_tmem;
   __shared__ int s_maxpos;
   __shared__ int s_abort;
@@ -219,6 +221,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
       mbar_init(&s_free[t], 4);  // one arrival per softmax warp of the tile
       mbar_init(&p_full[t], 4);
       mbar_init(&p_free[t], 1);
+      mbar_init(&drain[t], 1);
     }
     fence_barrier_init();
     s_maxpos = -1;
@@ -277,7 +280,15 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
         const int64_t blk = key0 >> 4;
         return blk < n_logical ? table[blk] : -1;
       };
+      // residency flags (restore copies in flight): a lane's block must have
+      // landed before its keys are fetched.  The flag of the next tile's block
+      // is loaded once this tile's copies are issued (its table entry has
+      // arrived by then), so a flag that is already set costs no wait.
+      auto flag_of = [&](int32_t pb) -> int32_t {
+        return (flags == nullptr || pb < 0 || pb >= pool_blocks) ? 1 : ld_acquire_gpu(flags + pb);
+      };
       int32_t p_cur = lookup(0);
+      int32_t f_cur = flag_of(p_cur);
       int issued = 0;
       for (int j = 0; j < T; ++j) {
         const int s = j % C::STAGES;
@@ -298,6 +309,31 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
         if (lane == 0 && j >= C::STAGES)
           ok = wait_bar(&kv_empty[s], ((j / C::STAGES) - 1) & 1, status, abort_flag);
         if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+        if (flags != nullptr) {
+          bool rdy = !valid || f_cur != 0;
+          if (!__all_sync(0xffffffffu, rdy)) {
+            const long long t0 = clock64();
+            while (true) {
+              if (!rdy) rdy = ld_acquire_gpu(flags + p) != 0;
+              if (__all_sync(0xffffffffu, rdy)) break;
+              // give up at the limit, or at once when another thread of this CTA
+              // or another CTA has timed out already (the status word says so)
+              if (__any_sync(0xffffffffu, *abort_flag != 0 || clock64() - t0 > flag_wait_cycles ||
+                                              (status != nullptr &&
+                                               *reinterpret_cast<volatile int32_t*>(status) == kStatusTimeout))) {
+                if (lane == 0) {
+                  set_status(status, kStatusTimeout);
+                  *abort_flag = 1;
+                }
+                ok = false;
+                break;
+              }
+              __nanosleep(128);
+            }
+            if (!__all_sync(0xffffffffu, ok)) break;
+          }
+          fence_proxy_async_global();  // the TMA reads come after the flags were seen
+        }
         if (lane == 0) {
           mbar_arrive_expect_tx(&k_full[s], C::KV_BYTES);
           mbar_arrive_expect_tx(&v_full[s], C::KV_BYTES);
@@ -322,12 +358,15 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
         }
         issued = j + 1;
         p_cur = p_nxt;
+        if (flags != nullptr) f_cur = flag_of(p_cur);
       }
       // drain: every fill issued has landed before shared memory is released
+      // (a bounded wait without the abort shortcut: after an abort the copies
+      // already issued still land)
       if (lane == 0) {
         for (int j = issued - C::STAGES < 0 ? 0 : issued - C::STAGES; j < issued; ++j) {
-          wait_bar(&k_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
-          wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag);
+          mbar_wait(&k_full[j % C::STAGES], (j / C::STAGES) & 1, status);
+          mbar_wait(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status);
         }
       }
     }
@@ -380,6 +419,10 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
         tc_fence_after();
         issue_pv(j);
       }
+      // every UMMA this thread issued has completed before TMEM is released
+      // (after an abort the softmax warps do not wait for the last ones)
+      umma_commit(&drain[t]);
+      mbar_wait(&drain[t], 0, status);
     }
   } else {
     // ---- softmax: thread = row of Q tile qt, all BN columns ----
@@ -636,7 +679,8 @@ template <int HD, bool F16>
 cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
                       const int32_t* table, int64_t n_logical, const void* pool,
                       int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
-                      int n_splits, int keys_per_split, int32_t* status, cudaStream_t st) {
+                      int n_splits, int keys_per_split, int32_t* status, const int32_t* flags,
+                      long long flag_wait, cudaStream_t st) {
   using C = AttnCfg<HD>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -658,7 +702,7 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
   launch_k(attn_tc_kernel<HD, F16>, dim3(grid), dim3(C::THREADS), C::SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, run_map, blk_map, pool_blocks, out, part_o,
-      part_lse, keys_per_split, n_splits, scale_log2, status);
+      part_lse, keys_per_split, n_splits, scale_log2, status, flags, flag_wait);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || n_splits == 1) return e;
   const int64_t rows = n * hq;
@@ -711,8 +755,10 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
                              int32_t hkv, int32_t hd, const int32_t* table, int64_t n_logical,
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,
                              uint16_t* out, void* scratch, int64_t scratch_bytes,
-                             int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st) {
+                             int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st,
+                             const int32_t* flags, int64_t flag_wait_cycles) {
   if (n <= 0) return cudaSuccess;
+  const long long fw = flag_wait_cycles > 0 ? flag_wait_cycles : kWaitCycles;
   int s = 1, per = 0;
   attention_split(n, hq, hkv, hd, max_keys, num_sms, &s, &per);
   // the combine reads the partials as 8- or 16-byte vectors
@@ -726,7 +772,7 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   (void)kv_dtype;  // the pool is fp16-encoded for both KV types: q, K, P, V are fp16
   if (attention_decode_applies(n, hq, hkv, hd)) {
     cudaError_t e = launch_attention_decode(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks, out,
-                                            part_o, part_lse, s, per, status, st);
+                                            part_o, part_lse, s, per, status, flags, fw, st);
     if (e != cudaSuccess || s == 1) return e;
     const int64_t rows = n * hq;
     if (hd == 64)
@@ -737,10 +783,10 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   }
   if (hd == 64)
     return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
-                               part_o, part_lse, s, per, status, st);
+                               part_o, part_lse, s, per, status, flags, fw, st);
   if (hd == 128)
     return launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
-                                part_o, part_lse, s, per, status, st);
+                                part_o, part_lse, s, per, status, flags, fw, st);
   return cudaErrorInvalidValue;
 }
 

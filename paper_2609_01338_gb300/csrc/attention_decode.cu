@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     const int32_t* __restrict__ table, int64_t n_logical, const uint16_t* __restrict__ pool,
     int64_t pool_blocks, uint16_t* __restrict__ out, float* __restrict__ part_o,
     float* __restrict__ part_lse, int blocks_per_split, int n_splits, float scale_log2,
-    int32_t* status) {
+    int32_t* status, const int32_t* __restrict__ flags, long long flag_wait_cycles) {
   using C = DecCfg<HD>;
   constexpr int DPL = C::DPL;
   extern __shared__ uint8_t smem_raw[];
@@ -189,6 +189,16 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     if (p < 0) {
       mbar_arrive(&pfull[s]);  // completes the phase with no data
       return;
+    }
+    if (flags != nullptr) {
+      // a restore copy into this block may still be in flight: wait (bounded)
+      // for its residency flag; on a timeout the status word says so and the
+      // phase completes with no data
+      if (!flag_wait(flags, p, status, flag_wait_cycles)) {
+        mbar_arrive(&pfull[s]);
+        return;
+      }
+      fence_proxy_async_global();
     }
     fence_proxy_async_smem();  // earlier generic reads of the slot before the async writes
     mbar_arrive_expect_tx(&pfull[s], C::SLOT);
@@ -370,7 +380,7 @@ template <int HD, int R>
 cudaError_t launch_dec(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
                        const int32_t* table, int64_t n_logical, const void* pool, int64_t pool_blocks,
                        uint16_t* out, float* part_o, float* part_lse, int n_splits, int blocks_per_split,
-                       int32_t* status, cudaStream_t st) {
+                       int32_t* status, const int32_t* flags, long long flag_wait, cudaStream_t st) {
   constexpr int SMEM = dec_smem_bytes<HD>();
   static_assert(SMEM <= 232448, "shared memory of one CTA");
   static_assert(kDecWarps * R * (HD + 2) * 4 <= DecCfg<HD>::RING, "warp partials fit in the rings");
@@ -386,7 +396,7 @@ cudaError_t launch_dec(const uint16_t* q, const int32_t* pos, int64_t n, int32_t
   dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(n_splits));
   launch_k(attn_decode_kernel<HD, R>, dim3(grid), dim3(kDecThreads), SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, static_cast<const uint16_t*>(pool), pool_blocks,
-      out, part_o, part_lse, blocks_per_split, n_splits, scale_log2, status);
+      out, part_o, part_lse, blocks_per_split, n_splits, scale_log2, status, flags, flag_wait);
   return cudaGetLastError();
 }
 
@@ -411,7 +421,8 @@ void attention_decode_split(int32_t hkv, int64_t max_keys, int num_sms, int* n_s
 cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
                                     int32_t hd, const int32_t* table, int64_t n_logical, const void* pool,
                                     int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
-                                    int n_splits, int keys_per_split, int32_t* status, cudaStream_t st) {
+                                    int n_splits, int keys_per_split, int32_t* status,
+                                    const int32_t* flags, long long flag_wait, cudaStream_t st) {
   if (!attention_decode_applies(n, hq, hkv, hd) || keys_per_split % 16 != 0 ||
       reinterpret_cast<uintptr_t>(pool) % 16 != 0)  // bulk copies start on 16-byte boundaries
     return cudaErrorInvalidValue;
@@ -421,7 +432,7 @@ cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64
 #define MZC_DEC_CASE(HDV, RV)                                                                              \
   if (hd == HDV && R == RV)                                                                                \
     return launch_dec<HDV, RV>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out, part_o, part_lse, \
-                               n_splits, bps, status, st);
+                               n_splits, bps, status, flags, flag_wait, st);
   MZC_DEC_CASE(64, 1)
   MZC_DEC_CASE(64, 2)
   MZC_DEC_CASE(64, 3)

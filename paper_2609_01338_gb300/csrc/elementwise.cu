@@ -43,8 +43,10 @@ __device__ __forceinline__ void unpack8_bf16(const uint4& v, float* f) {
 }
 
 // A value rounded to the KV storage precision (bf16 when !F16KV), encoded as
-// fp16: every normal-range bf16 value is exactly an fp16 value, so the pool
-// holds the stored values exactly while the attention reads one format.
+// fp16 so that the attention reads one format.  The encoding is exact for
+// bf16 values of magnitude 0 or in [2^-14, 65504]; below 2^-14 only fp16's
+// subnormal precision is kept, and from 65520 on the value becomes infinite
+// (the kernel then records MZC_ERR_OVERFLOW).
 template <bool F16KV>
 __device__ __forceinline__ float kv_round(float x) {
   if constexpr (F16KV) {
@@ -96,7 +98,7 @@ __global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t*
 
 // y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, fp16 out; one CTA per row.
 __global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ g, int d,
-                               float eps, uint16_t* __restrict__ y) {
+                               float eps, uint16_t* __restrict__ y, int32_t* status) {
   pdl_enter();
   __shared__ float red[32];
   const int64_t i = blockIdx.x;
@@ -110,12 +112,16 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, const float* __restr
   const float r = rsqrtf(ss / static_cast<float>(d) + eps);
   const float4* gr = reinterpret_cast<const float4*>(g);
   uint4* yr = reinterpret_cast<uint4*>(y + i * d);
+  float amax = 0.0f;
   for (int c = threadIdx.x; c < d / 8; c += blockDim.x) {
     float4 a = xr[2 * c], b = xr[2 * c + 1], ga = gr[2 * c], gb = gr[2 * c + 1];
     float f[8] = {a.x * r * ga.x, a.y * r * ga.y, a.z * r * ga.z, a.w * r * ga.w,
                   b.x * r * gb.x, b.y * r * gb.y, b.z * r * gb.z, b.w * r * gb.w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(f[e]));
     yr[c] = pack8<true>(f);
   }
+  note_f16_overflow(status, amax);
 }
 
 // The same RMSNorm, one warp per row with the row held in registers (read
@@ -127,7 +133,8 @@ constexpr int kRowVecs = 16;  // 8-float groups per lane: d <= 4096
 template <int G>
 __global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_warp_kernel(const float* __restrict__ x,
                                                            const float* __restrict__ g, int64_t n,
-                                                           float eps, uint16_t* __restrict__ y) {
+                                                           float eps, uint16_t* __restrict__ y,
+                                                           int32_t* status) {
   pdl_enter();
   constexpr int d = 256 * G;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
@@ -151,20 +158,25 @@ __global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_w
   const float r = rsqrtf(ss / static_cast<float>(d) + eps);
   const float4* gr = reinterpret_cast<const float4*>(g);
   uint4* yr = reinterpret_cast<uint4*>(y + i * d);
+  float amax = 0.0f;
 #pragma unroll
   for (int k = 0; k < G; ++k) {
     const int c = k * 32 + lane;
     const float4 ga = gr[2 * c], gb = gr[2 * c + 1];
     float f[8] = {a[k].x * r * ga.x, a[k].y * r * ga.y, a[k].z * r * ga.z, a[k].w * r * ga.w,
                   b[k].x * r * gb.x, b[k].y * r * gb.y, b[k].z * r * gb.z, b[k].w * r * gb.w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(f[e]));
     yr[c] = pack8<true>(f);
   }
+  note_f16_overflow(status, amax);  // the whole warp holds this row
 }
 
 template <int G>
 void launch_rmsnorm_warp(const float* x, const float* g, int64_t n, float eps, uint16_t* y,
-                         cudaStream_t st) {
-  launch_k(rmsnorm_warp_kernel<G>, dim3(static_cast<unsigned>((n + 7) / 8)), dim3(256), 0, st, x, g, n, eps, y);
+                         int32_t* status, cudaStream_t st) {
+  launch_k(rmsnorm_warp_kernel<G>, dim3(static_cast<unsigned>((n + 7) / 8)), dim3(256), 0, st, x, g, n, eps, y,
+           status);
 }
 
 // Rotary embedding (pairs (i, i + hd/2), angle pos * theta^(-2i/hd) from the
@@ -201,6 +213,7 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
   const int n_v = hkv * (hd / 8);
   const float* cs = cos_t + static_cast<int64_t>(p) * half;
   const float* sn = sin_t + static_cast<int64_t>(p) * half;
+  float amax = 0.0f;  // largest |value| this thread stores fp16-encoded
   for (int w = threadIdx.x; w < n_rot + n_v; w += blockDim.x) {
     if (w < n_rot) {
       const int head = w / rot_chunks, c = (w % rot_chunks) * 8;
@@ -231,6 +244,8 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
           y2[j] = kv_round<F16KV>(y2[j]);
         }
       }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) amax = fmaxf(amax, fmaxf(fabsf(y1[j]), fabsf(y2[j])));
       *reinterpret_cast<uint4*>(dst + c) = pack8<true>(y1);
       *reinterpret_cast<uint4*>(dst + c + half) = pack8<true>(y2);
     } else {
@@ -244,12 +259,16 @@ __global__ void rope_kv_kernel(const uint16_t* __restrict__ qkv, const int32_t* 
         float f[8];
         unpack8_f16(raw, f);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) f[j] = kv_round<false>(f[j]);
+        for (int j = 0; j < 8; ++j) {
+          f[j] = kv_round<false>(f[j]);
+          amax = fmaxf(amax, fabsf(f[j]));
+        }
         raw = pack8<true>(f);
       }
       *reinterpret_cast<uint4*>(dst) = raw;
     }
   }
+  note_f16_overflow(status, amax);
 }
 
 // logits[v] = sum_k h[k] * W[v][k], h = RMSNorm(x_row) * g kept in fp32.
@@ -357,12 +376,12 @@ cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed
 }
 
 cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
-                           uint16_t* y, cudaStream_t st) {
+                           uint16_t* y, cudaStream_t st, int32_t* status) {
   if (n <= 0) return cudaSuccess;
   switch (d % 256 == 0 ? d / 256 : 0) {
 #define MZC_RMS_CASE(G)                         \
   case G:                                       \
-    launch_rmsnorm_warp<G>(x, g, n, eps, y, st); \
+    launch_rmsnorm_warp<G>(x, g, n, eps, y, status, st); \
     break;
     MZC_RMS_CASE(1)
     MZC_RMS_CASE(2)
@@ -382,7 +401,7 @@ cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d,
     MZC_RMS_CASE(16)
 #undef MZC_RMS_CASE
     default:
-      launch_k(rmsnorm_kernel, dim3(static_cast<unsigned>(n)), dim3(256), 0, st, x, g, d, eps, y);
+      launch_k(rmsnorm_kernel, dim3(static_cast<unsigned>(n)), dim3(256), 0, st, x, g, d, eps, y, status);
   }
   static_assert(kRowVecs == 16, "warp kernel instances for d = 256 .. 4096");
   return cudaGetLastError();

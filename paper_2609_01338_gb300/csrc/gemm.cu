@@ -205,6 +205,7 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     };
     int local = 0;
     bool ok = true;
+    float amax = 0.0f;  // largest |value| this lane stores as fp16
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
       const int a = local & 1;
       ok = ok && pwait(&acc_full[a], (local >> 1) & 1, status, abort_flag);
@@ -226,8 +227,11 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
             tmem_ld32w(trow + g * 2 * kSwigluGroup + c, vg);
             tmem_ld32w(trow + g * 2 * kSwigluGroup + kSwigluGroup + c, vu);
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-              pk[c / 2 + i] = pack2<true>(silu_f(vg[2 * i]) * vu[2 * i], silu_f(vg[2 * i + 1]) * vu[2 * i + 1]);
+            for (int i = 0; i < 16; ++i) {
+              const float y0 = silu_f(vg[2 * i]) * vu[2 * i], y1 = silu_f(vg[2 * i + 1]) * vu[2 * i + 1];
+              amax = fmaxf(amax, fmaxf(fabsf(y0), fabsf(y1)));
+              pk[c / 2 + i] = pack2<true>(y0, y1);
+            }
           }
           uint8_t* box = stage_row(pk);
           if (lane == 0) {
@@ -246,7 +250,10 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
             float v[32];
             tmem_ld32w(trow + c + h, v);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) pk[h / 2 + i] = pack2<true>(v[2 * i], v[2 * i + 1]);
+            for (int i = 0; i < 16; ++i) {
+              amax = fmaxf(amax, fmaxf(fabsf(v[2 * i]), fabsf(v[2 * i + 1])));
+              pk[h / 2 + i] = pack2<true>(v[2 * i], v[2 * i + 1]);
+            }
           }
           uint8_t* box = stage_row(pk);
           if (lane == 0) {
@@ -275,6 +282,7 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     // every store has finished reading shared memory and reached global memory
     if (lane == 0) bulk_wait_all();
     __syncwarp();
+    if constexpr (EPI != EPI_ADD_F32) note_f16_overflow(status, amax);
   }
 
   tc_fence_before();
@@ -405,7 +413,7 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
                         const uint16_t* a_ptr) {
   if (m <= 0) return cudaSuccess;
   if (a_ptr && w.ptr && m <= kGemvMaxRows)
-    return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, st);
+    return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, status, st);
   if (m <= 256) {
     // weight-streaming bound with few N tiles: split K over a cluster
     static int sms = 0;

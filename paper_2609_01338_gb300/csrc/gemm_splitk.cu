@@ -233,6 +233,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const int t = threadIdx.x - 64;  // 0 .. 127
     const uint32_t part = smem_u32(smem);
     constexpr int CH = EPI == EPI_SWIGLU_BF16 ? 16 : 32;  // float4 chunks handled per row
+    float amax = 0.0f;  // largest |value| this thread stores as fp16
     for (int idx = t; idx < (r_end - r_begin) * CH; idx += 128) {
       const int r = r_begin + idx / CH, c = idx % CH;
       // all S loads are issued before the sum, which then runs in split order
@@ -262,9 +263,11 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
       }
       if constexpr (EPI == EPI_STORE_BF16) {
         const int col = nt * SBN + c * 4;
-        if (col < n)
+        if (col < n) {
+          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(acc.x), fabsf(acc.y)), fmaxf(fabsf(acc.z), fabsf(acc.w))));
           *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * n + col) =
               pack4_f16(acc.x, acc.y, acc.z, acc.w);
+        }
       } else if constexpr (EPI == EPI_ADD_F32) {
         const int col = nt * SBN + c * 4;
         if (col < n) {
@@ -279,12 +282,16 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
       } else {
         // gate columns 0..63 of the tile pair with up columns 64..127
         const int col = nt * (SBN / 2) + c * 4;
-        if (col < n / 2)
+        if (col < n / 2) {
+          const float y0 = silu_s(acc.x) * acc2.x, y1 = silu_s(acc.y) * acc2.y;
+          const float y2 = silu_s(acc.z) * acc2.z, y3 = silu_s(acc.w) * acc2.w;
+          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(y0), fabsf(y1)), fmaxf(fabsf(y2), fabsf(y3))));
           *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * (n / 2) + col) =
-              pack4_f16(silu_s(acc.x) * acc2.x, silu_s(acc.y) * acc2.y, silu_s(acc.z) * acc2.z,
-                        silu_s(acc.w) * acc2.w);
+              pack4_f16(y0, y1, y2, y3);
+        }
       }
     }
+    if constexpr (EPI != EPI_ADD_F32) note_f16_overflow(status, amax);
   }
 
   // ---- no CTA leaves while another may still read its partial ----

@@ -47,7 +47,8 @@ __device__ __forceinline__ float silu_g(float g) { return g / (1.0f + __expf(-g)
 template <int EPI, int MR, int KS>
 __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ a,
                                                    const uint16_t* __restrict__ w,
-                                                   void* __restrict__ out, int m, int n, int k) {
+                                                   void* __restrict__ out, int m, int n, int k,
+                                                   int32_t* status) {
   pdl_enter();
   constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
   constexpr int OUTS = 8 / KS;  // outputs per CTA
@@ -128,23 +129,25 @@ __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ 
   for (int i = 0; i < MR; ++i) {
     if (i >= m) break;
     if constexpr (EPI == EPI_STORE_BF16) {
+      if (fabsf(acc[0][i]) >= kF16Overflow) set_status(status, kStatusOverflow);
       static_cast<__half*>(out)[static_cast<int64_t>(i) * n + j] = __float2half_rn(acc[0][i]);
     } else if constexpr (EPI == EPI_ADD_F32) {
       static_cast<float*>(out)[static_cast<int64_t>(i) * n + j] += acc[0][i];
     } else {
-      static_cast<__half*>(out)[static_cast<int64_t>(i) * n_out + j] =
-          __float2half_rn(silu_g(acc[0][i]) * acc[1][i]);
+      const float y = silu_g(acc[0][i]) * acc[1][i];
+      if (fabsf(y) >= kF16Overflow) set_status(status, kStatusOverflow);
+      static_cast<__half*>(out)[static_cast<int64_t>(i) * n_out + j] = __float2half_rn(y);
     }
   }
 }
 
 template <int EPI, int MR, int KS>
 cudaError_t launch_mrk(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                       int64_t k, cudaStream_t st) {
+                       int64_t k, int32_t* status, cudaStream_t st) {
   const int64_t n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
   constexpr int OUTS = 8 / KS;
   launch_k(gemv_kernel<EPI, MR, KS>, dim3(static_cast<unsigned>((n_out + OUTS - 1) / OUTS)), dim3(256), 0, st,
-           a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k));
+           a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
   return cudaGetLastError();
 }
 
@@ -153,32 +156,33 @@ cudaError_t launch_mrk(const uint16_t* a, const uint16_t* w, void* out, int64_t 
 // rows measured 2.64).
 template <int EPI, int MR>
 cudaError_t launch_mr(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                      int64_t k, cudaStream_t st) {
+                      int64_t k, int32_t* status, cudaStream_t st) {
   constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
   const int64_t bytes = k * 2 * R;  // weight bytes of one output
-  if (bytes >= 6144) return launch_mrk<EPI, MR, 2>(a, w, out, m, n, k, st);
-  return launch_mrk<EPI, MR, 1>(a, w, out, m, n, k, st);
+  if (bytes >= 6144) return launch_mrk<EPI, MR, 2>(a, w, out, m, n, k, status, st);
+  return launch_mrk<EPI, MR, 1>(a, w, out, m, n, k, status, st);
 }
 
 template <int EPI>
 cudaError_t launch_epi(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                       int64_t k, cudaStream_t st) {
-  return m == 1 ? launch_mr<EPI, 1>(a, w, out, m, n, k, st) : launch_mr<EPI, 4>(a, w, out, m, n, k, st);
+                       int64_t k, int32_t* status, cudaStream_t st) {
+  return m == 1 ? launch_mr<EPI, 1>(a, w, out, m, n, k, status, st)
+                : launch_mr<EPI, 4>(a, w, out, m, n, k, status, st);
 }
 
 }  // namespace
 
 cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                        int64_t k, int epilogue, cudaStream_t st) {
+                        int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
   if (m <= 0) return cudaSuccess;
   if (m > kGemvMaxRows || k % 8 != 0) return cudaErrorInvalidValue;
   switch (epilogue) {
     case EPI_STORE_BF16:
-      return launch_epi<EPI_STORE_BF16>(a, w, out, m, n, k, st);
+      return launch_epi<EPI_STORE_BF16>(a, w, out, m, n, k, status, st);
     case EPI_ADD_F32:
-      return launch_epi<EPI_ADD_F32>(a, w, out, m, n, k, st);
+      return launch_epi<EPI_ADD_F32>(a, w, out, m, n, k, status, st);
     case EPI_SWIGLU_BF16:
-      return launch_epi<EPI_SWIGLU_BF16>(a, w, out, m, n, k, st);
+      return launch_epi<EPI_SWIGLU_BF16>(a, w, out, m, n, k, status, st);
     default:
       return cudaErrorInvalidValue;
   }

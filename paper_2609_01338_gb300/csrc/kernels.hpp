@@ -68,7 +68,7 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
 // when it is given the activation pointer.
 constexpr int kGemvMaxRows = 4;
 cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                        int64_t k, int epilogue, cudaStream_t st);
+                        int64_t k, int epilogue, int32_t* status, cudaStream_t st);
 
 // 8-bit swap codec (codec.cu).  block_elems = 2 * hkv * 16 * hd.
 int64_t q8_block_bytes(int64_t block_elems);
@@ -84,7 +84,7 @@ cudaError_t launch_wait_probe(int32_t arrive, int64_t limit_cycles, int32_t* sta
 cudaError_t launch_embed(const int32_t* tokens, int64_t n, const uint16_t* embed, int32_t d,
                          int64_t vocab, float* x, int32_t* status, cudaStream_t st);
 cudaError_t launch_rmsnorm(const float* x, const float* g, int64_t n, int32_t d, float eps,
-                           uint16_t* y, cudaStream_t st);
+                           uint16_t* y, cudaStream_t st, int32_t* status = nullptr);
 cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_t n, int32_t hq,
                                  int32_t hkv, int32_t hd, const float* cos_t, const float* sin_t,
                                  const int32_t* table, int64_t n_logical, void* pool,
@@ -107,12 +107,17 @@ void attention_decode_split(int32_t hkv, int64_t max_keys, int num_sms, int* n_s
 cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
                                     int32_t hd, const int32_t* table, int64_t n_logical, const void* pool,
                                     int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
-                                    int n_splits, int keys_per_split, int32_t* status, cudaStream_t st);
+                                    int n_splits, int keys_per_split, int32_t* status,
+                                    const int32_t* flags, long long flag_wait, cudaStream_t st);
+// flags (may be null): int32 per physical block, non-zero once the block's
+// data is in HBM; the kernels wait (bounded by flag_wait_cycles, 0 = the
+// default limit) for the flag of every block they read before fetching it.
 cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
                              int32_t hkv, int32_t hd, const int32_t* table, int64_t n_logical,
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,
                              uint16_t* out, void* scratch, int64_t scratch_bytes,
-                             int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st);
+                             int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st,
+                             const int32_t* flags = nullptr, int64_t flag_wait_cycles = 0);
 // Attention whose split-KV partials use a fixed array inside the library
 // (kAttnNoallocScratchBytes) instead of caller memory; no allocation.
 constexpr int64_t kAttnNoallocScratchBytes = 8LL << 20;

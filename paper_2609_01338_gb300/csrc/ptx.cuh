@@ -16,6 +16,10 @@ namespace mzc {
 constexpr long long kWaitCycles = 4000000000LL;
 constexpr int kStatusTimeout = 6;  // MZC_ERR_TIMEOUT
 constexpr int kStatusDevice = 7;   // MZC_ERR_DEVICE
+constexpr int kStatusOverflow = 8; // MZC_ERR_OVERFLOW
+// The smallest magnitude that rounds to infinity in fp16 (round to nearest
+// even: 65504 + half an ulp of 32).
+constexpr float kF16Overflow = 65520.0f;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -23,6 +27,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 
 __device__ __forceinline__ void set_status(int32_t* status, int code) {
   if (status) atomicCAS(status, 0, code);
+}
+
+// Records MZC_ERR_OVERFLOW when any lane of the (fully active) warp is about
+// to store, or has stored, a value of magnitude >= 65520 as fp16.  amax is the
+// lane's running maximum of |value| (fmaxf, so NaN inputs are not counted).
+__device__ __forceinline__ void note_f16_overflow(int32_t* status, float amax) {
+  if (__any_sync(0xffffffffu, amax >= kF16Overflow) && (threadIdx.x & 31) == 0)
+    set_status(status, kStatusOverflow);
 }
 
 // ---- mbarrier -------------------------------------------------------------
@@ -62,6 +74,41 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
+    if (clock64() - t0 > limit) {
+      set_status(status, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
+// ---- per-block residency flags (restore copies in flight) ----------------
+// A flag word per physical KV block: non-zero once the block's data is in
+// HBM.  The copy engine writes the flag after the block's data on the same
+// stream; a reader that sees it non-zero with an acquire load at GPU scope
+// sees the data, and a proxy fence then orders its TMA / bulk-copy reads
+// (async proxy) after that observation.
+__device__ __forceinline__ int32_t ld_acquire_gpu(const int32_t* p) {
+  int32_t v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Bounded wait until flags[p] is non-zero; false (MZC_ERR_TIMEOUT recorded)
+// when `limit` cycles pass first, or at once when the status word already
+// holds a timeout (another wait gave up: a missing flag is not waited for
+// once per block).
+__device__ __forceinline__ bool flag_wait(const int32_t* flags, int64_t p, int32_t* status,
+                                          long long limit) {
+  if (ld_acquire_gpu(flags + p) != 0) return true;
+  const long long t0 = clock64();
+  while (true) {
+    __nanosleep(128);
+    if (ld_acquire_gpu(flags + p) != 0) return true;
+    if (status != nullptr && *reinterpret_cast<volatile int32_t*>(status) == kStatusTimeout) return false;
     if (clock64() - t0 > limit) {
       set_status(status, kStatusTimeout);
       return false;

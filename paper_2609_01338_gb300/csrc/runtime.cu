@@ -102,6 +102,14 @@ struct mzc_ctx {
   uint8_t* d_rstage[2] = {nullptr, nullptr};
   cudaEvent_t ev_t0 = nullptr, ev_t1 = nullptr, ev_c0 = nullptr, ev_c1 = nullptr,
               ev_l0 = nullptr, ev_l1 = nullptr;
+  // streams passed in through mzc_options belong to the caller
+  bool own_cs = true, own_xs = true;
+  // MZC_WAIT_BLOCK_FLAG: a residency flag per physical block (non-zero = data
+  // present), cleared for a restore's destination blocks on the compute
+  // stream and set by the copy engine after each copied run (from h_ones)
+  int32_t* d_flags = nullptr;
+  int32_t* h_ones = nullptr;
+  cudaEvent_t ev_clear = nullptr;
   bool restore_issued = false, lm_timed = false, ttft_from_copy = false;
   // per-class launch counts and optional CUDA-event timing
   int32_t ktime_mask = 0;
@@ -151,10 +159,10 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
                  ctx->d_cos,     ctx->d_sin,   ctx->d_x,       ctx->d_h,       ctx->d_qkv,
                  ctx->d_q,       ctx->d_attn,  ctx->d_act,     ctx->d_meta,    ctx->d_logits,
                  ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list,
-                 ctx->d_rstage[0], ctx->d_rstage[1]};
+                 ctx->d_rstage[0], ctx->d_rstage[1], ctx->d_flags};
   for (void* p : dev)
     if (p) cudaFree(p);
-  void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging};
+  void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging, ctx->h_ones};
   for (void* p : host)
     if (p) cudaFreeHost(p);
   for (auto e : ctx->ev_pool) cudaEventDestroy(e);
@@ -162,11 +170,12 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
   for (auto e : ctx->ev_w) cudaEventDestroy(e);
   for (auto e : ctx->ev_h2d) cudaEventDestroy(e);
   for (auto e : ctx->ev_dec) cudaEventDestroy(e);
-  cudaEvent_t evs[] = {ctx->ev_t0, ctx->ev_t1, ctx->ev_c0, ctx->ev_c1, ctx->ev_l0, ctx->ev_l1};
+  cudaEvent_t evs[] = {ctx->ev_t0, ctx->ev_t1, ctx->ev_c0, ctx->ev_c1, ctx->ev_l0, ctx->ev_l1,
+                       ctx->ev_clear};
   for (auto e : evs)
     if (e) cudaEventDestroy(e);
-  if (ctx->cs) cudaStreamDestroy(ctx->cs);
-  if (ctx->xs) cudaStreamDestroy(ctx->xs);
+  if (ctx->cs && ctx->own_cs) cudaStreamDestroy(ctx->cs);
+  if (ctx->xs && ctx->own_xs) cudaStreamDestroy(ctx->xs);
   if (ctx->ds) cudaStreamDestroy(ctx->ds);
   delete ctx;
   return MZC_OK;
@@ -228,6 +237,14 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
     return ctx->fail(MZC_ERR_INVALID, "n_q_heads*head_dim must be a multiple of 64");
   if (ctx->opt.swap_codec != MZC_CODEC_NONE && ctx->opt.swap_codec != MZC_CODEC_Q8)
     return ctx->fail(MZC_ERR_INVALID, "unknown swap_codec");
+  if (ctx->opt.wait_mode != MZC_WAIT_LAYER_EVENT && ctx->opt.wait_mode != MZC_WAIT_BLOCK_FLAG)
+    return ctx->fail(MZC_ERR_INVALID, "unknown wait_mode");
+  // with the 8-bit store, kernels (not the copy engine) write the restored
+  // blocks; a flag they set could wait behind attention CTAs that spin on it
+  if (ctx->opt.wait_mode == MZC_WAIT_BLOCK_FLAG && ctx->opt.swap_codec != MZC_CODEC_NONE)
+    return ctx->fail(MZC_ERR_INVALID, "MZC_WAIT_BLOCK_FLAG needs swap_codec MZC_CODEC_NONE");
+  if (ctx->opt.debug_checks != 0 && ctx->opt.debug_checks != 1)
+    return ctx->fail(MZC_ERR_INVALID, "debug_checks must be 0 or 1");
   ctx->codec = ctx->opt.swap_codec;
   {
     const int64_t block_elems = 2LL * s.n_kv_heads * 16 * s.head_dim;
@@ -248,8 +265,18 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   ctx->block_bytes = ctx->st.block_bytes();
   const int64_t R = ctx->max_rows, F2 = 2 * ctx->f_pad;
 
-  CK(cudaStreamCreateWithFlags(&ctx->cs, cudaStreamNonBlocking));
-  CK(cudaStreamCreateWithFlags(&ctx->xs, cudaStreamNonBlocking));
+  if (ctx->opt.compute_stream) {
+    ctx->cs = static_cast<cudaStream_t>(ctx->opt.compute_stream);
+    ctx->own_cs = false;
+  } else {
+    CK(cudaStreamCreateWithFlags(&ctx->cs, cudaStreamNonBlocking));
+  }
+  if (ctx->opt.copy_stream) {
+    ctx->xs = static_cast<cudaStream_t>(ctx->opt.copy_stream);
+    ctx->own_xs = false;
+  } else {
+    CK(cudaStreamCreateWithFlags(&ctx->xs, cudaStreamNonBlocking));
+  }
   if (ctx->codec != MZC_CODEC_NONE) {
     CK(cudaStreamCreateWithFlags(&ctx->ds, cudaStreamNonBlocking));
     ctx->ev_h2d.assign(L, nullptr);
@@ -373,7 +400,32 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   CK(cudaMalloc(&ctx->d_list, L * ctx->nblk * 4));
   CK(cudaHostAlloc(&ctx->h_list, L * ctx->nblk * 4, cudaHostAllocDefault));
   CK(cudaHostAlloc(&ctx->h_staging, ctx->nblk * ctx->block_bytes, cudaHostAllocDefault));
+  if (ctx->opt.wait_mode == MZC_WAIT_BLOCK_FLAG) {
+    CK(cudaMalloc(&ctx->d_flags, ctx->st.pool_blocks() * 4));
+    CK(cudaMemset(ctx->d_flags, 1, ctx->st.pool_blocks() * 4));  // every block present
+    CK(cudaHostAlloc(&ctx->h_ones, ctx->nblk * 4, cudaHostAllocDefault));
+    for (int64_t i = 0; i < ctx->nblk; ++i) ctx->h_ones[i] = 1;
+    CK(cudaEventCreateWithFlags(&ctx->ev_clear, cudaEventDisableTiming));
+  }
   CK(cudaDeviceSynchronize());
+  return MZC_OK;
+}
+
+// debug_checks: every resident or in-flight (layer, block) maps to a physical
+// block inside the pool, and no two map to the same one.
+mzc_status debug_check_tables(mzc_ctx* ctx) {
+  std::vector<uint8_t> used(static_cast<size_t>(ctx->st.pool_blocks()), 0);
+  for (int32_t l = 0; l < ctx->shape.n_layers; ++l)
+    for (int64_t b = 0; b < ctx->nblk; ++b) {
+      const mzc::BlockEntry& e = ctx->st.at(l, b);
+      if (e.phys < 0) continue;
+      if (e.phys >= ctx->st.pool_blocks())
+        return ctx->fail(MZC_ERR_STATE, "debug check: layer " + std::to_string(l) + " block " +
+                                            std::to_string(b) + " maps outside the pool");
+      if (used[e.phys]++)
+        return ctx->fail(MZC_ERR_STATE, "debug check: physical block " + std::to_string(e.phys) +
+                                            " is mapped twice");
+    }
   return MZC_OK;
 }
 
@@ -419,14 +471,15 @@ mzc_status ensure_store(mzc_ctx* ctx) {
   return MZC_OK;
 }
 
-mzc_status check_status(mzc_ctx* ctx) {
+mzc_status check_status(mzc_ctx* ctx, const std::string& where = std::string()) {
   int32_t s = 0;
   CK(cudaMemcpy(&s, ctx->d_status, 4, cudaMemcpyDeviceToHost));
   if (s != 0) {
     CK(cudaMemset(ctx->d_status, 0, 4));
-    return ctx->fail(static_cast<mzc_status>(s), s == MZC_ERR_TIMEOUT
-                                                     ? "a device wait timed out"
-                                                     : "a device bounds check failed");
+    const char* what = s == MZC_ERR_TIMEOUT    ? "a device wait timed out"
+                       : s == MZC_ERR_OVERFLOW ? "an fp16 activation or K/V value overflowed (|x| >= 65520)"
+                                               : "a device bounds check failed";
+    return ctx->fail(static_cast<mzc_status>(s), where + what);
   }
   return MZC_OK;
 }
@@ -469,6 +522,16 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
   mzc::PrefillPlan P;
   mzc_status ss = ctx->st.prepare_prefill(n, ctx->max_rows, &P);
   if (ss != MZC_OK) return ctx->from_state(ss);
+  if (ctx->opt.debug_checks) {
+    mzc_status e = debug_check_tables(ctx);
+    if (e != MZC_OK) {
+      ctx->st.abort_prefill(P);
+      return e;
+    }
+  }
+  // per-block waits: the attention reads a block once its flag is set, so no
+  // layer event is waited on for the keys a restore copies in
+  const int32_t* flags = (ctx->d_flags && ctx->opt.overlap && ctx->restore_issued) ? ctx->d_flags : nullptr;
   const int64_t nrec = P.rec_end - P.rec_begin, rows = nrec + n;
   if (rows == 0) {
     ctx->st.complete(0);
@@ -552,7 +615,8 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
                      });
     };
     // attention of chunk rows [r0, r0 + nr) (r0 relative to the chunk)
-    auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab) {
+    auto attention = [&](int64_t r0, int64_t nr, int64_t mk, const int32_t* ltab,
+                         const int32_t* wait_flags = nullptr) {
       double fl, by;
       attn_work(c0 + r0, nr, &fl, &by);
       int sp = 1, per = 0;
@@ -562,7 +626,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         return mzc::launch_attention(ctx->d_q + r0 * hq * hd, cpos + r0, nr, s.n_q_heads, s.n_kv_heads,
                                      s.head_dim, ltab, ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(),
                                      s.kv_dtype, ctx->d_attn + r0 * hq * hd, ctx->d_scratch,
-                                     ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs);
+                                     ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs, wait_flags);
       });
     };
     const double norm_bytes = R * dd * 6.0 + dd * 4.0;
@@ -572,7 +636,8 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       const int32_t* ltab = dtab + l * ctx->nblk;
       if (P.w_wait[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_w[l], 0));
       CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-        return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+        return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
+                                   ctx->d_status);
       }));
       CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
       if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
@@ -583,7 +648,9 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       }));
       const bool wait_rec = n_rec_c > 0 && P.kv_wait_rec[l];
       const bool wait_prm = n_prm_c > 0 && P.kv_wait_prompt[l];
-      if (n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
+      if (flags && (wait_rec || wait_prm)) {
+        CKP(attention(0, cr, max_keys, ltab, flags));
+      } else if (n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
         // recompute rows read only resident keys: they run before the copy lands
         CKP(attention(0, n_rec_c, static_cast<int64_t>(hpos[c0 + n_rec_c - 1]) + 1, ltab));
         CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
@@ -594,10 +661,18 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       }
       CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
       CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-        return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs);
+        return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
+                                   ctx->d_status);
       }));
       CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
       CKP(gemm(ctx->tm_act, ctx->d_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
+      if (ctx->opt.debug_checks) {
+        // name the first layer whose kernels recorded a device error
+        CKP(cudaStreamSynchronize(cs));
+        mzc_status e = check_status(ctx, "layer " + std::to_string(l) + " (rows " + std::to_string(c0) +
+                                             ".." + std::to_string(c1) + "): ");
+        if (e != MZC_OK) return bail(e);
+      }
     }
     last_rows = cr;
   }
@@ -816,6 +891,16 @@ mzc_status mzc_restore_async(mzc_ctx* ctx) {
   if (!ctx->st.restore_in_flight()) return MZC_OK;
   cudaStream_t xs = ctx->xs;
   CK(cudaEventRecord(ctx->ev_c0, xs));
+  // per-block flags: the destination blocks read as absent from here on (their
+  // flags are cleared on the compute stream, ahead of any attention of the
+  // next prefill); the copy stream sets each run's flags after its data
+  const bool set_flags = ctx->d_flags && ctx->opt.overlap && ctx->codec == MZC_CODEC_NONE;
+  if (set_flags && !runs.empty()) {
+    for (const mzc_copy_run& r : runs)
+      CK(cudaMemsetAsync(ctx->d_flags + r.phys_begin, 0, static_cast<size_t>(r.n_blocks) * 4, ctx->cs));
+    CK(cudaEventRecord(ctx->ev_clear, ctx->cs));
+    CK(cudaStreamWaitEvent(xs, ctx->ev_clear, 0));
+  }
   size_t ri = 0, wi = 0;
   int64_t bytes = 0, copies = 0;
   for (int32_t l = 0; l < ctx->shape.n_layers; ++l) {
@@ -833,6 +918,9 @@ mzc_status mzc_restore_async(mzc_ctx* ctx) {
         const int64_t nb = static_cast<int64_t>(r.n_blocks) * ctx->block_bytes;
         CK(cudaMemcpyAsync(ctx->d_pool + r.phys_begin * ctx->block_bytes, ctx->h_store + r.host_off,
                            nb, cudaMemcpyHostToDevice, xs));
+        if (set_flags)
+          CK(cudaMemcpyAsync(ctx->d_flags + r.phys_begin, ctx->h_ones, static_cast<size_t>(r.n_blocks) * 4,
+                             cudaMemcpyHostToDevice, xs));
         bytes += nb;
         ++copies;
       }
@@ -1133,10 +1221,12 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
     const LayerDev& W = ctx->layers[0];
     const int64_t d = ctx->shape.d_model, hq = ctx->shape.n_q_heads, hd = ctx->shape.head_dim;
     auto layer_gemms = [&](int64_t m) -> cudaError_t {
-      cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, ctx->d_status, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_attn, W.tm_o, ctx->d_x, m, d, hq * hd, mzc::EPI_ADD_F32, ctx->d_status, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, ctx->d_status, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_act, W.tm_2, ctx->d_x, m, d, ctx->f_pad, mzc::EPI_ADD_F32, ctx->d_status, ctx->cs);
+      // (timing only: the activation buffers hold whatever the last prefill
+      // left, so the GEMMs report nothing to the status word)
+      cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, nullptr, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_attn, W.tm_o, ctx->d_x, m, d, hq * hd, mzc::EPI_ADD_F32, nullptr, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, nullptr, ctx->cs);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_act, W.tm_2, ctx->d_x, m, d, ctx->f_pad, mzc::EPI_ADD_F32, nullptr, ctx->cs);
       return e;
     };
     const int64_t sizes[3] = {128, 512, 2048};
@@ -1326,6 +1416,22 @@ mzc_status mzc_k_attention(const uint16_t* q, const int32_t* pos, int64_t n, int
   KCK(mzc::launch_attention(q, pos, n, hq, hkv, hd, block_table, n_logical, pool, pool_blocks,
                             kv_dtype, out, scratch, scratch_bytes, max_keys, sm_count(), status,
                             static_cast<cudaStream_t>(stream)));
+}
+
+mzc_status mzc_k_attention_wait(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
+                                int32_t hkv, int32_t hd, const int32_t* block_table, int64_t n_logical,
+                                const void* pool, int64_t pool_blocks, int32_t kv_dtype, uint16_t* out,
+                                int64_t max_keys, void* scratch, int64_t scratch_bytes,
+                                const int32_t* block_flags, int64_t flag_wait_cycles, int32_t* status,
+                                void* stream) {
+  if (!q || !pos || !block_table || !pool || !out || !block_flags || n < 0 || max_keys <= 0 ||
+      flag_wait_cycles < 0)
+    return MZC_ERR_INVALID;
+  if ((hd != 64 && hd != 128) || hkv <= 0 || hq % hkv != 0) return MZC_ERR_INVALID;
+  if (reinterpret_cast<uintptr_t>(pool) % 16 != 0) return MZC_ERR_INVALID;
+  KCK(mzc::launch_attention(q, pos, n, hq, hkv, hd, block_table, n_logical, pool, pool_blocks,
+                            kv_dtype, out, scratch, scratch_bytes, max_keys, sm_count(), status,
+                            static_cast<cudaStream_t>(stream), block_flags, flag_wait_cycles));
 }
 
 mzc_status mzc_k_attention_noalloc(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,

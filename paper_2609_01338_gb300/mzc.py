@@ -16,13 +16,15 @@ _lib = None
 
 MZC_OK, MZC_ERR_INVALID, MZC_ERR_RANGE, MZC_ERR_STATE = 0, 1, 2, 3
 MZC_ERR_OOM, MZC_ERR_CUDA, MZC_ERR_TIMEOUT, MZC_ERR_DEVICE = 4, 5, 6, 7
+MZC_ERR_OVERFLOW = 8
 MZC_KV_BF16, MZC_KV_FP16 = 0, 1
 MZC_CODEC_NONE, MZC_CODEC_Q8 = 0, 1
 MZC_COPY, MZC_DROP, MZC_AUTO = 0, 1, 2
 MZC_POLICY_COPY, MZC_POLICY_RECOMPUTE, MZC_POLICY_HYBRID = 0, 1, 2
 MZC_RESIDENT, MZC_SWAPPED, MZC_DROPPED, MZC_INFLIGHT, MZC_EMPTY = 0, 1, 2, 3, 4
+MZC_WAIT_LAYER_EVENT, MZC_WAIT_BLOCK_FLAG = 0, 1
 STATUS_NAMES = {0: "OK", 1: "INVALID", 2: "RANGE", 3: "STATE", 4: "OOM", 5: "CUDA",
-                6: "TIMEOUT", 7: "DEVICE"}
+                6: "TIMEOUT", 7: "DEVICE", 8: "OVERFLOW"}
 
 c_i32, c_i64, c_f32, c_f64, c_vp = (ctypes.c_int32, ctypes.c_int64, ctypes.c_float,
                                     ctypes.c_double, ctypes.c_void_p)
@@ -37,7 +39,9 @@ class mzc_model_shape(ctypes.Structure):
 
 class mzc_options(ctypes.Structure):
     _fields_ = [("pool_blocks", c_i64), ("max_rows", c_i64), ("host_store_bytes", c_i64),
-                ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32)]
+                ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32),
+                ("wait_mode", c_i32), ("debug_checks", c_i32), ("reserved", c_i32),
+                ("compute_stream", c_vp), ("copy_stream", c_vp)]
 
 
 class mzc_layer_weights(ctypes.Structure):
@@ -121,6 +125,8 @@ _SIGS = {
                         c_vp, c_i64, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_attention_noalloc": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64,
                                 c_i32, c_vp, c_i64, c_vp, c_vp],
+    "mzc_k_attention_wait": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_i64, c_vp, c_i64, c_i32,
+                             c_vp, c_i64, c_vp, c_i64, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
     "mzc_plan_split_ctx": [c_vp, c_i64, c_i64, c_vp],
     "mzc_k_wait_probe": [c_i32, c_i64, c_vp, c_vp, c_vp],
@@ -219,9 +225,13 @@ def make_weights(weights: dict):
 # ---- ctx entry points (same names as the C ABI) -------------------------
 
 def mzc_create(shape: dict, weights: dict, pool_blocks=0, max_rows=0, host_store_bytes=0,
-               overlap=1, device=0, swap_codec=MZC_CODEC_NONE):
+               overlap=1, device=0, swap_codec=MZC_CODEC_NONE, wait_mode=MZC_WAIT_LAYER_EVENT,
+               debug_checks=0, compute_stream=None, copy_stream=None):
+    """compute_stream / copy_stream: cudaStream_t handles (ints, e.g. a torch
+    stream's cuda_stream) owned by the caller, or None."""
     sh = make_shape(shape)
-    opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec)
+    opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec,
+                      wait_mode, debug_checks, 0, compute_stream, copy_stream)
     w, keep = make_weights(weights)
     out = c_vp()
     _call("mzc_create", ctypes.byref(sh), ctypes.byref(opt), ctypes.byref(w), ctypes.byref(out))
@@ -406,6 +416,15 @@ def mzc_k_attention(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks,
     return _call("mzc_k_attention", _ptr(q), _ptr(pos), n, hq, hkv, hd, _ptr(table), n_logical,
                  _ptr(pool), pool_blocks, kv_dtype, _ptr(out), max_keys, _ptr(scratch),
                  scratch_bytes, _ptr(status), stream)
+
+
+def mzc_k_attention_wait(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks, kv_dtype, out,
+                         max_keys, scratch, scratch_bytes, block_flags, flag_wait_cycles, status,
+                         stream=None):
+    """Attention that waits (bounded) for each block's residency flag."""
+    return _call("mzc_k_attention_wait", _ptr(q), _ptr(pos), n, hq, hkv, hd, _ptr(table), n_logical,
+                 _ptr(pool), pool_blocks, kv_dtype, _ptr(out), max_keys, _ptr(scratch),
+                 scratch_bytes, _ptr(block_flags), flag_wait_cycles, _ptr(status), stream)
 
 
 MZC_ATTENTION_NOALLOC_SCRATCH_BYTES = 8 << 20
