@@ -200,10 +200,12 @@ mzc_status mzc_prefill(mzc_ctx *ctx, const int32_t *tokens, int64_t n, float *lo
  * slightly more than asked at chunk granularity).  MZC_COPY swaps the blocks
  * to the pinned store (D2H, packed per layer) and frees their physical
  * blocks; MZC_DROP frees them for later recompute and is legal only across
- * all layers, with the dropped positions forming one contiguous range;
+ * all layers, with the dropped positions forming one contiguous range (it may
+ * also take SWAPPED blocks, whose host copies are then discarded);
  * MZC_AUTO splits [tok_begin, context_tokens) into a recomputed front and a
  * copied back by the ctx's policy (mzc_set_policy).  Every block in range
- * must be RESIDENT (else MZC_ERR_STATE, nothing changes).  With the
+ * must be RESIDENT (for DROP: RESIDENT or SWAPPED; else MZC_ERR_STATE,
+ * nothing changes).  With the
  * MZC_CODEC_Q8 option, copied blocks are quantized on the device before the
  * D2H copy, and restored blocks hold the decoded values (lossy; repeated
  * swaps give the same values again).  Synchronous. */
@@ -264,6 +266,68 @@ mzc_status mzc_plan_split_ctx(mzc_ctx *ctx, int64_t p, int64_t n_prompt, int64_t
  * Resident KV blocks, block tables and residency are unchanged.  Errors:
  * MZC_ERR_STATE while a restore is in flight or a recompute is pending. */
 mzc_status mzc_profile_measure(mzc_ctx *ctx, mzc_profile *out);
+
+/* Eviction policy: the paper's evict(size) (Sec. 5) driving its four-stage
+ * placement (Algorithm 1, Sec. 4.3), on this library's two restore paths:
+ * the host link (weights, and KV units evicted by COPY) and recompute (KV
+ * units evicted by DROP).  Units: a weight layer; a KV unit = one 16-token
+ * block of every layer (recompute regenerates all layers of a row at once).
+ * With q = floor(t_copy_w / t_rec_kv) and T = w_total * q:
+ *   MZC_STAGE_KV_ONLY   while more than T KV units remain: one unit at a
+ *                       time, to recompute if that path's total time with it
+ *                       stays strictly below the link's total time with it
+ *                       (link time counts evicted weights too), else to the
+ *                       link: the faster path takes more, in inverse
+ *                       proportion to the per-unit times;
+ *   MZC_STAGE_KV_AND_W  then, per step, one weight layer to the link and q KV
+ *                       units to recompute, so KV and weights run out together;
+ *   MZC_STAGE_W_ONLY    then the remaining weight layers;
+ *   MZC_STAGE_COMP_KV   nothing left to free on the device (the paper's last
+ *                       stage moves compressed KV to storage; no device memory
+ *                       is involved): the call stops.
+ * A step is never split, so slightly more than asked may be freed (as the
+ * paper's chunk granularity does, Sec. 6.2).
+ * Placement (backward-out, Sec. 4.4): recomputed units are the context's
+ * last kv_rec blocks of every layer, copied units the kv_copy blocks before
+ * them, evicted weights the last w_evicted layers.  As later calls add
+ * recompute units, the recomputed range grows backward over copied blocks
+ * (their host copies are discarded), so the placement stays balanced
+ * wherever eviction stops. */
+enum { MZC_STAGE_KV_ONLY = 1, MZC_STAGE_KV_AND_W = 2, MZC_STAGE_W_ONLY = 3, MZC_STAGE_COMP_KV = 4 };
+typedef struct {
+  double t_copy_w;   /* s: one layer's weights over the host link */
+  double t_copy_kv;  /* s: one KV unit over the host link */
+  double t_rec_kv;   /* s: one KV unit recomputed */
+  int64_t kv_total;  /* N_KV^total: KV units of the context, ceil(context / 16) */
+  int32_t w_total;   /* N_W^total: weight layers that may be evicted */
+  int32_t w_evicted; /* in/out: weight layers on the link path */
+  int64_t kv_copy;   /* in/out: KV units on the link path */
+  int64_t kv_rec;    /* in/out: KV units on the recompute path */
+  int64_t kv_bytes;  /* device bytes one KV unit frees */
+  int64_t w_bytes;   /* device bytes one weight layer frees */
+} mzc_evict_plan;
+
+/* Pure host arithmetic: advances plan's counts by Algorithm 1 until at least
+ * `bytes` are freed or nothing is left; *freed_out = bytes freed, *stage_out
+ * = the last stage taken (0 if bytes <= 0).  MZC_ERR_INVALID for negative
+ * times or counts, or counts beyond the totals. */
+mzc_status mzc_plan_evict_size(mzc_evict_plan *plan, int64_t bytes, int64_t *freed_out,
+                               int32_t *stage_out);
+/* evict(size) on this ctx: reads the current counts from the residency
+ * table (which must have the placement above: MZC_ERR_STATE otherwise, or
+ * while a restore or recompute is pending), takes the per-unit times from
+ * the ctx's profile (mzc_profile_measure or mzc_set_policy: t_copy_* = bytes
+ * / h2d rate; t_rec_kv = 16 rows through every layer at the profile's
+ * 2048-row projection rate and recompute attention rate over the whole
+ * context), plans, and evicts: COPY of the new copied blocks, DROP of the new
+ * recomputed range (over resident or swapped blocks), the new weight layers.
+ * After it, mzc_restore_async and mzc_recompute_tail(p, n) over the dropped
+ * range [p, context) restore everything.  Synchronous. */
+mzc_status mzc_evict_size(mzc_ctx *ctx, int64_t bytes, int64_t *freed_out, int32_t *stage_out);
+/* The plan mzc_evict_size starts from on this ctx: the current counts, the
+ * totals, the per-unit times and bytes (for a caller that wants to see or
+ * replay the policy's decision, e.g. with mzc_plan_evict_size).  Same errors. */
+mzc_status mzc_evict_size_plan(mzc_ctx *ctx, mzc_evict_plan *out);
 
 /* Shrinks the context to n_ctx positions (frees the blocks past it). */
 mzc_status mzc_truncate(mzc_ctx *ctx, int64_t n_ctx);
@@ -338,6 +402,11 @@ mzc_status mzc_state_evict(mzc_state *st, int32_t layer_begin, int32_t layer_end
                            int64_t tok_begin, int64_t tok_end, int32_t mode);
 mzc_status mzc_state_evict_blocks(mzc_state *st, const int32_t *layer,
                                   const int64_t *logical_block, int64_t n, int32_t mode);
+/* evict(size) on the bookkeeping alone (see mzc_evict_size), with the unit
+ * times and byte sizes from *times (its counts are ignored; the state's own
+ * are used). */
+mzc_status mzc_state_evict_size(mzc_state *st, const mzc_evict_plan *times, int64_t bytes,
+                                int64_t *freed_out, int32_t *stage_out);
 mzc_status mzc_state_recompute_tail(mzc_state *st, int64_t p, int64_t n);
 /* Plans the restore of every swapped block (forward-in); swapped blocks
  * become INFLIGHT.  Writes up to cap runs; *n_runs is the number planned

@@ -4,7 +4,9 @@ Per (layer, logical block): RESIDENT, SWAPPED, DROPPED, INFLIGHT or EMPTY,
 following the eviction/restore rules of the ABI: token ranges round outward
 to 16-token blocks (the paper evicts at chunk granularity, Sec. 4.2/6.2);
 COPY swaps resident blocks; DROP frees a contiguous token range across all
-layers for recompute; restore moves every swapped block to INFLIGHT; a
+layers for recompute, and may take swapped blocks too (their host copies are
+discarded: the eviction policy can move a unit from the copy path to the
+recompute path, Algorithm 1); restore moves every swapped block to INFLIGHT; a
 completed prefill makes in-flight and recomputed blocks RESIDENT and appends
 the prompt.  Physical block numbers are not modelled (any valid, distinct
 assignment is correct); the tests check them for validity only.
@@ -12,7 +14,8 @@ assignment is correct); the tests check them for validity only.
 Pinned by tests/test_oracle_state_pins.py: literal tables and status codes
 worked out by hand from the rules above (outward rounding, one contiguous
 all-layer DROP range, double eviction, prefill over dropped or swapped
-blocks, recompute range, truncation inside a dropped range).
+blocks, recompute range, truncation inside a dropped range, DROP over
+swapped blocks).
 """
 from __future__ import annotations
 
@@ -61,7 +64,8 @@ class StateModel:
         if self.inflight or self.pending:
             return STATE
         b0, b1 = t0 // 16, -(-t1 // 16)
-        if any(self.st[l][b] != RESIDENT for l in range(l0, l1) for b in range(b0, b1)):
+        allowed = (RESIDENT, SWAPPED) if mode == 1 else (RESIDENT,)
+        if any(self.st[l][b] not in allowed for l in range(l0, l1) for b in range(b0, b1)):
             return STATE
         if mode == 1:
             if l0 != 0 or l1 != self.L:

@@ -769,6 +769,16 @@ struct CostModel : CostModelShape {
     if (pre) *pre = g * qkv_frac + rec_attn + rw * (2.0 / 3.0) + fixed * 0.5;
     return g + rec_attn + prm_attn + rw + fixed;
   }
+  // one KV unit (16 rows, every layer) recomputed at the rear of an n_ctx
+  // context: the rows at the 2048-row projection rate, their attention over
+  // the whole context at the recompute rate, per-row kernels (the eviction
+  // policy's t_rec_kv, Algorithm 1)
+  double rec_unit_s(int64_t n_ctx) const {
+    const double per_row = gemm_s(2048.0) / 2048.0 +
+                           static_cast<double>(n_ctx) * attn_flops_pair / (p.attn_tflops * 1e12) +
+                           (p.attn_row_ns + p.row_ns) * 1e-9;
+    return 16.0 * per_row * s.n_layers;
+  }
   // predicted TTFT when [p0, s1) is recomputed and [s1, n_ctx) copied
   double ttft_s(int64_t p0, int64_t s1, int64_t n_ctx, int64_t n_prompt) const {
     double pre = 0.0;
@@ -1043,6 +1053,62 @@ mzc_status mzc_plan_split_ctx(mzc_ctx* ctx, int64_t p, int64_t n_prompt, int64_t
   mzc_status e = plan_split_impl(&ctx->shape, &pr, p, ctx->st.n_ctx(), n_prompt, raw ? 0.01 : 0.05,
                                  raw ? 0.95 : 1.0, s_out);
   return e == MZC_OK ? e : ctx->fail(e, "hybrid split failed");
+}
+
+mzc_status mzc_evict_size_plan(mzc_ctx* ctx, mzc_evict_plan* out) {
+  if (!ctx || !out) return MZC_ERR_INVALID;
+  const int32_t L = ctx->shape.n_layers;
+  int64_t c0 = 0, r0 = 0;
+  int32_t w0 = 0;
+  if (ctx->st.evicted_layout(&c0, &r0, &w0) != MZC_OK)
+    return ctx->fail(MZC_ERR_STATE, "evict_size needs the backward-out placement it makes (and no "
+                                    "restore or recompute pending)");
+  const double link = ctx->prof.h2d_gbs * 1e9;
+  if (!(link > 0)) return ctx->fail(MZC_ERR_INVALID, "the profile has no host-link rate");
+  mzc_evict_plan p{};
+  p.t_copy_w = static_cast<double>(ctx->layers[0].bytes) / link;
+  p.t_copy_kv = static_cast<double>(L) * static_cast<double>(ctx->slot_bytes) / link;
+  p.t_rec_kv = CostModel(ctx->shape, ctx->prof).rec_unit_s(ctx->st.n_ctx());
+  p.kv_total = ceil_div(ctx->st.n_ctx(), 16);
+  p.w_total = L;
+  p.w_evicted = w0;
+  p.kv_copy = c0;
+  p.kv_rec = r0;
+  p.kv_bytes = static_cast<int64_t>(L) * ctx->block_bytes;
+  p.w_bytes = static_cast<int64_t>(ctx->layers[0].bytes);
+  *out = p;
+  return MZC_OK;
+}
+
+mzc_status mzc_evict_size(mzc_ctx* ctx, int64_t bytes, int64_t* freed_out, int32_t* stage_out) {
+  if (!ctx) return MZC_ERR_INVALID;
+  const int32_t L = ctx->shape.n_layers;
+  mzc_evict_plan p{};
+  mzc_status e0 = mzc_evict_size_plan(ctx, &p);
+  if (e0 != MZC_OK) return e0;
+  const int64_t c0 = p.kv_copy, r0 = p.kv_rec;
+  const int32_t w0 = p.w_evicted;
+  int64_t freed = 0;
+  int32_t stage = 0;
+  mzc_status e = mzc_plan_evict_size(&p, bytes, &freed, &stage);
+  if (e != MZC_OK) return ctx->fail(e, "invalid eviction request");
+  mzc::EvictSizeSteps steps;
+  mzc::evict_size_steps(ctx->st.n_ctx(), L, c0, r0, w0, p, &steps);
+  if (steps.copy_t1 > steps.copy_t0) {
+    e = mzc_evict(ctx, 0, L, steps.copy_t0, steps.copy_t1, MZC_COPY);
+    if (e != MZC_OK) return e;
+  }
+  if (steps.drop_t1 > steps.drop_t0) {
+    e = mzc_evict(ctx, 0, L, steps.drop_t0, steps.drop_t1, MZC_DROP);
+    if (e != MZC_OK) return e;
+  }
+  if (steps.w1 > steps.w0) {
+    e = mzc_evict_weights(ctx, steps.w0, steps.w1);
+    if (e != MZC_OK) return e;
+  }
+  if (freed_out) *freed_out = freed;
+  if (stage_out) *stage_out = stage;
+  return MZC_OK;
 }
 
 mzc_status mzc_truncate(mzc_ctx* ctx, int64_t n_ctx) {

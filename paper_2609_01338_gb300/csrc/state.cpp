@@ -2,6 +2,7 @@
 #include "state.hpp"
 
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 
 namespace mzc {
@@ -130,11 +131,16 @@ mzc_status State::evict_range(int32_t l0, int32_t l1, int64_t t0, int64_t t1, in
   if (t0 < 0 || t1 > n_ctx_ || t0 >= t1) return fail(MZC_ERR_RANGE, "token range outside the context");
   if (inflight_ || rec_pending_) return fail(MZC_ERR_STATE, "a restore or recompute is pending");
   const int64_t b0 = t0 / 16, b1 = ceil_div(t1, 16);
+  // DROP may also take SWAPPED blocks (their host copies are discarded): the
+  // eviction policy can move a unit from the copy path to the recompute path
   for (int32_t l = l0; l < l1; ++l)
-    for (int64_t b = b0; b < b1; ++b)
-      if (at(l, b).st != MZC_RESIDENT)
-        return fail(MZC_ERR_STATE, "block " + std::to_string(b) + " of layer " +
-                                       std::to_string(l) + " is not resident");
+    for (int64_t b = b0; b < b1; ++b) {
+      const uint8_t st = at(l, b).st;
+      if (st != MZC_RESIDENT && !(mode == MZC_DROP && st == MZC_SWAPPED))
+        return fail(MZC_ERR_STATE, "block " + std::to_string(b) + " of layer " + std::to_string(l) +
+                                       (mode == MZC_DROP ? " is neither resident nor swapped"
+                                                         : " is not resident"));
+    }
   if (mode == MZC_DROP) {
     if (l0 != 0 || l1 != L)
       return fail(MZC_ERR_INVALID, "DROP must cover every layer (recompute regenerates all layers)");
@@ -144,7 +150,10 @@ mzc_status State::evict_range(int32_t l0, int32_t l1, int64_t t0, int64_t t1, in
     for (int32_t l = 0; l < L; ++l)
       for (int64_t b = b0; b < b1; ++b) {
         BlockEntry& e = at(l, b);
-        pool_.release(e.phys, 1);
+        if (e.st == MZC_SWAPPED)
+          drop_region_slot(e.region);
+        else
+          pool_.release(e.phys, 1);
         e = BlockEntry{};
         e.st = MZC_DROPPED;
       }
@@ -451,6 +460,94 @@ void State::counts(mzc_stats_t* o) const {
 void State::block_table(std::vector<int32_t>* out) const {
   out->resize(tab_.size());
   for (size_t i = 0; i < tab_.size(); ++i) (*out)[i] = tab_[i].phys;
+}
+
+// ---- eviction policy (Algorithm 1) -----------------------------------------
+
+int32_t plan_evict_size(mzc_evict_plan* p, int64_t bytes, int64_t* freed) {
+  const int64_t q = p->t_rec_kv > 0 ? static_cast<int64_t>(std::floor(p->t_copy_w / p->t_rec_kv)) : 0;
+  const int64_t T = static_cast<int64_t>(p->w_total) * q;
+  int64_t f = 0;
+  int32_t stage = 0;
+  while (f < bytes) {
+    const int64_t n_kv = p->kv_total - p->kv_copy - p->kv_rec;
+    const int64_t n_w = static_cast<int64_t>(p->w_total) - p->w_evicted;
+    if (n_kv > T) {  // KVonly: the unit to the path that stays faster with it (ties: link)
+      stage = MZC_STAGE_KV_ONLY;
+      const double rec = static_cast<double>(p->kv_rec + 1) * p->t_rec_kv;
+      const double link = static_cast<double>(p->kv_copy + 1) * p->t_copy_kv +
+                          static_cast<double>(p->w_evicted) * p->t_copy_w;
+      if (rec < link)
+        ++p->kv_rec;
+      else
+        ++p->kv_copy;
+      f += p->kv_bytes;
+    } else if (n_kv > 0 && n_w > 0) {  // KVandW: a layer, and q units to recompute
+      stage = MZC_STAGE_KV_AND_W;
+      const int64_t take = std::min(q, n_kv);
+      ++p->w_evicted;
+      p->kv_rec += take;
+      f += p->w_bytes + take * p->kv_bytes;
+    } else if (n_w > 0) {  // Wonly
+      stage = MZC_STAGE_W_ONLY;
+      ++p->w_evicted;
+      f += p->w_bytes;
+    } else {  // CompKV: nothing left to free on the device
+      stage = MZC_STAGE_COMP_KV;
+      break;
+    }
+  }
+  if (freed) *freed = f;
+  return stage;
+}
+
+mzc_status State::evicted_layout(int64_t* kv_copy, int64_t* kv_rec, int32_t* w_evicted) const {
+  if (inflight_ || rec_pending_) return MZC_ERR_STATE;
+  const int32_t L = shape_.n_layers;
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  auto column = [&](int64_t b) -> int {  // the state every layer shares, or -1
+    const uint8_t s0 = at(0, b).st;
+    for (int32_t l = 1; l < L; ++l)
+      if (at(l, b).st != s0) return -1;
+    return s0;
+  };
+  int64_t b = nb, rec = 0, copy = 0;
+  while (b > 0 && column(b - 1) == MZC_DROPPED) --b, ++rec;
+  while (b > 0 && column(b - 1) == MZC_SWAPPED) --b, ++copy;
+  for (int64_t c = 0; c < b; ++c)
+    if (column(c) != MZC_RESIDENT) return MZC_ERR_STATE;
+  int32_t w = 0;
+  while (w < L && w_state_[L - 1 - w] == MZC_SWAPPED) ++w;
+  for (int32_t l = 0; l < L - w; ++l)
+    if (w_state_[l] != MZC_RESIDENT) return MZC_ERR_STATE;
+  *kv_copy = copy;
+  *kv_rec = rec;
+  *w_evicted = w;
+  return MZC_OK;
+}
+
+void evict_size_steps(int64_t n_ctx, int32_t n_layers, int64_t c0, int64_t r0, int32_t w0,
+                      const mzc_evict_plan& p, EvictSizeSteps* out) {
+  const int64_t nb = ceil_div(n_ctx, 16);
+  const int64_t e0 = nb - r0 - c0;          // first evicted block before
+  const int64_t e1 = nb - p.kv_rec - p.kv_copy;  // ... after
+  const int64_t d0 = nb - r0;               // first dropped block before
+  const int64_t d1 = nb - p.kv_rec;         // ... after
+  EvictSizeSteps s;
+  // newly copied blocks: the resident ones in front of the old evicted range,
+  // minus any the new dropped range takes directly
+  const int64_t cb1 = std::min(e0, d1);
+  if (cb1 > e1) {
+    s.copy_t0 = e1 * 16;
+    s.copy_t1 = std::min(cb1 * 16, n_ctx);
+  }
+  if (d0 > d1) {
+    s.drop_t0 = d1 * 16;
+    s.drop_t1 = std::min(d0 * 16, n_ctx);
+  }
+  s.w0 = n_layers - p.w_evicted;
+  s.w1 = n_layers - w0;
+  *out = s;
 }
 
 }  // namespace mzc

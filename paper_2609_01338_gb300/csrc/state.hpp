@@ -124,6 +124,12 @@ class State {
   mzc_status truncate(int64_t n_ctx);
 
   int32_t weight_state(int32_t l) const { return w_state_[l]; }
+  // The evicted state as the eviction policy leaves it (backward-out): the
+  // last kv_rec blocks of every layer DROPPED, the kv_copy blocks before them
+  // SWAPPED in every layer, everything before RESIDENT, and the weights of
+  // the last w_evicted layers swapped.  MZC_ERR_STATE for any other shape, or
+  // while a restore or recompute is pending.
+  mzc_status evicted_layout(int64_t* kv_copy, int64_t* kv_rec, int32_t* w_evicted) const;
   // Longest run of free physical blocks (holds no live KV): length, start.
   int64_t largest_free_pool_run(int64_t* start) const { return pool_.largest_free(start); }
   void counts(mzc_stats_t* out) const;
@@ -151,5 +157,22 @@ class State {
 };
 
 int64_t ceil_div(int64_t a, int64_t b);
+
+// Algorithm 1's stages over the counts in *p (in/out) until at least `bytes`
+// are freed or nothing is left; returns the last stage taken (MZC_STAGE_*)
+// and the bytes freed in *freed.  Pure arithmetic.
+int32_t plan_evict_size(mzc_evict_plan* p, int64_t bytes, int64_t* freed);
+
+// The evictions that take a context of n_ctx positions from counts (c0, r0,
+// w0) to plan's counts, in this order: COPY of token range [copy_t0,
+// copy_t1) in every layer (blocks that were resident), DROP of [drop_t0,
+// drop_t1) in every layer (resident or swapped blocks, adjacent to the
+// dropped tail), weights of layers [w0, w1).  Empty ranges have t1 <= t0.
+struct EvictSizeSteps {
+  int64_t copy_t0 = 0, copy_t1 = 0, drop_t0 = 0, drop_t1 = 0;
+  int32_t w0 = 0, w1 = 0;
+};
+void evict_size_steps(int64_t n_ctx, int32_t n_layers, int64_t c0, int64_t r0, int32_t w0,
+                      const mzc_evict_plan& p, EvictSizeSteps* out);
 
 }  // namespace mzc

@@ -53,6 +53,63 @@ mzc_status mzc_state_evict_blocks(mzc_state* st, const int32_t* layer, const int
   return st->st.evict_blocks(layer, blk, n, mode, nullptr);
 }
 
+mzc_status mzc_plan_evict_size(mzc_evict_plan* plan, int64_t bytes, int64_t* freed_out,
+                               int32_t* stage_out) {
+  if (!plan) return MZC_ERR_INVALID;
+  const mzc_evict_plan& p = *plan;
+  if (!(p.t_copy_w >= 0) || !(p.t_copy_kv >= 0) || !(p.t_rec_kv >= 0) || p.kv_total < 0 ||
+      p.w_total < 0 || p.kv_copy < 0 || p.kv_rec < 0 || p.w_evicted < 0 ||
+      p.kv_copy + p.kv_rec > p.kv_total || p.w_evicted > p.w_total || p.kv_bytes < 0 || p.w_bytes < 0)
+    return MZC_ERR_INVALID;
+  // a step that frees no bytes would never end the loop
+  if (bytes > 0 && ((p.kv_total > p.kv_copy + p.kv_rec && p.kv_bytes <= 0) ||
+                    (p.w_total > p.w_evicted && p.w_bytes <= 0)))
+    return MZC_ERR_INVALID;
+  int64_t freed = 0;
+  const int32_t stage = mzc::plan_evict_size(plan, bytes, &freed);
+  if (freed_out) *freed_out = freed;
+  if (stage_out) *stage_out = stage;
+  return MZC_OK;
+}
+
+mzc_status mzc_state_evict_size(mzc_state* st, const mzc_evict_plan* times, int64_t bytes,
+                                int64_t* freed_out, int32_t* stage_out) {
+  if (!st || !times) return MZC_ERR_INVALID;
+  mzc::State& S = st->st;
+  mzc_evict_plan p = *times;
+  const int32_t L = S.shape().n_layers;
+  p.kv_total = mzc::ceil_div(S.n_ctx(), 16);
+  p.w_total = L;
+  int64_t c0 = 0, r0 = 0;
+  int32_t w0 = 0;
+  mzc_status e = S.evicted_layout(&c0, &r0, &w0);
+  if (e != MZC_OK) return e;
+  p.kv_copy = c0;
+  p.kv_rec = r0;
+  p.w_evicted = w0;
+  int64_t freed = 0;
+  int32_t stage = 0;
+  e = mzc_plan_evict_size(&p, bytes, &freed, &stage);
+  if (e != MZC_OK) return e;
+  mzc::EvictSizeSteps steps;
+  mzc::evict_size_steps(S.n_ctx(), L, c0, r0, w0, p, &steps);
+  if (steps.copy_t1 > steps.copy_t0) {
+    e = S.evict_range(0, L, steps.copy_t0, steps.copy_t1, MZC_COPY, nullptr);
+    if (e != MZC_OK) return e;
+  }
+  if (steps.drop_t1 > steps.drop_t0) {
+    e = S.evict_range(0, L, steps.drop_t0, steps.drop_t1, MZC_DROP, nullptr);
+    if (e != MZC_OK) return e;
+  }
+  if (steps.w1 > steps.w0) {
+    e = S.evict_weights(steps.w0, steps.w1);
+    if (e != MZC_OK) return e;
+  }
+  if (freed_out) *freed_out = freed;
+  if (stage_out) *stage_out = stage;
+  return MZC_OK;
+}
+
 mzc_status mzc_state_recompute_tail(mzc_state* st, int64_t p, int64_t n) {
   if (!st) return MZC_ERR_INVALID;
   return st->st.recompute_tail(p, n);

@@ -78,6 +78,15 @@ MZC_K_NCLASS = 6
 KERNEL_CLASS_NAMES = ("gemm", "attention", "rope_kv", "rmsnorm", "lm_head", "embed")
 
 
+class mzc_evict_plan(ctypes.Structure):
+    _fields_ = [("t_copy_w", c_f64), ("t_copy_kv", c_f64), ("t_rec_kv", c_f64),
+                ("kv_total", c_i64), ("w_total", c_i32), ("w_evicted", c_i32),
+                ("kv_copy", c_i64), ("kv_rec", c_i64), ("kv_bytes", c_i64), ("w_bytes", c_i64)]
+
+
+MZC_STAGE_KV_ONLY, MZC_STAGE_KV_AND_W, MZC_STAGE_W_ONLY, MZC_STAGE_COMP_KV = 1, 2, 3, 4
+
+
 class mzc_copy_run(ctypes.Structure):
     _fields_ = [("layer", c_i32), ("n_blocks", c_i32), ("host_off", c_i64),
                 ("phys_begin", c_i64)]
@@ -129,6 +138,10 @@ _SIGS = {
                              c_vp, c_i64, c_vp, c_i64, c_vp, c_i64, c_vp, c_vp],
     "mzc_k_lm_head": [c_vp, c_vp, c_i32, c_f32, c_vp, c_i64, c_vp, c_vp],
     "mzc_plan_split_ctx": [c_vp, c_i64, c_i64, c_vp],
+    "mzc_plan_evict_size": [P(mzc_evict_plan), c_i64, P(c_i64), P(c_i32)],
+    "mzc_evict_size": [c_vp, c_i64, P(c_i64), P(c_i32)],
+    "mzc_evict_size_plan": [c_vp, P(mzc_evict_plan)],
+    "mzc_state_evict_size": [c_vp, P(mzc_evict_plan), c_i64, P(c_i64), P(c_i32)],
     "mzc_k_wait_probe": [c_i32, c_i64, c_vp, c_vp, c_vp],
     "mzc_k_q8_encode": [c_vp, c_vp, c_i64, c_i32, c_i32, c_vp, c_vp],
     "mzc_k_q8_decode": [c_vp, c_i64, c_i32, c_i32, c_vp, c_i64, c_i32, c_vp, c_vp],
@@ -294,6 +307,33 @@ def mzc_profile_measure(ctx) -> mzc_profile:
     p = mzc_profile()
     _call("mzc_profile_measure", ctx, ctypes.byref(p), ctx=ctx)
     return p
+
+
+def mzc_plan_evict_size(plan: mzc_evict_plan, nbytes):
+    """Advances plan's counts (in place) by the eviction policy; returns
+    (freed bytes, last stage)."""
+    f, st = c_i64(), c_i32()
+    _call("mzc_plan_evict_size", ctypes.byref(plan), nbytes, ctypes.byref(f), ctypes.byref(st))
+    return f.value, st.value
+
+
+def mzc_evict_size(ctx, nbytes):
+    """evict(size): returns (freed bytes, last stage)."""
+    f, st = c_i64(), c_i32()
+    _call("mzc_evict_size", ctx, nbytes, ctypes.byref(f), ctypes.byref(st), ctx=ctx)
+    return f.value, st.value
+
+
+def mzc_evict_size_plan(ctx) -> mzc_evict_plan:
+    p = mzc_evict_plan()
+    _call("mzc_evict_size_plan", ctx, ctypes.byref(p), ctx=ctx)
+    return p
+
+
+def mzc_state_evict_size(state, times: mzc_evict_plan, nbytes):
+    f, st = c_i64(), c_i32()
+    _call("mzc_state_evict_size", state, ctypes.byref(times), nbytes, ctypes.byref(f), ctypes.byref(st))
+    return f.value, st.value
 
 
 def mzc_truncate(ctx, n_ctx):

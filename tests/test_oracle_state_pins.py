@@ -103,9 +103,30 @@ def test_double_eviction_is_a_state_error():
     assert m.append(256) == OK
     assert m.evict(0, 2, 0, 32, 0) == OK
     assert m.evict(0, 1, 16, 48, 0) == STATE   # block 1 is already SWAPPED
-    assert m.evict(0, 2, 0, 16, 1) == STATE    # a swapped block cannot be dropped
     assert m.evict_blocks([(1, 0)]) == STATE
     assert m.st[0] == _row(16, [(0, 16, RESIDENT), (0, 2, SWAPPED)])
+    assert m.evict(0, 2, 240, 256, 1) == OK
+    assert m.evict(0, 2, 240, 256, 1) == STATE  # dropped twice
+    assert m.evict(0, 2, 240, 256, 0) == STATE  # a dropped block cannot be swapped
+
+
+def test_drop_may_take_swapped_blocks():
+    """The eviction policy can move a unit from the copy path to the recompute
+    path: DROP over SWAPPED blocks discards their host copies."""
+    m = StateModel(2, 256)
+    assert m.append(256) == OK
+    assert m.evict(0, 2, 128, 256, 0) == OK    # blocks 8..15 swapped
+    assert m.evict(0, 2, 224, 256, 1) == OK    # blocks 14, 15: swapped -> dropped
+    want = _row(16, [(0, 16, RESIDENT), (8, 14, SWAPPED), (14, 16, DROPPED)])
+    assert m.st == [want, want]
+    assert m.drop == (224, 256)
+    # a range that is part resident, part swapped, adjacent to the drop
+    assert m.evict(0, 2, 112, 224, 1) == OK    # blocks 7 (resident) .. 13 (swapped)
+    want = _row(16, [(0, 16, RESIDENT), (7, 16, DROPPED)])
+    assert m.st == [want, want]
+    assert m.drop == (112, 256)
+    assert m.restore() == OK and not m.inflight  # nothing left to copy back
+    assert m.recompute_tail(112, 144) == OK
 
 
 def test_prefill_over_dropped_blocks_needs_the_recompute():
