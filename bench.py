@@ -51,21 +51,24 @@ METRIC = "TTFT ms vs evicted fraction (1 GB300); recompute tok/s; % BF16 tensor 
 
 
 def _traffic(kernel_class, workload):
-    """Per-launch DRAM bytes from the committed ncu capture, or None when the
-    capture was of another workload or the kernel's source changed since the
-    counters were taken."""
+    """Per-launch DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum)
+    from the committed ncu capture of this kernel class on this workload, or
+    None when there is none or the kernel's source changed since the counters
+    were taken."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
-            t = json.load(f)[kernel_class]
-        if t.get("workload") != workload:
-            return None
-        src = open(os.path.join(ROOT, t["source"]), "rb").read()
-        if hashlib.sha256(src).hexdigest()[:16] != t["source_sha"]:
-            return None
-        return t["bytes_per_launch"]
+            entries = json.load(f)["entries"]
+        for t in entries:
+            if t.get("class") != kernel_class or t.get("workload") != workload:
+                continue
+            src = open(os.path.join(ROOT, t["source"]), "rb").read()
+            if hashlib.sha256(src).hexdigest()[:16] != t["source_sha"]:
+                return None
+            return t["bytes_per_launch"]
     except Exception:
         return None
+    return None
 
 
 def _peaks():
