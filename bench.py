@@ -151,7 +151,7 @@ class Runner:
     """Owns one ctx on one GPU and knows how to put the evicted state at rest
     (untimed) and run one timed restore + prefill."""
 
-    def __init__(self, name, sc, device, codec=0):
+    def __init__(self, name, sc, device, codec=0, read_swapped=0):
         import synth
         import paper_2609_01338_gb300 as m
         self.m, self.name, self.sc = m, name, sc
@@ -164,7 +164,8 @@ class Runner:
         self.prompt = synth.tokens(synth.SEED_PROMPT, 0, sc["prompt"], sh["vocab"])
         max_rows = min(sh["max_ctx"], 16384 + 1024)
         t = time.time()
-        self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device, swap_codec=codec)
+        self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device, swap_codec=codec,
+                              read_swapped=read_swapped)
         self.t_create = time.time() - t
         t = time.time()
         m.mzc_prefill(self.c, self.ctx_tokens)  # long contexts run in causal chunks
@@ -538,7 +539,8 @@ def main():
     ap.add_argument("--impl", default="mzc", choices=["mzc", "reference"])
     ap.add_argument("--workload", default="3b_sweep",
                     choices=["3b_sweep", "1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed",
-                             "3b_order", "1b_decode", "3b_decode", "link", "kernels"])
+                             "3b_order", "1b_decode", "3b_decode", "3b_read_swapped", "link",
+                             "kernels"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--no-1b", action="store_true", help="3b_sweep: skip the 1B recompute keys")
@@ -588,7 +590,8 @@ def main():
     __graft_entry__.build()
     import paper_2609_01338_gb300 as m
 
-    r = Runner(name, sc, local, codec=1 if args.codec == "q8" else 0)
+    r = Runner(name, sc, local, codec=1 if args.codec == "q8" else 0,
+               read_swapped=1 if name == "3b_read_swapped" else 0)
     if name == "3b_sweep":
         run_headline(r, args, rank, world, local, dist)
         if dist:
@@ -596,6 +599,10 @@ def main():
         return
     if name == "3b_order":
         run_order(r, args, rank)
+        r.close()
+        return
+    if name == "3b_read_swapped":
+        run_read_swapped(r, args, rank)
         r.close()
         return
     if name.endswith("_decode"):
@@ -975,6 +982,43 @@ def run_order(r, args, rank):
     if rank == 0:
         print(json.dumps({"metric": "TTFT ms by eviction order", "workload": _describe("3b_order", r.sc),
                           "swap_codec": args.codec, "order": res, "points": pts}), flush=True)
+
+
+def run_read_swapped(r, args, rank):
+    """Swapped blocks restored by copy (mzc_restore_async, then the prefill)
+    against read in place by the attention kernels (the prefill alone, option
+    read_swapped), for token tails of the 3B context (Sec. 4.2's shared
+    buffers on a GB300: the same bytes cross the host link either way)."""
+    m, L, N = r.m, r.shape["n_layers"], r.N
+    res, pts = {}, []
+    for frac in r.sc["fractions"]:
+        p = max(0, N - int(np.ceil(frac * r.nblk)) * 16)
+        for mode in ("copy", "in_place"):
+            vals = []
+            if mode == "in_place":
+                m.mzc_evict(r.c, 0, L, p, N, m.MZC_COPY)  # stays swapped across the steps
+            for i in range(args.warmup + args.steps):
+                if mode == "copy":
+                    m.mzc_evict(r.c, 0, L, p, N, m.MZC_COPY)
+                    m.mzc_restore_async(r.c)
+                m.mzc_prefill(r.c, r.prompt, r.logits)
+                t = m.mzc_last_times(r.c)
+                m.mzc_truncate(r.c, N)
+                if i >= args.warmup:
+                    vals.append(float(t[3]))
+            if mode == "in_place":
+                m.mzc_restore_async(r.c)
+                m.mzc_sync(r.c)
+            pt = {"fraction": frac, "mode": mode, "ttft_ms": round(statistics.median(vals), 3),
+                  "p10": round(float(np.percentile(vals, 10)), 3),
+                  "p90": round(float(np.percentile(vals, 90)), 3),
+                  "swapped_bytes": int((N - p) * L * 2 * r.shape["n_kv_heads"] * r.shape["head_dim"] * 2)}
+            pts.append(pt)
+            res.setdefault(frac, {})[mode] = pt["ttft_ms"]
+            print(json.dumps(pt), file=sys.stderr, flush=True)
+    if rank == 0:
+        print(json.dumps({"metric": "TTFT ms: swapped blocks copied back vs read in place",
+                          "workload": _describe(r.name, r.sc), "ttft": res, "points": pts}), flush=True)
 
 
 def run_decode(r, args, rank):

@@ -110,7 +110,13 @@ typedef struct {
                                block inside the pool); during it, synchronize after each
                                layer and read the device status word, so an error names
                                the layer where it appeared.  Slower; results unchanged */
-  int32_t reserved;         /* 0 */
+  int32_t read_swapped;     /* 1: a prefill may read SWAPPED blocks in place from the pinned
+                               store (mapped host memory) when no mzc_restore_async was
+                               issued for them: the attention kernels fetch them over the
+                               host link with plain loads, and they stay SWAPPED (the
+                               paper's shared buffers, Sec. 4.2).  Not with MZC_CODEC_Q8.
+                               A block the new rows write into (the context's partial
+                               last block) must be resident: MZC_ERR_STATE otherwise */
   void *compute_stream;     /* cudaStream_t the prefill kernels run on, owned by the caller
                                (it must outlive the ctx); NULL = the ctx creates its own.
                                mzc_prefill synchronizes this stream before it returns */
@@ -191,7 +197,8 @@ mzc_status mzc_destroy(mzc_ctx *ctx);
  * Row sets larger than options->max_rows run in causal chunks of max_rows
  * rows (a chunk goes through all layers before the next).
  * Errors: MZC_ERR_STATE if any block the rows attend to is SWAPPED without a
- * restore in flight, or DROPPED without a pending recompute; MZC_ERR_OOM if
+ * restore in flight (unless the ctx reads swapped blocks in place, option
+ * read_swapped), or DROPPED without a pending recompute; MZC_ERR_OOM if
  * the pool is full; MZC_ERR_RANGE past max_ctx. */
 mzc_status mzc_prefill(mzc_ctx *ctx, const int32_t *tokens, int64_t n, float *logits_out);
 

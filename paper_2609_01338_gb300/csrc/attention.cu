@@ -175,7 +175,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     int64_t pool_blocks,
     uint16_t* __restrict__ out, float* __restrict__ part_o, float* __restrict__ part_lse,
     int keys_per_split, int n_splits, float scale_log2, int32_t* status,
-    const int32_t* __restrict__ flags, long long flag_wait_cycles) {
+    const int32_t* __restrict__ flags, long long flag_wait_cycles,
+    const uint16_t* __restrict__ host_pool, int64_t host_blocks) {
   using C = AttnCfg<HD>;
   constexpr int BN = C::BN;
   extern __shared__ uint8_t smem_raw[];
@@ -294,16 +295,20 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
         const int s = j % C::STAGES;
         const int32_t p_nxt = j + 1 < T ? lookup(j + 1) : kPast;
         int32_t p = p_cur;
-        if (p != kPast && (p < 0 || p >= pool_blocks)) {
+        // a swapped block read in place: entry -2 - slot of the pinned store
+        const bool host = host_pool != nullptr && p != kPast && p <= -2 &&
+                          -static_cast<int64_t>(p) - 2 < host_blocks;
+        if (p != kPast && !host && (p < 0 || p >= pool_blocks)) {
           set_status(status, kStatusDevice);  // its keys read another block
           p = kPast;
         }
-        const bool valid = p != kPast;
+        const bool valid = p != kPast && !host;  // fetched by TMA from the pool
+        const unsigned host_lanes = __ballot_sync(0xffffffffu, host);
         const int32_t first_raw = __shfl_sync(0xffffffffu, p, 0);
         const int32_t first = first_raw < 0 ? 0 : first_raw;
         // the tile's blocks are consecutive in the pool: one box per operand slice
         // (blocks past the key range are read too; their keys are masked)
-        const bool run = __all_sync(0xffffffffu, !valid || p == first + lane);
+        const bool run = host_lanes == 0 && __all_sync(0xffffffffu, !valid || p == first + lane);
         const int32_t mine = valid ? p : first;
         bool ok = true;
         if (lane == 0 && j >= C::STAGES)
@@ -334,9 +339,44 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
           }
           fence_proxy_async_global();  // the TMA reads come after the flags were seen
         }
+        uint32_t tma_bytes = C::KV_BYTES;
+        if (host_lanes != 0) {
+          // blocks held in pinned host memory: the warp copies their K and V
+          // rows over the host link with 16-byte cp.async (plain loads, no
+          // TMA) into the places the per-block TMA boxes would fill (128-byte
+          // swizzle), and each lane registers its copies on the stage's
+          // barriers before lane 0 arrives, so no phase completes early
+          constexpr int CPR = HD / 8;  // 16-byte chunks per row
+          for (unsigned hm = host_lanes; hm != 0; hm &= hm - 1) {
+            const int hl = __ffs(hm) - 1;
+            const int64_t hb = -static_cast<int64_t>(__shfl_sync(0xffffffffu, p, hl)) - 2;
+            const uint16_t* src = host_pool + hb * (2LL * hkv * 16 * HD);
+#pragma unroll 1
+            for (int ci = lane; ci < 16 * CPR; ci += 32) {
+              const int r = ci / CPR, cc = ci % CPR, c = cc >> 3, u = cc & 7;
+              const uint32_t off = c * (BN * 128) + hl * 16 * 128 + r * 128 + ((u ^ (r & 7)) << 4);
+              cp_async16(smem_u32(sK + s * C::KV_BYTES + off), src + (static_cast<int64_t>(yk + r)) * HD + cc * 8);
+            }
+          }
+          cp_async_mbar_arrive(&k_full[s]);
+          for (unsigned hm = host_lanes; hm != 0; hm &= hm - 1) {
+            const int hl = __ffs(hm) - 1;
+            const int64_t hb = -static_cast<int64_t>(__shfl_sync(0xffffffffu, p, hl)) - 2;
+            const uint16_t* src = host_pool + hb * (2LL * hkv * 16 * HD);
+#pragma unroll 1
+            for (int ci = lane; ci < 16 * CPR; ci += 32) {
+              const int r = ci / CPR, cc = ci % CPR, c = cc >> 3, u = cc & 7;
+              const uint32_t off = c * (BN * 128) + hl * 16 * 128 + r * 128 + ((u ^ (r & 7)) << 4);
+              cp_async16(smem_u32(sV + s * C::KV_BYTES + off), src + (static_cast<int64_t>(yv + r)) * HD + cc * 8);
+            }
+          }
+          cp_async_mbar_arrive(&v_full[s]);
+          tma_bytes = (NB - __popc(host_lanes)) * 16 * 128 * C::CB;
+          __syncwarp();
+        }
         if (lane == 0) {
-          mbar_arrive_expect_tx(&k_full[s], C::KV_BYTES);
-          mbar_arrive_expect_tx(&v_full[s], C::KV_BYTES);
+          mbar_arrive_expect_tx(&k_full[s], tma_bytes);
+          mbar_arrive_expect_tx(&v_full[s], tma_bytes);
         }
         __syncwarp();
         if (run) {
@@ -347,7 +387,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
               tma_load_3d(sV + s * C::KV_BYTES + c * (BN * 128), &pool_run, &v_full[s], c * 64, yv, first);
             }
           }
-        } else if (lane < NB) {
+        } else if (lane < NB && !host) {
 #pragma unroll
           for (int c = 0; c < C::CB; ++c) {
             tma_load_3d(sK + s * C::KV_BYTES + c * (BN * 128) + lane * 16 * 128, &pool_blk, &k_full[s],
@@ -403,6 +443,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
       bool ok = wait_bar(&k_full[0], 0, status, abort_flag);
       if (ok) {
         tc_fence_after();
+        if (host_pool != nullptr) fence_async_smem();
         issue_s(0);
       }
       for (int j = 0; ok && j < T; ++j) {
@@ -412,11 +453,13 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
           if (!wait_bar(&k_full[(j + 1) % C::STAGES], ((j + 1) / C::STAGES) & 1, status, abort_flag)) break;
           if (!wait_bar(&s_free[t], ph, status, abort_flag)) break;
           tc_fence_after();
+          if (host_pool != nullptr) fence_async_smem();  // cp.async-written K before the UMMA reads it
           issue_s(j + 1);
         }
         if (!wait_bar(&v_full[j % C::STAGES], (j / C::STAGES) & 1, status, abort_flag)) break;
         if (!wait_bar(&p_full[t], ph, status, abort_flag)) break;
         tc_fence_after();
+        if (host_pool != nullptr) fence_async_smem();  // ... and V
         issue_pv(j);
       }
       // every UMMA this thread issued has completed before TMEM is released
@@ -680,7 +723,8 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
                       const int32_t* table, int64_t n_logical, const void* pool,
                       int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
                       int n_splits, int keys_per_split, int32_t* status, const int32_t* flags,
-                      long long flag_wait, cudaStream_t st) {
+                      long long flag_wait, const uint16_t* host_pool, int64_t host_blocks,
+                      cudaStream_t st) {
   using C = AttnCfg<HD>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -702,7 +746,7 @@ cudaError_t launch_hd(const uint16_t* q, const int32_t* pos, int64_t n, int32_t 
       static_cast<float>(1.0 / std::sqrt(static_cast<double>(HD)) * 1.4426950408889634);
   launch_k(attn_tc_kernel<HD, F16>, dim3(grid), dim3(C::THREADS), C::SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, run_map, blk_map, pool_blocks, out, part_o,
-      part_lse, keys_per_split, n_splits, scale_log2, status, flags, flag_wait);
+      part_lse, keys_per_split, n_splits, scale_log2, status, flags, flag_wait, host_pool, host_blocks);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || n_splits == 1) return e;
   const int64_t rows = n * hq;
@@ -756,7 +800,8 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,
                              uint16_t* out, void* scratch, int64_t scratch_bytes,
                              int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st,
-                             const int32_t* flags, int64_t flag_wait_cycles) {
+                             const int32_t* flags, int64_t flag_wait_cycles, const void* host_pool,
+                             int64_t host_blocks) {
   if (n <= 0) return cudaSuccess;
   const long long fw = flag_wait_cycles > 0 ? flag_wait_cycles : kWaitCycles;
   int s = 1, per = 0;
@@ -772,7 +817,8 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   (void)kv_dtype;  // the pool is fp16-encoded for both KV types: q, K, P, V are fp16
   if (attention_decode_applies(n, hq, hkv, hd)) {
     cudaError_t e = launch_attention_decode(q, pos, n, hq, hkv, hd, table, n_logical, pool, pool_blocks, out,
-                                            part_o, part_lse, s, per, status, flags, fw, st);
+                                            part_o, part_lse, s, per, status, flags, fw,
+                                            static_cast<const uint16_t*>(host_pool), host_blocks, st);
     if (e != cudaSuccess || s == 1) return e;
     const int64_t rows = n * hq;
     if (hd == 64)
@@ -783,10 +829,12 @@ cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, i
   }
   if (hd == 64)
     return launch_hd<64, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
-                               part_o, part_lse, s, per, status, flags, fw, st);
+                               part_o, part_lse, s, per, status, flags, fw,
+                               static_cast<const uint16_t*>(host_pool), host_blocks, st);
   if (hd == 128)
     return launch_hd<128, true>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out,
-                                part_o, part_lse, s, per, status, flags, fw, st);
+                                part_o, part_lse, s, per, status, flags, fw,
+                                static_cast<const uint16_t*>(host_pool), host_blocks, st);
   return cudaErrorInvalidValue;
 }
 

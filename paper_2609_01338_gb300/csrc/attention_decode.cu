@@ -112,7 +112,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     const int32_t* __restrict__ table, int64_t n_logical, const uint16_t* __restrict__ pool,
     int64_t pool_blocks, uint16_t* __restrict__ out, float* __restrict__ part_o,
     float* __restrict__ part_lse, int blocks_per_split, int n_splits, float scale_log2,
-    int32_t* status, const int32_t* __restrict__ flags, long long flag_wait_cycles) {
+    int32_t* status, const int32_t* __restrict__ flags, long long flag_wait_cycles,
+    const uint16_t* __restrict__ host_pool, int64_t host_blocks) {
   using C = DecCfg<HD>;
   constexpr int DPL = C::DPL;
   extern __shared__ uint8_t smem_raw[];
@@ -176,6 +177,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     }
     const int32_t p = table[b];
     if (p >= 0 && p < pool_blocks) return p;
+    // a swapped block read in place: entry -2 - slot of the pinned store
+    if (host_pool != nullptr && p <= -2 && -static_cast<int64_t>(p) - 2 < host_blocks) return p;
     set_status(status, kStatusDevice);
     return -1;
   };
@@ -186,8 +189,25 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
   };
   auto issue = [&](int i, int32_t p) {  // issuer lane, physical block p of block i
     const int s = i % C::STAGES;
-    if (p < 0) {
+    if (p == -1) {
       mbar_arrive(&pfull[s]);  // completes the phase with no data
+      return;
+    }
+    if (p <= -2) {
+      // in pinned host memory: the block's K and V rows of head g over the
+      // host link with 16-byte cp.async (plain loads), tracked by the slot's
+      // barrier, then this thread's own arrival
+      const uint16_t* hb = host_pool + (-static_cast<int64_t>(p) - 2) * blk_elems;
+      const uint16_t* ks = hb + static_cast<int64_t>(g) * 16 * HD;
+      const uint16_t* vs = hb + static_cast<int64_t>(hkv + g) * 16 * HD;
+      const uint32_t dk = smem_u32(pring + s * C::SLOT), dv = dk + C::HALF;
+#pragma unroll 4
+      for (int c = 0; c < C::HALF / 16; ++c) {
+        cp_async16(dk + c * 16, ks + c * 8);
+        cp_async16(dv + c * 16, vs + c * 8);
+      }
+      cp_async_mbar_arrive(&pfull[s]);
+      mbar_arrive(&pfull[s]);
       return;
     }
     if (flags != nullptr) {
@@ -245,7 +265,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) attn_decode_kernel(
     }
     done = i + 1;
     const int b = b_begin + pair + kDecPairs * i;
-    const bool valid = pblk >= 0;
+    const bool valid = pblk != -1;  // in the pool, or in host memory (<= -2)
     const uint16_t* kh = reinterpret_cast<const uint16_t*>(pring + s * C::SLOT) + (8 * hk) * HD + lane * DPL;
     const uint16_t* vh = reinterpret_cast<const uint16_t*>(pring + s * C::SLOT + C::HALF) + (8 * hk) * HD +
                          lane * DPL;
@@ -380,7 +400,8 @@ template <int HD, int R>
 cudaError_t launch_dec(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq, int32_t hkv,
                        const int32_t* table, int64_t n_logical, const void* pool, int64_t pool_blocks,
                        uint16_t* out, float* part_o, float* part_lse, int n_splits, int blocks_per_split,
-                       int32_t* status, const int32_t* flags, long long flag_wait, cudaStream_t st) {
+                       int32_t* status, const int32_t* flags, long long flag_wait,
+                       const uint16_t* host_pool, int64_t host_blocks, cudaStream_t st) {
   constexpr int SMEM = dec_smem_bytes<HD>();
   static_assert(SMEM <= 232448, "shared memory of one CTA");
   static_assert(kDecWarps * R * (HD + 2) * 4 <= DecCfg<HD>::RING, "warp partials fit in the rings");
@@ -396,7 +417,8 @@ cudaError_t launch_dec(const uint16_t* q, const int32_t* pos, int64_t n, int32_t
   dim3 grid(static_cast<unsigned>(hkv), static_cast<unsigned>(n_splits));
   launch_k(attn_decode_kernel<HD, R>, dim3(grid), dim3(kDecThreads), SMEM, st,
       q, pos, static_cast<int>(n), hq, hkv, table, n_logical, static_cast<const uint16_t*>(pool), pool_blocks,
-      out, part_o, part_lse, blocks_per_split, n_splits, scale_log2, status, flags, flag_wait);
+      out, part_o, part_lse, blocks_per_split, n_splits, scale_log2, status, flags, flag_wait, host_pool,
+      host_blocks);
   return cudaGetLastError();
 }
 
@@ -422,7 +444,8 @@ cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64
                                     int32_t hd, const int32_t* table, int64_t n_logical, const void* pool,
                                     int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
                                     int n_splits, int keys_per_split, int32_t* status,
-                                    const int32_t* flags, long long flag_wait, cudaStream_t st) {
+                                    const int32_t* flags, long long flag_wait, const uint16_t* host_pool,
+                                    int64_t host_blocks, cudaStream_t st) {
   if (!attention_decode_applies(n, hq, hkv, hd) || keys_per_split % 16 != 0 ||
       reinterpret_cast<uintptr_t>(pool) % 16 != 0)  // bulk copies start on 16-byte boundaries
     return cudaErrorInvalidValue;
@@ -432,7 +455,7 @@ cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64
 #define MZC_DEC_CASE(HDV, RV)                                                                              \
   if (hd == HDV && R == RV)                                                                                \
     return launch_dec<HDV, RV>(q, pos, n, hq, hkv, table, n_logical, pool, pool_blocks, out, part_o, part_lse, \
-                               n_splits, bps, status, flags, flag_wait, st);
+                               n_splits, bps, status, flags, flag_wait, host_pool, host_blocks, st);
   MZC_DEC_CASE(64, 1)
   MZC_DEC_CASE(64, 2)
   MZC_DEC_CASE(64, 3)

@@ -108,16 +108,21 @@ cudaError_t launch_attention_decode(const uint16_t* q, const int32_t* pos, int64
                                     int32_t hd, const int32_t* table, int64_t n_logical, const void* pool,
                                     int64_t pool_blocks, uint16_t* out, float* part_o, float* part_lse,
                                     int n_splits, int keys_per_split, int32_t* status,
-                                    const int32_t* flags, long long flag_wait, cudaStream_t st);
+                                    const int32_t* flags, long long flag_wait, const uint16_t* host_pool,
+                                    int64_t host_blocks, cudaStream_t st);
 // flags (may be null): int32 per physical block, non-zero once the block's
 // data is in HBM; the kernels wait (bounded by flag_wait_cycles, 0 = the
 // default limit) for the flag of every block they read before fetching it.
+// host_pool (may be null): device-accessible base of pinned host memory
+// holding host_blocks KV blocks in the pool's block layout; a block-table
+// entry -2 - i names host block i, read in place with plain loads.
 cudaError_t launch_attention(const uint16_t* q, const int32_t* pos, int64_t n, int32_t hq,
                              int32_t hkv, int32_t hd, const int32_t* table, int64_t n_logical,
                              const void* pool, int64_t pool_blocks, int32_t kv_dtype,
                              uint16_t* out, void* scratch, int64_t scratch_bytes,
                              int64_t max_keys, int num_sms, int32_t* status, cudaStream_t st,
-                             const int32_t* flags = nullptr, int64_t flag_wait_cycles = 0);
+                             const int32_t* flags = nullptr, int64_t flag_wait_cycles = 0,
+                             const void* host_pool = nullptr, int64_t host_blocks = 0);
 // Attention whose split-KV partials use a fixed array inside the library
 // (kAttnNoallocScratchBytes) instead of caller memory; no allocation.
 constexpr int64_t kAttnNoallocScratchBytes = 8LL << 20;

@@ -351,6 +351,11 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
+// The mbarrier tracks every cp.async this thread issued so far: its pending
+// count goes up by one now and down by one (an arrival) once they complete.
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 
 // pack two floats into a 16-bit pair (low = a)
 template <bool F16>

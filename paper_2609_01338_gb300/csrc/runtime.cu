@@ -88,6 +88,7 @@ struct mzc_ctx {
   int64_t scratch_bytes = 0;
   int32_t* d_status = nullptr;
   uint8_t* h_store = nullptr;
+  uint16_t* h_store_dev = nullptr;  // device view of the mapped store (read_swapped)
   uint8_t* d_staging = nullptr;
   int32_t* d_list = nullptr;
   int32_t* h_list = nullptr;
@@ -245,6 +246,11 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
     return ctx->fail(MZC_ERR_INVALID, "MZC_WAIT_BLOCK_FLAG needs swap_codec MZC_CODEC_NONE");
   if (ctx->opt.debug_checks != 0 && ctx->opt.debug_checks != 1)
     return ctx->fail(MZC_ERR_INVALID, "debug_checks must be 0 or 1");
+  if (ctx->opt.read_swapped != 0 && ctx->opt.read_swapped != 1)
+    return ctx->fail(MZC_ERR_INVALID, "read_swapped must be 0 or 1");
+  // in-place reads need the blocks as stored (not 8-bit codes)
+  if (ctx->opt.read_swapped && ctx->opt.swap_codec != MZC_CODEC_NONE)
+    return ctx->fail(MZC_ERR_INVALID, "read_swapped needs swap_codec MZC_CODEC_NONE");
   ctx->codec = ctx->opt.swap_codec;
   {
     const int64_t block_elems = 2LL * s.n_kv_heads * 16 * s.head_dim;
@@ -252,6 +258,7 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   }
   mzc_status ss = ctx->st.init(s, ctx->opt.pool_blocks, ctx->opt.host_store_bytes, ctx->slot_bytes);
   if (ss != MZC_OK) return ctx->fail(ss, ctx->st.error());
+  ctx->st.set_read_swapped(ctx->opt.read_swapped != 0);
   if (!weights || !weights->embed || !weights->lm_head || !weights->final_norm || !weights->layers)
     return ctx->fail(MZC_ERR_INVALID, "weights are incomplete");
   CK(cudaSetDevice(ctx->opt.device));
@@ -467,7 +474,13 @@ mzc_status poison(mzc_ctx* ctx, const std::vector<int32_t>& phys) {
 
 mzc_status ensure_store(mzc_ctx* ctx) {
   if (ctx->h_store) return MZC_OK;
-  CK(cudaHostAlloc(&ctx->h_store, ctx->st.host_store_bytes(), cudaHostAllocDefault));
+  if (ctx->opt.read_swapped) {
+    // mapped, so the attention kernels can read swapped blocks in place
+    CK(cudaHostAlloc(&ctx->h_store, ctx->st.host_store_bytes(), cudaHostAllocMapped));
+    CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&ctx->h_store_dev), ctx->h_store, 0));
+  } else {
+    CK(cudaHostAlloc(&ctx->h_store, ctx->st.host_store_bytes(), cudaHostAllocDefault));
+  }
   return MZC_OK;
 }
 
@@ -550,8 +563,11 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     hpos[nrec + i] = static_cast<int32_t>(P.prompt_begin + i);
   }
   std::vector<int32_t> tab;
-  ctx->st.block_table(&tab);
+  ctx->st.block_table(&tab, ctx->opt.read_swapped != 0);
   std::memcpy(htab, tab.data(), tab.size() * 4);
+  // swapped blocks this prefill reads in place from the mapped store
+  const void* host_pool = ctx->opt.read_swapped ? ctx->h_store_dev : nullptr;
+  const int64_t host_blocks = host_pool ? ctx->st.host_slots() : 0;
   const size_t mbytes = static_cast<size_t>(rows) * 8 + tab.size() * 4;
   int32_t* dtok = reinterpret_cast<int32_t*>(ctx->d_meta);
   int32_t* dpos = dtok + rows;
@@ -626,7 +642,8 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         return mzc::launch_attention(ctx->d_q + r0 * hq * hd, cpos + r0, nr, s.n_q_heads, s.n_kv_heads,
                                      s.head_dim, ltab, ctx->nblk, ctx->d_pool, ctx->st.pool_blocks(),
                                      s.kv_dtype, ctx->d_attn + r0 * hq * hd, ctx->d_scratch,
-                                     ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs, wait_flags);
+                                     ctx->scratch_bytes, mk, ctx->num_sms, ctx->d_status, cs, wait_flags, 0,
+                                     host_pool, host_blocks);
       });
     };
     const double norm_bytes = R * dd * 6.0 + dd * 4.0;

@@ -331,10 +331,16 @@ mzc_status State::prepare_prefill(int64_t n_prompt, int64_t max_rows, PrefillPla
   if (has_drop() && !rec_pending_)
     return fail(MZC_ERR_STATE, "dropped blocks without a pending recompute");
   const int64_t nb = ceil_div(n_ctx_, 16);
+  // a block the new rows write into: the context's last block when it is partial
+  const int64_t write_blk = (n_ctx_ % 16 && n_prompt > 0) ? n_ctx_ / 16 : -1;
   for (int32_t l = 0; l < L; ++l) {
     if (w_state_[l] == MZC_SWAPPED) return fail(MZC_ERR_STATE, "layer weights swapped, no restore in flight");
-    for (int64_t b = 0; b < nb; ++b)
-      if (at(l, b).st == MZC_SWAPPED) return fail(MZC_ERR_STATE, "swapped blocks without a restore in flight");
+    for (int64_t b = 0; b < nb; ++b) {
+      if (at(l, b).st != MZC_SWAPPED) continue;
+      if (!read_swapped_) return fail(MZC_ERR_STATE, "swapped blocks without a restore in flight");
+      if (b == write_blk)
+        return fail(MZC_ERR_STATE, "the block the new rows write into is swapped: restore it first");
+    }
   }
   PrefillPlan P;
   P.rec_begin = rec_pending_ ? drop_t0_ : 0;
@@ -457,9 +463,17 @@ void State::counts(mzc_stats_t* o) const {
   o->pool_free_blocks = pool_.free_total();
 }
 
-void State::block_table(std::vector<int32_t>* out) const {
+void State::block_table(std::vector<int32_t>* out, bool host_slots) const {
   out->resize(tab_.size());
-  for (size_t i = 0; i < tab_.size(); ++i) (*out)[i] = tab_[i].phys;
+  for (size_t i = 0; i < tab_.size(); ++i) {
+    const BlockEntry& e = tab_[i];
+    if (host_slots && e.st == MZC_SWAPPED) {
+      const int64_t slot = (regions_[e.region].host_off + static_cast<int64_t>(e.idx) * slot_bytes_) / slot_bytes_;
+      (*out)[i] = static_cast<int32_t>(-2 - slot);
+    } else {
+      (*out)[i] = e.phys;
+    }
+  }
 }
 
 // ---- eviction policy (Algorithm 1) -----------------------------------------

@@ -133,8 +133,13 @@ class State {
   // Longest run of free physical blocks (holds no live KV): length, start.
   int64_t largest_free_pool_run(int64_t* start) const { return pool_.largest_free(start); }
   void counts(mzc_stats_t* out) const;
-  // Block table rows [L][nblk_max] (phys or -1) for the device.
-  void block_table(std::vector<int32_t>* out) const;
+  // Block table rows [L][nblk_max] (phys or -1) for the device.  With
+  // host_slots, a SWAPPED block's entry is -2 - (its slot in the pinned store,
+  // in units of slot_bytes), for kernels that read it in place.
+  void block_table(std::vector<int32_t>* out, bool host_slots = false) const;
+  // Whether a prefill may read SWAPPED blocks in place (no restore issued).
+  void set_read_swapped(bool on) { read_swapped_ = on; }
+  int64_t host_slots() const { return host_bytes_ / slot_bytes_; }
 
  private:
   mzc_status fail(mzc_status s, const std::string& msg) {
@@ -153,6 +158,7 @@ class State {
   int64_t drop_t0_ = -1, drop_t1_ = -1;
   bool rec_pending_ = false;
   bool inflight_ = false;
+  bool read_swapped_ = false;
   std::string err_;
 };
 

@@ -40,7 +40,7 @@ class mzc_model_shape(ctypes.Structure):
 class mzc_options(ctypes.Structure):
     _fields_ = [("pool_blocks", c_i64), ("max_rows", c_i64), ("host_store_bytes", c_i64),
                 ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32),
-                ("wait_mode", c_i32), ("debug_checks", c_i32), ("reserved", c_i32),
+                ("wait_mode", c_i32), ("debug_checks", c_i32), ("read_swapped", c_i32),
                 ("compute_stream", c_vp), ("copy_stream", c_vp)]
 
 
@@ -239,12 +239,12 @@ def make_weights(weights: dict):
 
 def mzc_create(shape: dict, weights: dict, pool_blocks=0, max_rows=0, host_store_bytes=0,
                overlap=1, device=0, swap_codec=MZC_CODEC_NONE, wait_mode=MZC_WAIT_LAYER_EVENT,
-               debug_checks=0, compute_stream=None, copy_stream=None):
+               debug_checks=0, compute_stream=None, copy_stream=None, read_swapped=0):
     """compute_stream / copy_stream: cudaStream_t handles (ints, e.g. a torch
     stream's cuda_stream) owned by the caller, or None."""
     sh = make_shape(shape)
     opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec,
-                      wait_mode, debug_checks, 0, compute_stream, copy_stream)
+                      wait_mode, debug_checks, read_swapped, compute_stream, copy_stream)
     w, keep = make_weights(weights)
     out = c_vp()
     _call("mzc_create", ctypes.byref(sh), ctypes.byref(opt), ctypes.byref(w), ctypes.byref(out))

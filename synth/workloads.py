@@ -51,6 +51,10 @@ SCENARIOS = {
     # forward-in, 128-token prompt
     "3b_order": dict(model=THREE_B, context=32768, fractions=(0.25, 0.50),
                      orders=("backward", "forward", "random"), random_draws=5, prompt=128),
+    # swapped token tails of the 3B context restored by copy vs read in place by
+    # the attention kernels, 128-token prompt
+    "3b_read_swapped": dict(model=THREE_B, context=32768, fractions=(0.10, 0.25, 0.50, 1.0),
+                            prompt=128),
     # decode after the first token: single-token steps over a resident context
     "1b_decode": dict(model=ONE_B, context=8192, prompt=1, decode=True),
     "3b_decode": dict(model=THREE_B, context=32768, prompt=1, decode=True),
