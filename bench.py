@@ -151,7 +151,7 @@ class Runner:
     """Owns one ctx on one GPU and knows how to put the evicted state at rest
     (untimed) and run one timed restore + prefill."""
 
-    def __init__(self, name, sc, device, codec=0, read_swapped=0):
+    def __init__(self, name, sc, device, codec=0, read_swapped=0, wait_mode=0):
         import synth
         import paper_2609_01338_gb300 as m
         self.m, self.name, self.sc = m, name, sc
@@ -165,7 +165,7 @@ class Runner:
         max_rows = min(sh["max_ctx"], 16384 + 1024)
         t = time.time()
         self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device, swap_codec=codec,
-                              read_swapped=read_swapped)
+                              read_swapped=read_swapped, wait_mode=wait_mode)
         self.t_create = time.time() - t
         t = time.time()
         m.mzc_prefill(self.c, self.ctx_tokens)  # long contexts run in causal chunks
@@ -245,9 +245,9 @@ class Runner:
 HEADLINE = (1.0, "hybrid")
 
 
-def _config(name, sc, codec, n_gpus):
+def _config(name, sc, codec, n_gpus, wait_mode="event"):
     """The `config` object; both arms print the same one."""
-    cfg = {"workload": _describe(name, sc), "swap_codec": codec,
+    cfg = {"workload": _describe(name, sc), "swap_codec": codec, "wait_mode": wait_mode,
            "l2": "inputs larger than L2 (weights + KV >> 129 MB)",
            "parallelism": f"replicas x{n_gpus}" if n_gpus > 1 else "single GPU",
            "timed": "restore + recompute + prompt prefill + logits D2H per step; eviction between steps untimed"}
@@ -427,7 +427,7 @@ def run_reference(args, name, sc, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(statistics.mean(walls) * 1e3, 3), "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": _config(name, sc, args.codec, args.gpus),
+            "config": _config(name, sc, args.codec, args.gpus, args.wait_mode),
             "extrapolated": {"rows_per_timed_step": int(per), "rows_per_step": int(total),
                              "note": "value scales each step's sampled rows to the whole step; "
                                      "ms_per_step is the sampled step's own wall time"},
@@ -549,6 +549,9 @@ def main():
     ap.add_argument("--profile-json", default=None,
                     help="3b_sweep: load the per-unit profile from this file if it exists, else "
                          "measure it and save it there")
+    ap.add_argument("--wait-mode", default="event", choices=["event", "flag"],
+                    help="how attention waits for restored blocks: per-layer events, or per-block "
+                         "residency flags (MZC_WAIT_BLOCK_FLAG)")
     ap.add_argument("--codec", default="none", choices=["none", "q8"],
                     help="swap codec of the pinned store: none, or 8-bit groups (q8)")
     args = ap.parse_args()
@@ -591,7 +594,8 @@ def main():
     import paper_2609_01338_gb300 as m
 
     r = Runner(name, sc, local, codec=1 if args.codec == "q8" else 0,
-               read_swapped=1 if name == "3b_read_swapped" else 0)
+               read_swapped=1 if name == "3b_read_swapped" else 0,
+               wait_mode=1 if args.wait_mode == "flag" else 0)
     if name == "3b_sweep":
         run_headline(r, args, rank, world, local, dist)
         if dist:
@@ -643,7 +647,7 @@ def _single_line(r, args, world, name, sc, res, dist, clocks, wall):
         "ms_per_step": round(statistics.mean(res["dev"]), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": _config(name, sc, args.codec, world),
+        "config": _config(name, sc, args.codec, world, args.wait_mode),
         "recompute_tok_s": round(rec_rows / (v * 1e-3), 1) if rec_rows else None,
         "rows_per_step": rows,
         "gemm_tflops": round(gemm_tfs, 1) if gemm_tfs else None,
@@ -750,7 +754,7 @@ def run_headline(r, args, rank, world, local, dist):
         "ms_per_step": round(statistics.mean(head["dev"]), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": _config(name, sc, args.codec, world),
+        "config": _config(name, sc, args.codec, world, args.wait_mode),
         "sweep": sweep, "hybrid_vs_policies": vs, "points": pts, "profile": prof,
         "roofline": _roofline(head["ks"], head["dom"], peaks, src, name),
         **line_extra,
