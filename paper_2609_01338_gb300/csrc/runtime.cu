@@ -665,7 +665,13 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       }));
       const bool wait_rec = n_rec_c > 0 && P.kv_wait_rec[l];
       const bool wait_prm = n_prm_c > 0 && P.kv_wait_prompt[l];
-      if (flags && (wait_rec || wait_prm)) {
+      if (flags && n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
+        // recomputed rows read only resident keys: their own launch, with no
+        // flags, ahead of the prompt rows (in one launch the prompt rows' CTAs,
+        // dispatched first, would hold the SMs while they wait on the copies)
+        CKP(attention(0, n_rec_c, static_cast<int64_t>(hpos[c0 + n_rec_c - 1]) + 1, ltab));
+        CKP(attention(n_rec_c, n_prm_c, max_keys, ltab, flags));
+      } else if (flags && (wait_rec || wait_prm)) {
         CKP(attention(0, cr, max_keys, ltab, flags));
       } else if (n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
         // recompute rows read only resident keys: they run before the copy lands
