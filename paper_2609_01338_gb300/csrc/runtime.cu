@@ -609,6 +609,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
   // come last, so the last chunk holds the row whose logits are returned.
   const int64_t chunk = ctx->max_rows;
   int64_t last_rows = 0;
+  const bool want_logits = n > 0 && logits_out != nullptr;
   for (int64_t c0 = 0; c0 < rows; c0 += chunk) {
     const int64_t c1 = std::min(rows, c0 + chunk), cr = c1 - c0;
     const int64_t rec_hi = std::min(c1, nrec);          // recompute rows [c0, rec_hi)
@@ -665,6 +666,45 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       }));
       const bool wait_rec = n_rec_c > 0 && P.kv_wait_rec[l];
       const bool wait_prm = n_prm_c > 0 && P.kv_wait_prompt[l];
+      if (l == L - 1) {
+        // Every row's K/V of the last layer are written above.  The layer's
+        // output (attention, O, MLP) feeds only the logits, i.e. the call's
+        // last row: the other rows stop here, and without logits all do.
+        if (want_logits && c1 == rows) {
+          const int64_t r = cr - 1;
+          const double f = static_cast<double>(hq) * hd;
+          if (flags && wait_prm) {
+            CKP(attention(r, 1, max_keys, ltab, flags));
+          } else {
+            if (wait_prm) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+            CKP(attention(r, 1, max_keys, ltab));
+          }
+          auto row_gemm = [&](const void* a_row, const mzc::GemmWeight& w, void* out_row, int64_t N, int64_t K,
+                              int epi) {
+            const double out_b = epi == mzc::EPI_ADD_F32 ? N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? N * 1.0 : N * 2.0);
+            return klaunch(ctx, MZC_K_GEMM, 2.0 * N * K, 2.0 * (K + static_cast<double>(N) * K) + out_b, 1, [&] {
+              return mzc::launch_gemm(ctx->tm_h, w, out_row, 1, N, K, epi, ctx->d_status, cs,
+                                      static_cast<const uint16_t*>(a_row));
+            });
+          };
+          CKP(row_gemm(ctx->d_attn + r * hq * hd, W.tm_o, ctx->d_x + r * d, d, static_cast<int64_t>(f),
+                       mzc::EPI_ADD_F32));
+          CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, dd * 10.0, 1, [&] {
+            return mzc::launch_rmsnorm(ctx->d_x + r * d, W.ffn_norm, 1, static_cast<int32_t>(d), s.rms_eps,
+                                       ctx->d_h + r * d, cs, ctx->d_status);
+          }));
+          CKP(row_gemm(ctx->d_h + r * d, W.tm_13, ctx->d_act + r * ctx->f_pad, 2 * ctx->f_pad, d,
+                       mzc::EPI_SWIGLU_BF16));
+          CKP(row_gemm(ctx->d_act + r * ctx->f_pad, W.tm_2, ctx->d_x + r * d, d, ctx->f_pad, mzc::EPI_ADD_F32));
+        }
+        if (ctx->opt.debug_checks) {
+          CKP(cudaStreamSynchronize(cs));
+          mzc_status e = check_status(ctx, "layer " + std::to_string(l) + " (rows " + std::to_string(c0) +
+                                               ".." + std::to_string(c1) + "): ");
+          if (e != MZC_OK) return bail(e);
+        }
+        continue;
+      }
       if (flags && n_rec_c > 0 && n_prm_c > 0 && wait_prm && !wait_rec) {
         // recomputed rows read only resident keys: their own launch, with no
         // flags, ahead of the prompt rows (in one launch the prompt rows' CTAs,
