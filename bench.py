@@ -546,6 +546,13 @@ def main():
     ap.add_argument("--no-1b", action="store_true", help="3b_sweep: skip the 1B recompute keys")
     ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
     ap.add_argument("--policies", default=None, help="comma list overriding the sweep's policies")
+    ap.add_argument("--profile", default=None,
+                    help="3b_sweep: the per-unit profile as 9 comma-separated numbers in "
+                         "mzc_profile's field order (h2d_gbs, gemm_us_128, gemm_us_512, "
+                         "gemm_us_2048, attn_tflops, attn_row_ns, attn_prompt_tflops, row_ns, "
+                         "layer_us), as a default line's `profile` prints them; used instead of "
+                         "measuring it (a run under ncu would plan from its own serialised "
+                         "kernel times)")
     ap.add_argument("--profile-json", default=None,
                     help="3b_sweep: load the per-unit profile from this file if it exists, else "
                          "measure it and save it there")
@@ -674,7 +681,13 @@ def run_headline(r, args, rank, world, local, dist):
     import torch
     m = r.m
     sc, name = r.sc, r.name
-    if args.profile_json and os.path.exists(args.profile_json):
+    if args.profile:
+        vals = [float(x) for x in args.profile.split(",")]
+        if len(vals) != len(m.mzc_profile._fields_):
+            raise SystemExit("--profile takes %d numbers" % len(m.mzc_profile._fields_))
+        r.profile = m.mzc_profile(*vals)
+        m.mzc_set_policy(r.c, m.MZC_POLICY_HYBRID, r.profile)
+    elif args.profile_json and os.path.exists(args.profile_json):
         # a profile saved by an earlier run (an ncu run would otherwise plan
         # from its own serialised kernel times)
         with open(args.profile_json) as f:

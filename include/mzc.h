@@ -450,10 +450,39 @@ mzc_status mzc_k_rmsnorm(const float *x, const float *g, int64_t n, int32_t d, f
  * Kernel by m: up to 4 rows a GEMV streaming W (K split over two warps for
  * rows of 6 KB and more); up to 256 rows, when n is a multiple of 128, the K
  * range split over a thread-block cluster with the partials summed in a
- * fixed order; otherwise the persistent tcgen05 GEMM.  Each path gives the
- * same bits on every run. */
+ * fixed order; above 512 rows the paired-SM kernel (two CTAs of a cluster
+ * share 256 x 256 tiles through tcgen05 cta_group::2 MMAs) unless its tiles
+ * need more waves than single-CTA ones; otherwise the persistent single-CTA
+ * tcgen05 GEMM.  Each path gives the same bits on every run. */
 mzc_status mzc_k_gemm(const uint16_t *a, const uint16_t *w, void *out, int64_t m, int64_t n,
                       int64_t k, int32_t epilogue, void *stream);
+
+/* The residual-add GEMM (epilogue 1 of mzc_k_gemm: out fp32 [m][n] += A W^T,
+ * the O and down projections of every decoder layer) with the persistent
+ * kernel's last, partial wave split over k (stream-K), as the prefill runs
+ * it.  The last wave's R tiles are shared by up to 2R CTAs (all SMs at most,
+ * at least 4 k-blocks of 64 each); each CTA's partial sum is reduce-added into
+ * out in a fixed order per tile (highest k first), so the bits are the same
+ * on every run, though they differ from mzc_k_gemm's single add per element.
+ * The split is taken when the k-blocks it saves, (1 - R / SMs) x k / 64,
+ * reach 24 (the ordered adds cost about that much): long-K projections such
+ * as down.  Shapes and kernel choice as mzc_k_gemm; only the single-CTA
+ * persistent kernel splits (m of 257-512 rows, or m > 4 when n is not a
+ * multiple of 128, or above 512 rows when the paired kernel is not taken).
+ *   flags   DEVICE, n_flags uint64 entries, caller-owned; any contents.  The
+ *           kernel stores (epoch << 32 | k-block) values in the first R.
+ *   n_flags at least the device's SM count (else MZC_ERR_INVALID).
+ *   epoch   nonzero, and different from the epoch of every earlier launch
+ *           that used the same flags (a stale value could then match and the
+ *           order of the adds, though not their sum, would be lost).  Launches
+ *           sharing flags must run in stream order.
+ *   status  DEVICE int32 or NULL: MZC_ERR_TIMEOUT when a CTA waited longer
+ *           than about two seconds for the segment above it.
+ *   split_ctas  HOST int64 or NULL: the number of CTAs sharing the split
+ *           tiles (0: this shape ran unsplit). */
+mzc_status mzc_k_gemm_split(const uint16_t *a, const uint16_t *w, float *out, int64_t m,
+                            int64_t n, int64_t k, uint64_t *flags, int64_t n_flags,
+                            uint32_t epoch, int32_t *status, int64_t *split_ctas, void *stream);
 /* Host helper: interleaves gate [f][d] and up [f][d] into the [2f][d] row
  * order epilogue 2 reads (per 64 output features: 64 gate rows then the
  * matching 64 up rows).  f must be a multiple of 64. */

@@ -31,6 +31,27 @@ cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// The same with thread-block clusters of cluster_x CTAs along x.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t st, unsigned cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cluster_x;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
 
 // Row group of the SwiGLU weight interleave: 64 gate rows, then the matching
@@ -56,12 +77,29 @@ cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const struct GemmWeight& w
                                cudaStream_t st, bool* launched);
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 
+// State for splitting the residual-add GEMM's last wave over k: a device
+// array of n_flags uint64 (at least the number of SMs; any contents) and the
+// epoch of the last split launch.  Launches that share it run in stream
+// order; each split launch takes the next nonzero 32-bit epoch, so flag values
+// left by earlier launches never match.
+struct GemmSplit {
+  uint64_t* flags = nullptr;
+  int64_t n_flags = 0;
+  uint32_t epoch = 0;
+  int64_t last_ctas = 0;  // CTAs that shared the split tiles in the last launch (0: unsplit)
+};
+inline uint32_t next_split_epoch(GemmSplit* s) {
+  if (++s->epoch == 0) s->epoch = 1;
+  return s->epoch;
+}
+
 // C = A W^T; A map [>= m][k] with box rows 128.  The W map used is the one
-// whose box matches the tile width gemm_box_n(m, n, epilogue) selects.
+// whose box matches the tile width gemm_box_n(m, n, epilogue) selects.  With
+// `split`, the residual-add epilogue splits its last partial wave over k.
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
-                        const uint16_t* a_ptr = nullptr);
+                        const uint16_t* a_ptr = nullptr, GemmSplit* split = nullptr);
 
 // Few-row projections (decode steps; gemv.cu): A fp16 [m][k], W fp16 [n][k],
 // same epilogues as the GEMM; launch_gemm takes this path for m <= kGemvMaxRows

@@ -110,6 +110,8 @@ struct mzc_ctx {
   // stream and set by the copy engine after each copied run (from h_ones)
   int32_t* d_flags = nullptr;
   int32_t* h_ones = nullptr;
+  // order flags of the residual-add GEMMs whose last wave is split over k
+  mzc::GemmSplit gsplit;
   cudaEvent_t ev_clear = nullptr;
   bool restore_issued = false, lm_timed = false, ttft_from_copy = false;
   // per-class launch counts and optional CUDA-event timing
@@ -160,7 +162,7 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
                  ctx->d_cos,     ctx->d_sin,   ctx->d_x,       ctx->d_h,       ctx->d_qkv,
                  ctx->d_q,       ctx->d_attn,  ctx->d_act,     ctx->d_meta,    ctx->d_logits,
                  ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list,
-                 ctx->d_rstage[0], ctx->d_rstage[1], ctx->d_flags};
+                 ctx->d_rstage[0], ctx->d_rstage[1], ctx->d_flags, ctx->gsplit.flags};
   for (void* p : dev)
     if (p) cudaFree(p);
   void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging, ctx->h_ones};
@@ -401,6 +403,9 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   if (scratch > 0) CK(cudaMalloc(&ctx->d_scratch, scratch));
   CK(cudaMalloc(&ctx->d_status, 4));
   CK(cudaMemset(ctx->d_status, 0, 4));
+  ctx->gsplit.n_flags = std::max(ctx->num_sms, 256);
+  CK(cudaMalloc(&ctx->gsplit.flags, ctx->gsplit.n_flags * 8));
+  CK(cudaMemset(ctx->gsplit.flags, 0, ctx->gsplit.n_flags * 8));
   CK(cudaMalloc(&ctx->d_staging, ctx->nblk * ctx->block_bytes));
   if (ctx->codec != MZC_CODEC_NONE)
     for (auto& b : ctx->d_rstage) CK(cudaMalloc(&b, ctx->nblk * ctx->slot_bytes));
@@ -628,7 +633,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
                      [&] {
                        return mzc::launch_gemm(ta, w, out, cr, N, K, epi, ctx->d_status, cs,
-                                               static_cast<const uint16_t*>(a_ptr));
+                                               static_cast<const uint16_t*>(a_ptr), &ctx->gsplit);
                      });
     };
     // attention of chunk rows [r0, r0 + nr) (r0 relative to the chunk)
@@ -1352,10 +1357,10 @@ mzc_status mzc_profile_measure(mzc_ctx* ctx, mzc_profile* out) {
     auto layer_gemms = [&](int64_t m) -> cudaError_t {
       // (timing only: the activation buffers hold whatever the last prefill
       // left, so the GEMMs report nothing to the status word)
-      cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, nullptr, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_attn, W.tm_o, ctx->d_x, m, d, hq * hd, mzc::EPI_ADD_F32, nullptr, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, nullptr, ctx->cs);
-      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_act, W.tm_2, ctx->d_x, m, d, ctx->f_pad, mzc::EPI_ADD_F32, nullptr, ctx->cs);
+      cudaError_t e = mzc::launch_gemm(ctx->tm_h, W.tm_qkv, ctx->d_qkv, m, ctx->qkv_dim, d, mzc::EPI_STORE_BF16, nullptr, ctx->cs, nullptr, &ctx->gsplit);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_attn, W.tm_o, ctx->d_x, m, d, hq * hd, mzc::EPI_ADD_F32, nullptr, ctx->cs, nullptr, &ctx->gsplit);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_h, W.tm_13, ctx->d_act, m, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16, nullptr, ctx->cs, nullptr, &ctx->gsplit);
+      if (e == cudaSuccess) e = mzc::launch_gemm(ctx->tm_act, W.tm_2, ctx->d_x, m, d, ctx->f_pad, mzc::EPI_ADD_F32, nullptr, ctx->cs, nullptr, &ctx->gsplit);
       return e;
     };
     const int64_t sizes[3] = {128, 512, 2048};
@@ -1502,6 +1507,34 @@ mzc_status mzc_k_gemm(const uint16_t* a, const uint16_t* w, void* out, int64_t m
       !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
     return MZC_ERR_CUDA;
   KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, nullptr, static_cast<cudaStream_t>(stream), a));
+}
+
+mzc_status mzc_k_gemm_split(const uint16_t* a, const uint16_t* w, float* out, int64_t m, int64_t n,
+                            int64_t k, uint64_t* flags, int64_t n_flags, uint32_t epoch, int32_t* status,
+                            int64_t* split_ctas, void* stream) {
+  if (split_ctas) *split_ctas = 0;
+  if (!a || !w || !out || !flags || m < 0 || n <= 0 || k <= 0 || k % 8 != 0 || n % 16 != 0 ||
+      epoch == 0)
+    return MZC_ERR_INVALID;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return MZC_ERR_CUDA;
+  if (n_flags < sms) return MZC_ERR_INVALID;
+  if (m == 0) return MZC_OK;
+  CUtensorMap ta;
+  mzc::GemmWeight tw;
+  if (!mzc::make_tmap_f16(&ta, a, static_cast<uint64_t>(m), static_cast<uint64_t>(k), 128) ||
+      !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
+    return MZC_ERR_CUDA;
+  mzc::GemmSplit split;
+  split.flags = flags;
+  split.n_flags = n_flags;
+  split.epoch = epoch - 1;  // the launch takes the next one: `epoch`
+  const cudaError_t e = mzc::launch_gemm(ta, tw, out, m, n, k, mzc::EPI_ADD_F32, status,
+                                         static_cast<cudaStream_t>(stream), a, &split);
+  if (split_ctas) *split_ctas = split.last_ctas;
+  KCK(e);
 }
 
 mzc_status mzc_k_swiglu_pack(const uint16_t* gate, const uint16_t* up, int64_t f, int64_t d,

@@ -127,6 +127,8 @@ _SIGS = {
     "mzc_state_counts": [c_vp, P(mzc_stats_t)],
     "mzc_k_rmsnorm": [c_vp, c_vp, c_i64, c_i32, c_f32, c_vp, c_vp],
     "mzc_k_gemm": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_vp],
+    "mzc_k_gemm_split": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_vp, c_i64, ctypes.c_uint32, c_vp,
+                         c_vp, c_vp],
     "mzc_k_swiglu_pack": [c_vp, c_vp, c_i64, c_i64, c_vp],
     "mzc_k_rope_kv_write": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_i64,
                             c_vp, c_i64, c_i32, c_vp, c_vp, c_vp],
@@ -430,6 +432,15 @@ def mzc_k_rmsnorm(x, g, n, d, eps, y, stream=None):
 
 def mzc_k_gemm(a, w, out, m, n, k, epilogue, stream=None):
     return _call("mzc_k_gemm", _ptr(a), _ptr(w), _ptr(out), m, n, k, epilogue, stream)
+
+
+def mzc_k_gemm_split(a, w, out, m, n, k, flags, epoch, status=None, stream=None):
+    """Residual-add GEMM with the last wave split over k; returns the number
+    of CTAs that shared the split tiles (0 = ran unsplit)."""
+    ctas = ctypes.c_int64()
+    _call("mzc_k_gemm_split", _ptr(a), _ptr(w), _ptr(out), m, n, k, _ptr(flags), flags.numel(),
+          epoch, _ptr(status), ctypes.byref(ctas), stream)
+    return ctas.value
 
 
 def mzc_k_swiglu_pack(gate, up):

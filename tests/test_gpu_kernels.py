@@ -28,8 +28,11 @@ def _rand_bf16(tid, shape, sigma=1.0):
 # ---- GEMM (tcgen05 / TMEM / TMA) -------------------------------------------
 
 # m <= 4: the few-row GEMV path; larger m: the tcgen05 GEMM
+# m > 512: the paired-SM kernel (256 x 256 tiles over a CTA pair), with an odd
+# M-tile count (4224 rows: 33 tiles) and N not a multiple of 256 (384)
 GEMM_SHAPES = [(1, 64, 64), (2, 1024, 2048), (4, 3072, 3072), (7, 80, 72), (128, 256, 512),
-               (130, 384, 320), (300, 1024, 2048), (1000, 512, 256), (4224, 3072, 2048)]
+               (130, 384, 320), (300, 1024, 2048), (1000, 512, 256), (1000, 384, 320),
+               (4224, 3072, 2048)]
 
 
 def _act16(tid, shape):
@@ -52,7 +55,7 @@ def test_gemm_store_f16(mm, nn, kk):
 
 
 @pytest.mark.parametrize("mm,nn,kk", [(1, 2048, 8192), (3, 3072, 1024), (5, 64, 128), (200, 256, 768),
-                                     (4224, 2048, 2048)])
+                                     (1300, 640, 200), (4224, 2048, 2048)])
 def test_gemm_residual_add(mm, nn, kk):
     torch = _torch()
     a = _act16(3, (mm, kk))
@@ -68,7 +71,7 @@ def test_gemm_residual_add(mm, nn, kk):
 
 
 @pytest.mark.parametrize("mm,f,kk", [(1, 1024, 2048), (3, 128, 256), (4, 256, 512), (260, 384, 512),
-                                     (70, 704, 256),
+                                     (70, 704, 256), (900, 384, 512),
                                      (4224, 1024, 2048)])
 def test_gemm_swiglu(mm, f, kk):
     torch = _torch()
