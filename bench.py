@@ -540,7 +540,7 @@ def main():
     ap.add_argument("--workload", default="3b_sweep",
                     choices=["3b_sweep", "1b_recompute", "tiny", "3b_scattered_copy", "3b_mixed",
                              "3b_order", "1b_decode", "3b_decode", "3b_read_swapped", "link",
-                             "kernels"])
+                             "kernels", "projections"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--no-1b", action="store_true", help="3b_sweep: skip the 1B recompute keys")
@@ -569,13 +569,13 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     name = args.workload
-    if name in ("link", "kernels"):
+    if name in ("link", "kernels", "projections"):
         import torch
         if not torch.cuda.is_available():
             raise SystemExit("bench.py needs a CUDA GPU")
         import __graft_entry__
         __graft_entry__.build()
-        (run_link if name == "link" else run_kernels)(args)
+        {"link": run_link, "kernels": run_kernels, "projections": run_projections}[name](args)
         return
     sc = _workload(name)
     if args.fractions:
@@ -949,6 +949,55 @@ def run_kernels(args):
         out["kernels"][nm] = k
     torch.cuda.synchronize()
     assert int(status.item()) == 0
+    print(json.dumps(out), flush=True)
+
+
+PROJECTIONS = {  # name: (rows, n, k, epilogue) of one decoder layer's projections
+    "1b_qkv": (4224, 3072, 2048, 0), "1b_o": (4224, 2048, 2048, 1),
+    "1b_gate_up": (4224, 16384, 2048, 2), "1b_down": (4224, 2048, 8192, 1),
+    "3b_qkv": (2576, 5120, 3072, 0), "3b_o": (2576, 3072, 3072, 1),
+    "3b_gate_up": (2576, 16384, 3072, 2), "3b_down": (2576, 3072, 8192, 1),
+}
+
+
+def run_projections(args):
+    """The four projections of one decoder layer at the 1B recompute step's
+    4224 rows and at the 3B value step's 2576 rows (hybrid, f = 1), one launch
+    at a time through mzc_k_gemm: CUDA-event time per launch with L2 flushed
+    before each (a 512 MB write), FLOPs over that time against the measured
+    BF16 burst and sustained peaks.  Under 1.5 GB of device memory: also the
+    driver of the ncu captures of the GEMM kernels (tensor-pipe activity per
+    projection)."""
+    import torch
+    import paper_2609_01338_gb300 as m
+    peaks, src = _peaks()
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    gen = torch.Generator(device="cuda").manual_seed(0)
+    out = {"metric": "prefill projections alone: FLOPs over CUDA-event time, L2 flushed before each launch",
+           "peak_tflops_burst": peaks["bf16_tflops"], "peak_tflops_sustained": peaks["bf16_tflops_sustained"],
+           "peak_source": src, "projections": {}}
+    for name, (rows, n, k, epi) in PROJECTIONS.items():
+        a = (torch.randn((rows, k), device="cuda", generator=gen) * 0.5).half().view(torch.int16)
+        w = (torch.randn((n, k), device="cuda", generator=gen) * 0.02).half().view(torch.int16)
+        o = (torch.zeros((rows, n), device="cuda") if epi == 1 else
+             torch.empty((rows, n // 2 if epi == 2 else n), dtype=torch.int16, device="cuda"))
+        ts = []
+        for i in range(max(1, args.warmup) + max(1, args.steps)):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            m.mzc_k_gemm(a, w, o, rows, n, k, epi)
+            e1.record()
+            e1.synchronize()
+            if i >= max(1, args.warmup):
+                ts.append(e0.elapsed_time(e1))
+        ms = statistics.median(ts)
+        tf = 2.0 * rows * n * k / (ms * 1e-3) / 1e12
+        out["projections"][name] = {
+            "rows": rows, "n": n, "k": k, "us": round(ms * 1e3, 2), "tflops": round(tf, 1),
+            "frac_sustained": round(tf / peaks["bf16_tflops_sustained"], 4),
+            "frac_burst": round(tf / peaks["bf16_tflops"], 4)}
+        del a, w, o
     print(json.dumps(out), flush=True)
 
 
