@@ -284,6 +284,50 @@ def test_q8_swap_overlapped_with_prompt_matches_sync_restore(tiny):
     assert np.array_equal(outs[0], outs[1])
 
 
+def test_q8_copies_with_recomputed_tail(tiny):
+    """8-bit copies of [256, 384) restored while the dropped tail [384, 512)
+    is recomputed and the prompt runs: the copies hold the oracle's decode of
+    its encoding, the logits equal the restore-first run bit for bit and the
+    oracle's forward of the tail and the prompt over the decoded copies; a
+    sync with copies pending and nothing to recompute decodes them too."""
+    sh, w, L = tiny["shape"], tiny["w"], tiny["shape"]["n_layers"]
+    e = 2 * sh["n_kv_heads"] * 16 * sh["head_dim"]
+    blocks = [(l, b) for l in range(L) for b in range(16, 24)]  # positions [256, 384)
+
+    def read(c):
+        return np.stack([np.concatenate(m.mzc_read_kv(c, l, b, sh)) for l, b in blocks])
+
+    outs = []
+    for overlap in (1, 0):
+        c = _new(tiny, swap_codec=m.MZC_CODEC_Q8, overlap=overlap)
+        m.mzc_prefill(c, tiny["ctx"])
+        want = oracle.q8_decode_blocks(oracle.q8_encode_blocks(read(c)), e, sh["kv_dtype"])
+        m.mzc_evict(c, 0, L, 384, 512, m.MZC_DROP)
+        m.mzc_evict(c, 0, L, 256, 384, m.MZC_COPY)
+        m.mzc_restore_async(c)
+        m.mzc_recompute_tail(c, 384, 128)
+        outs.append(_logits(tiny, c, tiny["prm"]))
+        assert np.array_equal(read(c), want)
+        if overlap:
+            k, v = m.mzc_read_kv_all(c, 384, sh)
+            kv = oracle.KVState(sh, sh["max_ctx"])
+            kv.k[:, :384], kv.v[:, :384] = k, v
+            toks = np.concatenate([tiny["ctx"][384:512], tiny["prm"]])
+            ref = oracle.forward(sh, w, kv, toks, np.arange(384, 544))
+        m.mzc_destroy(c)
+    assert np.array_equal(outs[0], outs[1])
+    assert np.max(np.abs(outs[0] - ref)) < LOGIT_TOL
+    # copies pending at a sync with nothing to recompute: decoded by the sync
+    c = _new(tiny, swap_codec=m.MZC_CODEC_Q8)
+    m.mzc_prefill(c, tiny["ctx"])
+    want = oracle.q8_decode_blocks(oracle.q8_encode_blocks(read(c)), e, sh["kv_dtype"])
+    m.mzc_evict(c, 0, L, 0, 512, m.MZC_COPY)
+    m.mzc_restore_async(c)
+    m.mzc_sync(c)
+    assert np.array_equal(read(c), want)
+    m.mzc_destroy(c)
+
+
 def test_decode_steps_match_oracle(tiny):
     """Decode after the first token: single-token steps (the few-row GEMV
     projections, one-row attention) match the oracle's forward of the same
