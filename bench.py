@@ -703,9 +703,13 @@ def run_headline(r, args, rank, world, local, dist):
     clk = Clocks(local)
     t_all = time.perf_counter()
     pts, head = [], None
+    # the value point: HEADLINE, or the first point when --fractions /
+    # --policies leave it out (a partial sweep, e.g. for a profiler run)
+    grid = [(f, p) for f in sc["fractions"] for p in sc["policies"]]
+    vp = HEADLINE if HEADLINE in grid else grid[0]
     for frac in sc["fractions"]:
         for pol in sc["policies"]:
-            is_head = (frac, pol) == HEADLINE
+            is_head = (frac, pol) == vp
             # the value point also takes the roofline steps; every point times
             # its kernel classes in the last warm-up step
             res = _timed_workload(r, args, dist if is_head else None, name,
@@ -757,8 +761,6 @@ def run_headline(r, args, rank, world, local, dist):
         r1.close()
         del r1
     clocks = clk.stop()
-    if head is None:
-        raise SystemExit(f"the sweep has no {HEADLINE[1]} point at f = {HEADLINE[0]}")
     v, e2e = max_over_ranks([statistics.median(head["dev"]), statistics.median(head["host"])], dist, "cuda")
     st = head["st"]
     line = {
@@ -767,7 +769,8 @@ def run_headline(r, args, rank, world, local, dist):
         "ms_per_step": round(statistics.mean(head["dev"]), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": _config(name, sc, args.codec, world, args.wait_mode),
+        "config": {**_config(name, sc, args.codec, world, args.wait_mode),
+                   "value_point": {"fraction": vp[0], "policy": vp[1]}},
         "sweep": sweep, "hybrid_vs_policies": vs, "points": pts, "profile": prof,
         "roofline": _roofline(head["ks"], head["dom"], peaks, src, name),
         **line_extra,
