@@ -358,23 +358,26 @@ def _oracle_step(name, sc, idx):
 def _sample_note(name, sc, n_rows, total, extra=""):
     sh = sc["model"]
     _, copy_bytes = _oracle_rows(name, sc)
-    return (f"{n_rows} of {total} rows (evenly spaced over the step's recomputed tail and prompt) "
-            f"through all {sh['n_layers']} layers over a KV-conditioned state of "
-            f"{sc['context'] + sc['prompt']} positions, scaled x{total / n_rows:.1f} (extrapolated), "
+    rows = (f"all {total} rows of the step (unsampled)" if n_rows >= total else
+            f"{n_rows} of {total} rows (evenly spaced over the step's recomputed tail and prompt)")
+    scale = "" if n_rows >= total else f", scaled x{total / n_rows:.1f} (extrapolated)"
+    return (f"{rows} through all {sh['n_layers']} layers over a KV-conditioned state of "
+            f"{sc['context'] + sc['prompt']} positions{scale}, "
             f"plus one LM-head row and a host memcpy of the {copy_bytes / 1e9:.2f} GB the step restores "
             f"by copy{extra}")
 
 
-def cpu_baseline(name, sc):
+def cpu_baseline(name, sc, full=False):
     """The oracle on the GPU machine's host cores: 4 x cores rows of the step
-    (every core busy), a 1-thread time on 2 rows, the CPU model, and the tiny
-    workload run unsampled."""
+    (every core busy), or every row with `full` (minutes at 1B scale), a
+    1-thread time on 2 rows, the CPU model, and the tiny workload run
+    unsampled."""
     import oracle
     oracle.build()
     cores = oracle.num_threads()
     pos, _ = _oracle_rows(name, sc)
     # the tiny workload runs whole (a small sample would be mostly per-call cost)
-    n = pos.size if name == "tiny" else min(pos.size, 4 * cores)
+    n = pos.size if (name == "tiny" or full) else min(pos.size, 4 * cores)
     idx = np.unique(np.linspace(0, pos.size - 1, n).astype(int))
     ms, wall, total = _oracle_step(name, sc, idx)
     oracle.set_num_threads(1)
@@ -542,6 +545,9 @@ def main():
                              "3b_order", "1b_decode", "3b_decode", "3b_read_swapped", "link",
                              "kernels", "projections"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-full", action="store_true",
+                    help="time the oracle on every row of the step, unsampled (about 4 minutes "
+                         "for 1b_recompute on 16 cores), instead of a 4 x cores-row sample")
     ap.add_argument("--no-kernel-timing", action="store_true")
     ap.add_argument("--no-1b", action="store_true", help="3b_sweep: skip the 1B recompute keys")
     ap.add_argument("--fractions", default=None, help="comma list overriding the sweep's fractions")
@@ -629,7 +635,7 @@ def main():
     r.close()
     del r
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(name, sc)
+        line["cpu_baseline"] = cpu_baseline(name, sc, args.cpu_full)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:
@@ -790,7 +796,7 @@ def run_headline(r, args, rank, world, local, dist):
             "tensor_peak_frac_attention_burst", "kernel_ms_per_step", "roofline", "e2e", "gpu_launches")}
         line["recompute_1b"]["workload"] = l1["config"]["workload"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(name, sc)
+        line["cpu_baseline"] = cpu_baseline(name, sc, args.cpu_full)
     if rank == 0:
         print(json.dumps(line), flush=True)
 
