@@ -17,6 +17,12 @@
 // one fp32 add per element as in a read-modify-write).  The output tensor map
 // spans exactly m rows and n columns, so rows >= m (computed on whatever the A
 // buffer holds) are clipped by the TMA unit.
+//
+// Two kernels: the single-CTA persistent kernel (gemm_persistent_kernel) and,
+// for the tensor-bound projections above 512 rows, the paired-SM kernel
+// (gemm_pair_kernel: 256 x 256 tiles over the two CTAs of a cluster with
+// tcgen05.mma.cta_group::2, each CTA staging only its own A rows and half of
+// the W k-block).  Both share the epilogue (EpiWarp).
 #include <cstdio>
 #include <mutex>
 
