@@ -964,15 +964,20 @@ mzc_status mzc_restore_async(mzc_ctx* ctx) {
   CK(cudaSetDevice(ctx->opt.device));
   std::vector<mzc_copy_run> runs;
   std::vector<int32_t> wl;
-  mzc_status s = ctx->st.plan_restore(&runs, &wl);
-  if (s != MZC_OK) return ctx->from_state(s);
-  if (!ctx->st.restore_in_flight()) return MZC_OK;
-  cudaStream_t xs = ctx->xs;
-  CK(cudaEventRecord(ctx->ev_c0, xs));
   // per-block flags: the destination blocks read as absent from here on (their
   // flags are cleared on the compute stream, ahead of any attention of the
   // next prefill); the copy stream sets each run's flags after its data
   const bool set_flags = ctx->d_flags && ctx->opt.overlap && ctx->codec == MZC_CODEC_NONE;
+  // The plan is made a layer at a time, each layer's copies issued before the
+  // next layer is planned, so the first copy leaves as soon as its layer is
+  // planned.  With per-block flags every destination is planned first: the
+  // flags are cleared before any copy.
+  bool any = false;
+  mzc_status s = set_flags ? ctx->st.plan_restore(&runs, &wl) : ctx->st.begin_restore(&any);
+  if (s != MZC_OK) return ctx->from_state(s);
+  if (!ctx->st.restore_in_flight()) return MZC_OK;
+  cudaStream_t xs = ctx->xs;
+  CK(cudaEventRecord(ctx->ev_c0, xs));
   if (set_flags && !runs.empty()) {
     for (const mzc_copy_run& r : runs)
       CK(cudaMemsetAsync(ctx->d_flags + r.phys_begin, 0, static_cast<size_t>(r.n_blocks) * 4, ctx->cs));
@@ -982,6 +987,11 @@ mzc_status mzc_restore_async(mzc_ctx* ctx) {
   size_t ri = 0, wi = 0;
   int64_t bytes = 0, copies = 0;
   for (int32_t l = 0; l < ctx->shape.n_layers; ++l) {
+    if (!set_flags) {
+      bool w = false;
+      ctx->st.plan_restore_layer(l, &runs, &w);
+      if (w) wl.push_back(l);
+    }
     if (wi < wl.size() && wl[wi] == l) {
       const LayerDev& Ld = ctx->layers[l];
       CK(cudaMemcpyAsync(Ld.base, Ld.host_master, Ld.bytes, cudaMemcpyHostToDevice, xs));

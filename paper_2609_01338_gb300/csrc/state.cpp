@@ -273,7 +273,8 @@ mzc_status State::recompute_tail(int64_t p, int64_t n) {
   return MZC_OK;
 }
 
-mzc_status State::plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int32_t>* weight_layers) {
+mzc_status State::begin_restore(bool* any) {
+  *any = false;
   if (inflight_) return fail(MZC_ERR_STATE, "a restore is already in flight");
   const int32_t L = shape_.n_layers;
   const int64_t nb = ceil_div(n_ctx_, 16);
@@ -281,46 +282,61 @@ mzc_status State::plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int3
   for (int32_t l = 0; l < L; ++l)
     for (int64_t b = 0; b < nb; ++b) need += at(l, b).st == MZC_SWAPPED;
   if (need > pool_.free_total()) return fail(MZC_ERR_OOM, "KV pool cannot hold the restored blocks");
-  if (runs) runs->clear();
-  if (weight_layers) weight_layers->clear();
-  bool any = false;
-  for (int32_t l = 0; l < L; ++l) {  // forward-in: earliest layer first
-    if (w_state_[l] == MZC_SWAPPED) {
-      w_state_[l] = MZC_INFLIGHT;
-      if (weight_layers) weight_layers->push_back(l);
-      any = true;
-    }
-    // swapped blocks of layer l grouped by region, slot order
-    std::map<int32_t, std::vector<int64_t>> by_region;
-    for (int64_t b = 0; b < nb; ++b)
-      if (at(l, b).st == MZC_SWAPPED) by_region[at(l, b).region].push_back(b);
-    for (auto& kv : by_region) {
-      const Region& R = regions_[kv.first];
-      auto& blocks = kv.second;  // ascending logical index == ascending slot
-      auto ranges = pool_.alloc_runs((int64_t)blocks.size());
-      size_t bi = 0;
-      for (auto& rg : ranges) {
-        for (int64_t j = 0; j < rg.second; ++j, ++bi) {
-          BlockEntry& e = at(l, blocks[bi]);
-          e.st = MZC_INFLIGHT;
-          e.phys = (int32_t)(rg.first + j);
-          int64_t off = R.host_off + (int64_t)e.idx * slot_bytes_;
-          // extend the previous run when host and device are both contiguous
-          if (runs && !runs->empty()) {
-            mzc_copy_run& pr = runs->back();
-            if (pr.layer == l && pr.phys_begin + pr.n_blocks == e.phys &&
-                pr.host_off + (int64_t)pr.n_blocks * slot_bytes_ == off) {
-              pr.n_blocks += 1;
-              continue;
-            }
+  bool w = false;
+  for (int32_t l = 0; l < L; ++l) w = w || w_state_[l] == MZC_SWAPPED;
+  *any = need > 0 || w;
+  inflight_ = *any;
+  return MZC_OK;
+}
+
+void State::plan_restore_layer(int32_t l, std::vector<mzc_copy_run>* runs, bool* weight) {
+  const int64_t nb = ceil_div(n_ctx_, 16);
+  *weight = false;
+  if (w_state_[l] == MZC_SWAPPED) {
+    w_state_[l] = MZC_INFLIGHT;
+    *weight = true;
+  }
+  // swapped blocks of layer l grouped by region, slot order
+  std::map<int32_t, std::vector<int64_t>> by_region;
+  for (int64_t b = 0; b < nb; ++b)
+    if (at(l, b).st == MZC_SWAPPED) by_region[at(l, b).region].push_back(b);
+  for (auto& kv : by_region) {
+    const Region& R = regions_[kv.first];
+    auto& blocks = kv.second;  // ascending logical index == ascending slot
+    auto ranges = pool_.alloc_runs((int64_t)blocks.size());
+    size_t bi = 0;
+    for (auto& rg : ranges) {
+      for (int64_t j = 0; j < rg.second; ++j, ++bi) {
+        BlockEntry& e = at(l, blocks[bi]);
+        e.st = MZC_INFLIGHT;
+        e.phys = (int32_t)(rg.first + j);
+        int64_t off = R.host_off + (int64_t)e.idx * slot_bytes_;
+        // extend the previous run when host and device are both contiguous
+        if (runs && !runs->empty()) {
+          mzc_copy_run& pr = runs->back();
+          if (pr.layer == l && pr.phys_begin + pr.n_blocks == e.phys &&
+              pr.host_off + (int64_t)pr.n_blocks * slot_bytes_ == off) {
+            pr.n_blocks += 1;
+            continue;
           }
-          if (runs) runs->push_back(mzc_copy_run{l, 1, off, (int64_t)e.phys});
         }
+        if (runs) runs->push_back(mzc_copy_run{l, 1, off, (int64_t)e.phys});
       }
-      any = true;
     }
   }
-  inflight_ = any;
+}
+
+mzc_status State::plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int32_t>* weight_layers) {
+  bool any = false;
+  mzc_status s = begin_restore(&any);
+  if (s != MZC_OK) return s;
+  if (runs) runs->clear();
+  if (weight_layers) weight_layers->clear();
+  for (int32_t l = 0; any && l < shape_.n_layers; ++l) {  // forward-in: earliest layer first
+    bool w = false;
+    plan_restore_layer(l, runs, &w);
+    if (w && weight_layers) weight_layers->push_back(l);
+  }
   return MZC_OK;
 }
 

@@ -110,6 +110,13 @@ class State {
   // Forward-in restore plan of every swapped block and weight unit; swapped
   // blocks become INFLIGHT with their destination physical block assigned.
   mzc_status plan_restore(std::vector<mzc_copy_run>* runs, std::vector<int32_t>* weight_layers);
+  // The same plan a layer at a time, so that a caller can issue layer l's
+  // copies before it plans layer l + 1: begin_restore validates the whole
+  // restore (the pool holds every swapped block) and marks it in flight when
+  // there is anything to restore (*any); then plan_restore_layer(l) for l = 0,
+  // 1, ... appends layer l's runs and sets *weight when its weights come back.
+  mzc_status begin_restore(bool* any);
+  void plan_restore_layer(int32_t l, std::vector<mzc_copy_run>* runs, bool* weight);
   bool restore_in_flight() const { return inflight_; }
 
   // Validates a prefill of n_prompt new tokens and allocates the blocks its
