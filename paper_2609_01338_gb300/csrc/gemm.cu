@@ -332,7 +332,23 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // the prologue above touches no memory another kernel writes
+  // The prologue above touches no memory another kernel writes.  Neither do
+  // the weights: the producer issues the W loads of its first tile's first
+  // stages before it waits for the previous kernel (whose output A is), so
+  // weight streaming starts under that kernel's tail.
+  int pre = 0;
+  if (warp == 0 && lane == 0) {
+    WorkItem w0;
+    if (sched_item(sched, 0, &w0)) {
+      int mt0, nt0;
+      tile_coords(w0.tile, num_m, num_n, band, &mt0, &nt0);
+      pre = min(STAGES, w0.kb1 - w0.kb0);
+      for (int i = 0; i < pre; ++i) {
+        mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
+        tma_load_2d(sB + i * C::B_BYTES, &tmw, &full[i], (w0.kb0 + i) * BK, nt0 * BN);
+      }
+    }
+  }
   pdl_enter();
   const uint32_t tmem = s_tmem;
 
@@ -351,9 +367,9 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+          if (it >= pre) mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);  // else done above
           tma_load_2d(sA + s * C::A_BYTES, &tma, &full[s], kb * BK, mt * BM);
-          tma_load_2d(sB + s * C::B_BYTES, &tmw, &full[s], kb * BK, nt * BN);
+          if (it >= pre) tma_load_2d(sB + s * C::B_BYTES, &tmw, &full[s], kb * BK, nt * BN);
         }
       }
       // drain the last fill of every ring slot before shared memory is
@@ -559,7 +575,20 @@ __global__ void __launch_bounds__(192, 1) gemm_pair_kernel(
   // both CTAs' barriers are initialised before either arrives on the other's
   cluster_sync_all();
   tc_fence_after();
-  // the prologue above touches no memory another kernel writes
+  // The prologue above touches no memory another kernel writes.  Neither do
+  // the weights: each producer issues its W half of the first unit's first
+  // stages before it waits for the previous kernel (whose output A is).
+  int pre = 0;
+  if (warp == 0 && lane == 0 && cid < units) {
+    int mp0, nt0;
+    tile_coords(cid, unit_m, num_n, band, &mp0, &nt0);
+    pre = min(S, num_k);
+    const uint32_t full0 = map_rank(smem_u32(full), 0);
+    for (int i = 0; i < pre; ++i) {
+      if (rank == 0) mbar_arrive_expect_tx(&full[i], 2 * C::STAGE_BYTES);
+      tma_load_2d_pair(sB + i * C::B_BYTES, &tmw, full0 + i * 8, i * BK, nt0 * BN + rank * 128);
+    }
+  }
   pdl_enter();
   const uint32_t tmem = s_tmem;
 
@@ -579,9 +608,9 @@ __global__ void __launch_bounds__(192, 1) gemm_pair_kernel(
             ok = false;
             break;
           }
-          if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * C::STAGE_BYTES);
+          if (rank == 0 && it >= pre) mbar_arrive_expect_tx(&full[s], 2 * C::STAGE_BYTES);
           tma_load_2d_pair(sA + s * C::A_BYTES, &tma, full0 + s * 8, kb * BK, mt * BM);
-          tma_load_2d_pair(sB + s * C::B_BYTES, &tmw, full0 + s * 8, kb * BK, nt * BN + rank * 128);
+          if (it >= pre) tma_load_2d_pair(sB + s * C::B_BYTES, &tmw, full0 + s * 8, kb * BK, nt * BN + rank * 128);
         }
       }
       // every fill issued (by both CTAs) has landed before shared memory is

@@ -111,7 +111,15 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // the prologue above touches no memory another kernel writes
+  // The prologue above touches no memory another kernel writes.  Neither do
+  // the weights: the producer issues the first stages' W loads before it waits
+  // for the previous kernel (whose output A is), so weight streaming starts
+  // under that kernel's tail.
+  const int pre = (warp == 0 && lane == 0) ? min(STAGES, kb1 - kb0) : 0;
+  for (int i = 0; i < pre; ++i) {
+    mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
+    tma_load_2d(smem + i * C::STAGE_BYTES + MT * C::A_BYTES, &tmw, &full[i], (kb0 + i) * SBK, nt * SBN);
+  }
   pdl_enter();
   const uint32_t tmem = s_tmem;
 
@@ -127,10 +135,10 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
           break;
         }
         uint8_t* base = smem + st * C::STAGE_BYTES;
-        mbar_arrive_expect_tx(&full[st], C::STAGE_BYTES);
+        if (it >= pre) mbar_arrive_expect_tx(&full[st], C::STAGE_BYTES);  // else done above
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) tma_load_2d(base + mt * C::A_BYTES, &tma, &full[st], kb * SBK, mt * SBM);
-        tma_load_2d(base + MT * C::A_BYTES, &tmw, &full[st], kb * SBK, nt * SBN);
+        if (it >= pre) tma_load_2d(base + MT * C::A_BYTES, &tmw, &full[st], kb * SBK, nt * SBN);
       }
       // every fill issued has landed before the ring is reused for the partial
       for (int i = it - STAGES < 0 ? 0 : it - STAGES; i < it; ++i)
