@@ -230,9 +230,28 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     tma_prefetch_desc(&pool_run);
     tma_prefetch_desc(&pool_blk);
   }
-  if (warp == C::PRODUCER_WARP) tmem_alloc(&s_tmem, C::TMEM_COLS);
+  if (warp == C::PRODUCER_WARP) {
+    tmem_alloc(&s_tmem, C::TMEM_COLS);
+    tc_fence_before();  // the TMEM address, read by the other warps after the barrier below
+  }
   // the prologue above touches no memory another kernel writes
   pdl_enter();
+
+  // the producer finds the key range itself (the largest position of the
+  // CTA's rows) and reads the first key tile's block-table entries while the
+  // softmax warps load Q, so the first K/V fetch does not wait for Q
+  int prod_kv_len = 0;
+  int32_t prod_tab0 = -1;
+  if (warp == C::PRODUCER_WARP) {
+    const int t_lo = r0 / group, t_hi = (min(R, r0 + C::ROWS) - 1) / group;
+    int mp = -1;
+    for (int t = t_lo + lane; t <= t_hi; t += 32) mp = max(mp, pos[t]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mp = max(mp, __shfl_xor_sync(0xffffffffu, mp, off));
+    prod_kv_len = mp + 1;
+    const int64_t blk0 = static_cast<int64_t>(split * keys_per_split) / 16 + lane;
+    if (lane < BN / 16 && blk0 < n_logical) prod_tab0 = table[blk0];
+  }
 
   // softmax threads: tile and row; the Q tiles in the UMMA K-major layout
   const int qt = tid >> 7;  // Q tile of the softmax warps
@@ -253,17 +272,21 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     }
     cp_async_commit();
   }
-  __syncthreads();
-  if (warp < C::PRODUCER_WARP && row_pos >= 0) atomicMax(&s_maxpos, row_pos);
-  if (warp < C::PRODUCER_WARP) {
-    cp_async_wait<0>();
-    fence_async_smem();  // Q (generic-proxy writes) visible to the tensor core
+  __syncthreads();  // barriers initialised, TMEM allocated
+  int kv_len = prod_kv_len;
+  if (warp != C::PRODUCER_WARP) {
+    if (row_pos >= 0) atomicMax(&s_maxpos, row_pos);
+    if (warp < C::PRODUCER_WARP) {
+      cp_async_wait<0>();
+      fence_async_smem();  // Q (generic-proxy writes) visible to the tensor core
+    }
+    tc_fence_before();
+    // the softmax and UMMA warps only: Q loaded and every row position seen
+    asm volatile("bar.sync 1, %0;" ::"n"(C::THREADS - 32) : "memory");
+    kv_len = s_maxpos + 1;
   }
-  tc_fence_before();
-  __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  const int kv_len = s_maxpos + 1;
   const int k_begin = split * keys_per_split;
   const int k_end = min(kv_len, k_begin + keys_per_split);
   const int T = k_end > k_begin ? (k_end - k_begin + BN - 1) / BN : 0;
@@ -288,7 +311,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
       auto flag_of = [&](int32_t pb) -> int32_t {
         return (flags == nullptr || pb < 0 || pb >= pool_blocks) ? 1 : ld_acquire_gpu(flags + pb);
       };
-      int32_t p_cur = lookup(0);
+      // tile 0's entries were read before the barrier
+      int32_t p_cur = (lane >= NB || k_begin + lane * 16 >= k_end) ? kPast : prod_tab0;
       int32_t f_cur = flag_of(p_cur);
       int issued = 0;
       for (int j = 0; j < T; ++j) {
@@ -583,35 +607,106 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, AttnCfg<HD>::CTAS_PER_SM
     const float o_scale = l > 0.0f ? 1.0f / l : 0.0f;
     const int t = rr / group, h = g * group + rr % group;
     const int64_t orow = static_cast<int64_t>(t) * hq + h;
-#pragma unroll
-    for (int c = 0; c < HD; c += 64) {
-      float o[64];
-      if (have_o) {
-        tmem_ld64w(trow + o_col + c, o);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 64; ++i) o[i] = 0.0f;
-      }
-      if (rr < R) {
-        if (n_splits == 1) {
-          uint4* dst = reinterpret_cast<uint4*>(out + orow * HD + c);
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            dst[u] = make_uint4(pack2<true>(o[8 * u] * o_scale, o[8 * u + 1] * o_scale),
-                                pack2<true>(o[8 * u + 2] * o_scale, o[8 * u + 3] * o_scale),
-                                pack2<true>(o[8 * u + 4] * o_scale, o[8 * u + 5] * o_scale),
-                                pack2<true>(o[8 * u + 6] * o_scale, o[8 * u + 7] * o_scale));
-        } else {
-          float4* dst = reinterpret_cast<float4*>(
-              part_o + (static_cast<int64_t>(split) * n * hq + orow) * HD + c);
-#pragma unroll
-          for (int u = 0; u < 16; ++u)
-            dst[u] = make_float4(o[4 * u] * o_scale, o[4 * u + 1] * o_scale, o[4 * u + 2] * o_scale,
-                                 o[4 * u + 3] * o_scale);
+    // At head dim 128 the warp's 32 rows go through its quarter of the
+    // tile's Q shared memory (every UMMA that reads it has completed: S(Tq-1)
+    // before the softmax loaded it), HD x 2 bytes a row per pass, 16-byte
+    // units XOR-swizzled by row; then each store instruction writes whole
+    // rows, where a thread storing its own row touches 32 rows per
+    // instruction (measured 1-3% faster at head dim 128, 2% slower at 64,
+    // whose kernel is short of registers).  After an abort the tile's UMMAs
+    // may still read Q, and nothing is written.
+    constexpr int U = HD / 8;  // 16-byte units of a staged row
+    uint4* stg = reinterpret_cast<uint4*>(sQ + qt * C::Q_BYTES) + (warp & 3) * 32 * U;
+    const int wr0 = r0 + qt * C::BM + (warp & 3) * 32;  // tile row of lane 0
+    const bool write_rows = Tq == 0 || have_o;
+    auto store_rows = [&](auto dst_row) {
+      __syncwarp();
+#pragma unroll 4
+      for (int it = 0; it < U; ++it) {
+        const int k = it * 32 + lane, rw = k / U, un = k % U;
+        const int rrw = wr0 + rw;
+        if (rrw < R) {
+          const int64_t orw = static_cast<int64_t>(rrw / group) * hq + g * group + rrw % group;
+          dst_row(orw)[un] = stg[rw * U + (un ^ (rw & (U - 1)))];
         }
       }
+      __syncwarp();
+    };
+    if (HD == 64 && write_rows) {
+#pragma unroll
+      for (int c = 0; c < HD; c += 64) {
+        float o[64];
+        if (have_o) {
+          tmem_ld64w(trow + o_col + c, o);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 64; ++i) o[i] = 0.0f;
+        }
+        if (rr < R) {
+          if (n_splits == 1) {
+            uint4* dst = reinterpret_cast<uint4*>(out + orow * HD + c);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              dst[u] = make_uint4(pack2<true>(o[8 * u] * o_scale, o[8 * u + 1] * o_scale),
+                                  pack2<true>(o[8 * u + 2] * o_scale, o[8 * u + 3] * o_scale),
+                                  pack2<true>(o[8 * u + 4] * o_scale, o[8 * u + 5] * o_scale),
+                                  pack2<true>(o[8 * u + 6] * o_scale, o[8 * u + 7] * o_scale));
+          } else {
+            float4* dst = reinterpret_cast<float4*>(
+                part_o + (static_cast<int64_t>(split) * n * hq + orow) * HD + c);
+#pragma unroll
+            for (int u = 0; u < 16; ++u)
+              dst[u] = make_float4(o[4 * u] * o_scale, o[4 * u + 1] * o_scale,
+                                   o[4 * u + 2] * o_scale, o[4 * u + 3] * o_scale);
+          }
+        }
+      }
+    } else if (write_rows && n_splits == 1) {
+#pragma unroll
+      for (int c = 0; c < HD; c += 64) {
+        float o[64];
+        if (have_o) {
+          tmem_ld64w(trow + o_col + c, o);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 64; ++i) o[i] = 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          stg[lane * U + ((c / 8 + u) ^ (lane & (U - 1)))] =
+              make_uint4(pack2<true>(o[8 * u] * o_scale, o[8 * u + 1] * o_scale),
+                         pack2<true>(o[8 * u + 2] * o_scale, o[8 * u + 3] * o_scale),
+                         pack2<true>(o[8 * u + 4] * o_scale, o[8 * u + 5] * o_scale),
+                         pack2<true>(o[8 * u + 6] * o_scale, o[8 * u + 7] * o_scale));
+      }
+      store_rows([&](int64_t orw) { return reinterpret_cast<uint4*>(out + orw * HD); });
+    } else if (write_rows) {
+      // fp32 partials: two passes of HD/2 columns
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float o[HD / 2];
+        if (have_o) {
+          if constexpr (HD == 128) {
+            tmem_ld64w(trow + o_col + half * 64, o);
+          } else {
+            tmem_ld32w(trow + o_col + half * 32, o);  // not reached: head dim 64 stores directly
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < HD / 2; ++i) o[i] = 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          stg[lane * U + (u ^ (lane & (U - 1)))] = make_uint4(
+              __float_as_uint(o[4 * u] * o_scale), __float_as_uint(o[4 * u + 1] * o_scale),
+              __float_as_uint(o[4 * u + 2] * o_scale), __float_as_uint(o[4 * u + 3] * o_scale));
+        store_rows([&](int64_t orw) {
+          return reinterpret_cast<uint4*>(part_o + (static_cast<int64_t>(split) * n * hq + orw) * HD +
+                                          half * (HD / 2));
+        });
+      }
     }
-    if (rr < R && n_splits > 1)
+    if (write_rows && rr < R && n_splits > 1)
       part_lse[static_cast<int64_t>(split) * n * hq + orow] = l > 0.0f ? m_ref + log2f(l) : -INFINITY;
   }
 

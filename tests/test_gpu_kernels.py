@@ -333,6 +333,20 @@ def test_attention_split_kv_long_context(hq, hkv, hd, kvd):
     assert rel_err(got2, ref2) < 1e-2
 
 
+@pytest.mark.parametrize("hq,hkv,hd,kvd,n", [(24, 8, 128, 0, 128), (32, 8, 64, 1, 96),
+                                             (24, 8, 128, 1, 171)])
+def test_attention_split_kv_half_last_row_tile(hq, hkv, hd, kvd, n):
+    """A prompt whose rows per KV head (n x hq/hkv) leave the last 256-row
+    tile with one Q tile of two (or a single row), split over the keys: the
+    padding Q tile gets no work and every real row is merged over all splits."""
+    ctx = 4224 + n
+    pos = np.arange(ctx - n, ctx).astype(np.int32)  # the prompt's diagonal is in every split's reach
+    got, ref, sb = _attention_case(hq, hkv, hd, kvd, ctx, pos, seed=n)
+    assert sb > 0  # the split path ran
+    assert rel_err(got, ref) < 1e-2
+    assert np.mean(np.abs(got - ref)) < 2e-3 * np.max(np.abs(ref))
+
+
 @pytest.mark.parametrize("hq,hkv,hd,kvd,n,ctx", [
     (32, 8, 64, 1, 1, 8197),     # 1B decode token: 4 rows per KV head, split-KV, ragged end
     (32, 8, 64, 1, 1, 70_000),   # more than 32 blocks per warp pair and split
