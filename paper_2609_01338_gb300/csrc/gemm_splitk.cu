@@ -13,10 +13,11 @@
 //   - the epilogue warps copy the fp32 partial to shared memory (the ring is
 //     free by then) and the cluster synchronises;
 //   - CTA s then sums rows [s*RS, (s+1)*RS) of the S partials, read through
-//     distributed shared memory in split order (the same sum on every run),
-//     applies the epilogue (fp16 store, fp32 residual add, SwiGLU) and writes
-//     the rows out; a second cluster barrier keeps every partial alive until
-//     all CTAs have read it.
+//     distributed shared memory in split order (the same sum on every run;
+//     all threads, several row chunks' loads in flight per thread), applies
+//     the epilogue (fp16 store, fp32 residual add, SwiGLU) and writes the
+//     rows out; a second cluster barrier keeps every partial alive until all
+//     CTAs have read it.
 // Every thread of every CTA passes both cluster barriers exactly once (no
 // early exit on any path); the pipeline waits are bounded as elsewhere.
 #include <algorithm>
@@ -30,6 +31,10 @@ namespace mzc {
 namespace {
 
 constexpr int SBM = 128, SBN = 128, SBK = 64;
+// row chunks whose remote loads each thread has in flight in the reduction
+#ifndef MZC_SK_ITEMS
+#define MZC_SK_ITEMS 2
+#endif
 
 template <int MT>
 struct SKCfg {
@@ -205,69 +210,88 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   // ---- every partial of the cluster is in shared memory ----
   cluster_sync_all();
 
-  if (warp >= 2) {
-    // ---- rows [s*RS, (s+1)*RS) summed over the S partials in split order ----
+  {
+    // ---- rows [s*RS, (s+1)*RS) summed over the S partials in split order
+    // (the same sum on every run), by all 192 threads.  Each thread issues
+    // the remote loads (and residual reads) of ITEMS row chunks before it
+    // sums any of them: one chunk at a time left every thread waiting out
+    // the distributed-shared-memory latency once per chunk ----
     const int rows = min(MT * SBM, m);
     const int RS = (rows + S - 1) / S;
     const int r_begin = s * RS, r_end = min(rows, r_begin + RS);
-    const int t = threadIdx.x - 64;  // 0 .. 127
     const uint32_t part = smem_u32(smem);
     constexpr int CH = EPI == EPI_SWIGLU_BF16 ? 16 : 32;  // float4 chunks handled per row
+    constexpr int ITEMS = EPI == EPI_SWIGLU_BF16 ? 2 : MZC_SK_ITEMS;
+    const int n_items = max(0, r_end - r_begin) * CH;
     float amax = 0.0f;  // largest |value| this thread stores as fp16
-    for (int idx = t; idx < (r_end - r_begin) * CH; idx += 128) {
-      const int r = r_begin + idx / CH, c = idx % CH;
-      // all S loads are issued before the sum, which then runs in split order
-      float4 v[8], u[8];
+    for (int i0 = threadIdx.x; i0 < n_items; i0 += ITEMS * 192) {
+      float4 v[ITEMS][8], u[ITEMS][8], x[ITEMS];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        if (j < S) {
-          v[j] = ld_cluster_f4(map_rank(part + part_off(r, c), j));
-          if constexpr (EPI == EPI_SWIGLU_BF16) u[j] = ld_cluster_f4(map_rank(part + part_off(r, c + 16), j));
-        }
-      }
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f), acc2 = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int h = 0; h < ITEMS; ++h) {
+        const int idx = i0 + h * 192;
+        if (idx < n_items) {
+          const int r = r_begin + idx / CH, c = idx % CH;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        if (j < S) {
-          acc.x += v[j].x;
-          acc.y += v[j].y;
-          acc.z += v[j].z;
-          acc.w += v[j].w;
-          if constexpr (EPI == EPI_SWIGLU_BF16) {
-            acc2.x += u[j].x;
-            acc2.y += u[j].y;
-            acc2.z += u[j].z;
-            acc2.w += u[j].w;
+          for (int j = 0; j < 8; ++j) {
+            if (j < S) {
+              v[h][j] = ld_cluster_f4(map_rank(part + part_off(r, c), j));
+              if constexpr (EPI == EPI_SWIGLU_BF16) u[h][j] = ld_cluster_f4(map_rank(part + part_off(r, c + 16), j));
+            }
+          }
+          if constexpr (EPI == EPI_ADD_F32) {
+            const int col = nt * SBN + c * 4;
+            if (col < n) x[h] = *reinterpret_cast<const float4*>(static_cast<const float*>(out) + static_cast<int64_t>(r) * n + col);
           }
         }
       }
-      if constexpr (EPI == EPI_STORE_BF16) {
-        const int col = nt * SBN + c * 4;
-        if (col < n) {
-          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(acc.x), fabsf(acc.y)), fmaxf(fabsf(acc.z), fabsf(acc.w))));
-          *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * n + col) =
-              pack4_f16(acc.x, acc.y, acc.z, acc.w);
+#pragma unroll
+      for (int h = 0; h < ITEMS; ++h) {
+        const int idx = i0 + h * 192;
+        if (idx >= n_items) continue;
+        const int r = r_begin + idx / CH, c = idx % CH;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f), acc2 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (j < S) {
+            acc.x += v[h][j].x;
+            acc.y += v[h][j].y;
+            acc.z += v[h][j].z;
+            acc.w += v[h][j].w;
+            if constexpr (EPI == EPI_SWIGLU_BF16) {
+              acc2.x += u[h][j].x;
+              acc2.y += u[h][j].y;
+              acc2.z += u[h][j].z;
+              acc2.w += u[h][j].w;
+            }
+          }
         }
-      } else if constexpr (EPI == EPI_ADD_F32) {
-        const int col = nt * SBN + c * 4;
-        if (col < n) {
-          float4* o = reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<int64_t>(r) * n + col);
-          float4 x = *o;
-          x.x += acc.x;
-          x.y += acc.y;
-          x.z += acc.z;
-          x.w += acc.w;
-          *o = x;
-        }
-      } else {
-        // gate columns 0..63 of the tile pair with up columns 64..127
-        const int col = nt * (SBN / 2) + c * 4;
-        if (col < n / 2) {
-          const float y0 = silu_s(acc.x) * acc2.x, y1 = silu_s(acc.y) * acc2.y;
-          const float y2 = silu_s(acc.z) * acc2.z, y3 = silu_s(acc.w) * acc2.w;
-          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(y0), fabsf(y1)), fmaxf(fabsf(y2), fabsf(y3))));
-          *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * (n / 2) + col) =
-              pack4_f16(y0, y1, y2, y3);
+        if constexpr (EPI == EPI_STORE_BF16) {
+          const int col = nt * SBN + c * 4;
+          if (col < n) {
+            amax = fmaxf(amax, fmaxf(fmaxf(fabsf(acc.x), fabsf(acc.y)), fmaxf(fabsf(acc.z), fabsf(acc.w))));
+            *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * n + col) =
+                pack4_f16(acc.x, acc.y, acc.z, acc.w);
+          }
+        } else if constexpr (EPI == EPI_ADD_F32) {
+          const int col = nt * SBN + c * 4;
+          if (col < n) {
+            float4 y = x[h];
+            y.x += acc.x;
+            y.y += acc.y;
+            y.z += acc.z;
+            y.w += acc.w;
+            *reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<int64_t>(r) * n + col) = y;
+          }
+        } else {
+          // gate columns 0..63 of the tile pair with up columns 64..127
+          const int col = nt * (SBN / 2) + c * 4;
+          if (col < n / 2) {
+            const float y0 = silu_s(acc.x) * acc2.x, y1 = silu_s(acc.y) * acc2.y;
+            const float y2 = silu_s(acc.z) * acc2.z, y3 = silu_s(acc.w) * acc2.w;
+            amax = fmaxf(amax, fmaxf(fmaxf(fabsf(y0), fabsf(y1)), fmaxf(fabsf(y2), fabsf(y3))));
+            *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + static_cast<int64_t>(r) * (n / 2) + col) =
+                pack4_f16(y0, y1, y2, y3);
+          }
         }
       }
     }
