@@ -567,13 +567,12 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     htok[nrec + i] = tokens[i];
     hpos[nrec + i] = static_cast<int32_t>(P.prompt_begin + i);
   }
-  std::vector<int32_t> tab;
-  ctx->st.block_table(&tab, ctx->opt.read_swapped != 0);
-  std::memcpy(htab, tab.data(), tab.size() * 4);
+  ctx->st.block_table_into(htab, ctx->opt.read_swapped != 0);
+  const size_t tab_entries = static_cast<size_t>(ctx->st.table_entries());
   // swapped blocks this prefill reads in place from the mapped store
   const void* host_pool = ctx->opt.read_swapped ? ctx->h_store_dev : nullptr;
   const int64_t host_blocks = host_pool ? ctx->st.host_slots() : 0;
-  const size_t mbytes = static_cast<size_t>(rows) * 8 + tab.size() * 4;
+  const size_t mbytes = static_cast<size_t>(rows) * 8 + tab_entries * 4;
   int32_t* dtok = reinterpret_cast<int32_t*>(ctx->d_meta);
   int32_t* dpos = dtok + rows;
   int32_t* dtab = dpos + rows;

@@ -194,6 +194,7 @@ mzc_status State::evict_range(int32_t l0, int32_t l1, int64_t t0, int64_t t1, in
       e.phys = -1;
       e.region = rid;
       e.idx = (int32_t)(b - b0);
+      maybe_swapped_ = true;
     }
     if (moves) moves->push_back(std::move(mv));
   }
@@ -249,6 +250,7 @@ mzc_status State::evict_blocks(const int32_t* layer, const int64_t* blk, int64_t
       e.phys = -1;
       e.region = rid;
       e.idx = (int32_t)i;
+      maybe_swapped_ = true;
     }
     if (moves) moves->push_back(std::move(mv));
   }
@@ -279,8 +281,11 @@ mzc_status State::begin_restore(bool* any) {
   const int32_t L = shape_.n_layers;
   const int64_t nb = ceil_div(n_ctx_, 16);
   int64_t need = 0;
-  for (int32_t l = 0; l < L; ++l)
-    for (int64_t b = 0; b < nb; ++b) need += at(l, b).st == MZC_SWAPPED;
+  if (maybe_swapped_) {
+    for (int32_t l = 0; l < L; ++l)
+      for (int64_t b = 0; b < nb; ++b) need += at(l, b).st == MZC_SWAPPED;
+    maybe_swapped_ = need > 0;
+  }
   if (need > pool_.free_total()) return fail(MZC_ERR_OOM, "KV pool cannot hold the restored blocks");
   bool w = false;
   for (int32_t l = 0; l < L; ++l) w = w || w_state_[l] == MZC_SWAPPED;
@@ -351,7 +356,7 @@ mzc_status State::prepare_prefill(int64_t n_prompt, int64_t max_rows, PrefillPla
   const int64_t write_blk = (n_ctx_ % 16 && n_prompt > 0) ? n_ctx_ / 16 : -1;
   for (int32_t l = 0; l < L; ++l) {
     if (w_state_[l] == MZC_SWAPPED) return fail(MZC_ERR_STATE, "layer weights swapped, no restore in flight");
-    for (int64_t b = 0; b < nb; ++b) {
+    for (int64_t b = 0; maybe_swapped_ && b < nb; ++b) {
       if (at(l, b).st != MZC_SWAPPED) continue;
       if (!read_swapped_) return fail(MZC_ERR_STATE, "swapped blocks without a restore in flight");
       if (b == write_blk)
@@ -390,7 +395,8 @@ mzc_status State::prepare_prefill(int64_t n_prompt, int64_t max_rows, PrefillPla
   const int64_t last_partial = (n_ctx_ % 16) ? n_ctx_ / 16 : -1;
   for (int32_t l = 0; l < L; ++l) {
     P.w_wait[l] = w_state_[l] == MZC_INFLIGHT;
-    for (int64_t b = 0; b < nb; ++b) {
+    // blocks are INFLIGHT only while a restore is
+    for (int64_t b = 0; inflight_ && b < nb; ++b) {
       if (at(l, b).st != MZC_INFLIGHT) continue;
       P.kv_wait_prompt[l] = 1;
       if (b * 16 < P.rec_end) P.kv_wait_rec[l] = 1;
@@ -421,9 +427,12 @@ void State::abort_prefill(const PrefillPlan& P) {
 void State::complete(int64_t n_prompt) {
   const int32_t L = shape_.n_layers;
   const int64_t nb_new = ceil_div(n_ctx_ + n_prompt, 16);
+  // with no restore and no recompute pending only the new blocks (those
+  // prepare_prefill allocated past the context) change state
+  const int64_t b_first = (inflight_ || rec_pending_) ? 0 : ceil_div(n_ctx_, 16);
   for (int32_t l = 0; l < L; ++l) {
     if (w_state_[l] == MZC_INFLIGHT) w_state_[l] = MZC_RESIDENT;
-    for (int64_t b = 0; b < nb_new; ++b) {
+    for (int64_t b = b_first; b < nb_new; ++b) {
       BlockEntry& e = at(l, b);
       if (e.st == MZC_INFLIGHT) {
         drop_region_slot(e.region);
@@ -481,13 +490,22 @@ void State::counts(mzc_stats_t* o) const {
 
 void State::block_table(std::vector<int32_t>* out, bool host_slots) const {
   out->resize(tab_.size());
-  for (size_t i = 0; i < tab_.size(); ++i) {
+  block_table_into(out->data(), host_slots);
+}
+
+void State::block_table_into(int32_t* out, bool host_slots) const {
+  const size_t n = tab_.size();
+  if (!host_slots || !maybe_swapped_) {
+    for (size_t i = 0; i < n; ++i) out[i] = tab_[i].phys;
+    return;
+  }
+  for (size_t i = 0; i < n; ++i) {
     const BlockEntry& e = tab_[i];
-    if (host_slots && e.st == MZC_SWAPPED) {
+    if (e.st == MZC_SWAPPED) {
       const int64_t slot = (regions_[e.region].host_off + static_cast<int64_t>(e.idx) * slot_bytes_) / slot_bytes_;
-      (*out)[i] = static_cast<int32_t>(-2 - slot);
+      out[i] = static_cast<int32_t>(-2 - slot);
     } else {
-      (*out)[i] = e.phys;
+      out[i] = e.phys;
     }
   }
 }

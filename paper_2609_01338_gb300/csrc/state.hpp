@@ -144,6 +144,9 @@ class State {
   // host_slots, a SWAPPED block's entry is -2 - (its slot in the pinned store,
   // in units of slot_bytes), for kernels that read it in place.
   void block_table(std::vector<int32_t>* out, bool host_slots = false) const;
+  // the same table written to out[0 .. n_layers * nblk_max) (e.g. a pinned staging buffer)
+  void block_table_into(int32_t* out, bool host_slots = false) const;
+  int64_t table_entries() const { return static_cast<int64_t>(tab_.size()); }
   // Whether a prefill may read SWAPPED blocks in place (no restore issued).
   void set_read_swapped(bool on) { read_swapped_ = on; }
   int64_t host_slots() const { return host_bytes_ / slot_bytes_; }
@@ -166,6 +169,9 @@ class State {
   bool rec_pending_ = false;
   bool inflight_ = false;
   bool read_swapped_ = false;
+  // false only once a scan found no SWAPPED block since the last eviction to
+  // host: the per-step scans for swapped blocks are skipped while it is false
+  bool maybe_swapped_ = false;
   std::string err_;
 };
 
