@@ -84,6 +84,7 @@ struct mzc_ctx {
   size_t meta_bytes = 0;
   float* d_logits = nullptr;
   float* h_logits = nullptr;
+  int32_t* h_status = nullptr;  // inside h_logits' allocation, after the vocab floats
   void* d_scratch = nullptr;
   int64_t scratch_bytes = 0;
   int32_t* d_status = nullptr;
@@ -392,7 +393,10 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   CK(cudaHostAlloc(&ctx->h_meta, ctx->meta_bytes, cudaHostAllocMapped));
   CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&ctx->h_meta_dev), ctx->h_meta, 0));
   CK(cudaMalloc(&ctx->d_logits, V * 4));
-  CK(cudaHostAlloc(&ctx->h_logits, V * 4, cudaHostAllocDefault));
+  // the logits, then one word for the status read back with each step
+  CK(cudaHostAlloc(&ctx->h_logits, V * 4 + 16, cudaHostAllocDefault));
+  ctx->h_status = reinterpret_cast<int32_t*>(ctx->h_logits + V);
+  *ctx->h_status = 0;
   int64_t scratch = 0;
   for (int64_t n = 1; n <= std::min<int64_t>(R, 8192); ++n) {
     int sp = 1, per = 0;
@@ -755,6 +759,14 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     ctx->lm_timed = true;
   }
   CKP(cudaEventRecord(ctx->ev_t1, cs));
+  // the status word comes back with the step (after the copy stream's work
+  // too), so a clean step costs no extra round trip to read it
+  if (ctx->restore_issued) CKP(cudaStreamWaitEvent(cs, ctx->ev_c1, 0));
+  CKP(cudaMemcpyAsync(ctx->h_status, ctx->d_status, 4, cudaMemcpyDeviceToHost, cs));
+  // the host side of the restore's completion runs while the device works:
+  // nothing reads the table before this call returns, and both streams are
+  // synchronised below (a failed step still leaves the copied blocks valid)
+  ctx->st.complete_restore();
   CKP(cudaStreamSynchronize(cs));
   if (ctx->restore_issued) CKP(cudaStreamSynchronize(ctx->xs));
 #undef CKP
@@ -763,7 +775,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     if (cudaEventElapsedTime(&ms, ke.a, ke.b) == cudaSuccess) ctx->kstat[ke.cls].ms += ms;
   }
   ctx->kev.clear();
-  mzc_status st = check_status(ctx);
+  mzc_status st = *ctx->h_status == 0 ? MZC_OK : check_status(ctx);
   if (st != MZC_OK) {
     ctx->st.abort_prefill(P);
     return st;

@@ -424,21 +424,35 @@ void State::abort_prefill(const PrefillPlan& P) {
   }
 }
 
-void State::complete(int64_t n_prompt) {
+void State::complete_restore() {
+  if (!inflight_) return;
   const int32_t L = shape_.n_layers;
-  const int64_t nb_new = ceil_div(n_ctx_ + n_prompt, 16);
-  // with no restore and no recompute pending only the new blocks (those
-  // prepare_prefill allocated past the context) change state
-  const int64_t b_first = (inflight_ || rec_pending_) ? 0 : ceil_div(n_ctx_, 16);
+  const int64_t nb = ceil_div(n_ctx_, 16);
   for (int32_t l = 0; l < L; ++l) {
     if (w_state_[l] == MZC_INFLIGHT) w_state_[l] = MZC_RESIDENT;
-    for (int64_t b = b_first; b < nb_new; ++b) {
+    for (int64_t b = 0; b < nb; ++b) {
       BlockEntry& e = at(l, b);
       if (e.st == MZC_INFLIGHT) {
         drop_region_slot(e.region);
         e.st = MZC_RESIDENT;
         e.region = e.idx = -1;
-      } else if (e.st == MZC_DROPPED && rec_pending_) {
+      }
+    }
+  }
+  inflight_ = false;
+}
+
+void State::complete(int64_t n_prompt) {
+  complete_restore();
+  const int32_t L = shape_.n_layers;
+  const int64_t nb_new = ceil_div(n_ctx_ + n_prompt, 16);
+  // what changes now: the recomputed blocks (DROPPED, given physical blocks
+  // by prepare_prefill) and the new blocks past the context
+  const int64_t b_first = rec_pending_ ? std::min(drop_t0_ / 16, ceil_div(n_ctx_, 16)) : ceil_div(n_ctx_, 16);
+  for (int32_t l = 0; l < L; ++l) {
+    for (int64_t b = b_first; b < nb_new; ++b) {
+      BlockEntry& e = at(l, b);
+      if (e.st == MZC_DROPPED && rec_pending_) {
         e.st = MZC_RESIDENT;
       } else if (e.st == MZC_EMPTY && e.phys >= 0) {
         e.st = MZC_RESIDENT;
@@ -449,7 +463,6 @@ void State::complete(int64_t n_prompt) {
     rec_pending_ = false;
     drop_t0_ = drop_t1_ = -1;
   }
-  inflight_ = false;
   n_ctx_ += n_prompt;
 }
 

@@ -125,6 +125,11 @@ class State {
   // After the prefill (or a sync) completed on the device: in-flight and
   // recomputed blocks become RESIDENT, the context grows by the prompt.
   void complete(int64_t n_prompt);
+  // The restore's part of complete(): in-flight blocks and weights become
+  // RESIDENT and their host slots are released (no-op without a restore).
+  // The runtime calls it once every copy of the restore has been enqueued
+  // ahead of the work that waits for it, while the device still runs.
+  void complete_restore();
   // Undo prepare_prefill's allocations when the launch failed.
   void abort_prefill(const PrefillPlan& plan);
 
