@@ -172,9 +172,66 @@ __global__ void __launch_bounds__(256, G <= 8 ? 3 : (G <= 12 ? 2 : 1)) rmsnorm_w
   note_f16_overflow(status, amax);  // the whole warp holds this row
 }
 
+// The same RMSNorm for short row sets (a prompt of a few hundred rows): one
+// 128-thread CTA per row, the row and the scale vector loaded together and
+// held in registers.  With one warp per row a 128-row call ran on 16 SMs, each
+// pulling 96 KB through one round trip of loads; here 128 SMs share it.
+template <int G>
+__global__ void __launch_bounds__(128) rmsnorm_cta_kernel(const float* __restrict__ x,
+                                                          const float* __restrict__ g, float eps,
+                                                          uint16_t* __restrict__ y, int32_t* status) {
+  pdl_enter();
+  __shared__ float red[32];
+  constexpr int d = 256 * G, NG = 32 * G;   // 8-float groups in a row
+  constexpr int PER = (NG + 127) / 128;     // groups per thread
+  const int64_t i = blockIdx.x;
+  const int t = threadIdx.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + i * d);
+  const float4* gr = reinterpret_cast<const float4*>(g);
+  float4 a[PER], b[PER], ga[PER], gb[PER];
+  float ss = 0.0f;
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    const int c = k * 128 + t;
+    if (c < NG) {
+      a[k] = xr[2 * c];
+      b[k] = xr[2 * c + 1];
+      ga[k] = gr[2 * c];
+      gb[k] = gr[2 * c + 1];
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < PER; ++k)
+    if (k * 128 + t < NG)
+      ss += a[k].x * a[k].x + a[k].y * a[k].y + a[k].z * a[k].z + a[k].w * a[k].w +
+            b[k].x * b[k].x + b[k].y * b[k].y + b[k].z * b[k].z + b[k].w * b[k].w;
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / static_cast<float>(d) + eps);
+  uint4* yr = reinterpret_cast<uint4*>(y + i * d);
+  float amax = 0.0f;
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    const int c = k * 128 + t;
+    if (c >= NG) continue;
+    float f[8] = {a[k].x * r * ga[k].x, a[k].y * r * ga[k].y, a[k].z * r * ga[k].z, a[k].w * r * ga[k].w,
+                  b[k].x * r * gb[k].x, b[k].y * r * gb[k].y, b[k].z * r * gb[k].z, b[k].w * r * gb[k].w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(f[e]));
+    yr[c] = pack8<true>(f);
+  }
+  note_f16_overflow(status, amax);
+}
+
+// rows up to which the one-CTA-per-row form is used
+constexpr int64_t kRmsCtaRows = 512;
+
 template <int G>
 void launch_rmsnorm_warp(const float* x, const float* g, int64_t n, float eps, uint16_t* y,
                          int32_t* status, cudaStream_t st) {
+  if (n <= kRmsCtaRows) {
+    launch_k(rmsnorm_cta_kernel<G>, dim3(static_cast<unsigned>(n)), dim3(128), 0, st, x, g, eps, y, status);
+    return;
+  }
   launch_k(rmsnorm_warp_kernel<G>, dim3(static_cast<unsigned>((n + 7) / 8)), dim3(256), 0, st, x, g, n, eps, y,
            status);
 }

@@ -188,7 +188,10 @@ def test_q8_codec_matches_oracle(hkv, hd, kvd):
 
 # ---- RMSNorm, embedding, LM head --------------------------------------------
 
-@pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072), (5, 320), (3, 4608), (9, 4096)])
+# n <= 512 takes one CTA per row, more rows one warp per row (d a multiple of
+# 256), other widths the generic kernel
+@pytest.mark.parametrize("n,d", [(1, 256), (37, 2048), (300, 3072), (5, 320), (3, 4608), (9, 4096),
+                                 (512, 3072), (513, 3072), (1100, 2048), (700, 4096), (600, 320)])
 def test_rmsnorm(n, d):
     torch = _torch()
     rng = np.random.default_rng(n)
