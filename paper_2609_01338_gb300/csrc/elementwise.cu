@@ -470,12 +470,18 @@ cudaError_t launch_rope_kv_write(const uint16_t* qkv, const int32_t* pos, int64_
                                  int64_t pool_blocks, int32_t kv_dtype, uint16_t* q_out,
                                  int32_t* status, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
+  // a short row set (a prompt) has one CTA per row on as many SMs, each thread
+  // walking its work items one load round trip after another: up to 1024
+  // threads then give each item its own thread; longer row sets, bound by
+  // HBM, keep 128-thread CTAs, several per SM
+  const int items = (hq + hkv) * (hd / 16) + hkv * (hd / 8);
+  const int threads = n <= 512 ? std::min(1024, std::max(128, (items + 31) / 32 * 32)) : 128;
   if (kv_dtype == 1)
-    launch_k(rope_kv_kernel<true>, dim3(static_cast<unsigned>(n)), dim3(128), 0, st,
+    launch_k(rope_kv_kernel<true>, dim3(static_cast<unsigned>(n)), dim3(static_cast<unsigned>(threads)), 0, st,
         qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
         pool_blocks, q_out, status);
   else
-    launch_k(rope_kv_kernel<false>, dim3(static_cast<unsigned>(n)), dim3(128), 0, st,
+    launch_k(rope_kv_kernel<false>, dim3(static_cast<unsigned>(n)), dim3(static_cast<unsigned>(threads)), 0, st,
         qkv, pos, hq, hkv, hd, cos_t, sin_t, table, n_logical, static_cast<uint16_t*>(pool),
         pool_blocks, q_out, status);
   return cudaGetLastError();
