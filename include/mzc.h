@@ -123,6 +123,13 @@ typedef struct {
   void *copy_stream;        /* cudaStream_t of the restore copies, owned by the caller;
                                NULL = own.  The same stream as compute_stream is accepted
                                and serializes restore and prefill (no overlap) */
+  int32_t separate_norm;    /* 0 (default): for row sets of 5-256 rows each RMSNorm after
+                               the first is folded into the projections around it (the
+                               residual-add GEMM writes x * g and the rows' partial sums
+                               of squares; the next projection scales its rows by
+                               1 / RMS); 1: every RMSNorm runs as its own kernel, as for
+                               larger row sets (ablation).  Results agree within the
+                               fp16 rounding of the projection inputs */
 } mzc_options;
 
 /* Weights, host memory, bf16 bit patterns, row-major [out_features][in_features]
@@ -456,6 +463,30 @@ mzc_status mzc_k_rmsnorm(const float *x, const float *g, int64_t n, int32_t d, f
  * tcgen05 GEMM.  Each path gives the same bits on every run. */
 mzc_status mzc_k_gemm(const uint16_t *a, const uint16_t *w, void *out, int64_t m, int64_t n,
                       int64_t k, int32_t epilogue, void *stream);
+
+/* RMSNorm folded into the two projections around it, as mzc_prefill runs row
+ * sets of 5-256 rows (the pre-norm of the decoder layer: RMSNorm(x) W^T =
+ * diag(1 / RMS(x)) ((x * g) W^T), so the norm needs no launch of its own).
+ * m: 5..256 rows (MZC_ERR_INVALID otherwise).  All pointers DEVICE.
+ *   mzc_k_gemm_norm_out: the residual add x fp32 [m][n] += A W^T (epilogue 1
+ *     of mzc_k_gemm, on the split-K kernel; A fp16 [m][k], W fp16 [n][k]),
+ *     writing besides x  h fp16 [m][n] = x * g  (g fp32 [n]) and
+ *     ss fp32 [m][n / 128], ss[r][t] = the sum of the new x[r][c]^2 over the
+ *     columns c of tile t (128t .. 128t + 127).  n a multiple of 128, k of 8;
+ *     MZC_ERR_INVALID when the split-K kernel does not take the shape.
+ *   mzc_k_gemm_norm_in: epilogue 0 or 2 of mzc_k_gemm on diag(rstd) (h W^T),
+ *     h fp16 [m][k] from mzc_k_gemm_norm_out (d = k), W fp16 [n][k],
+ *     rstd_r = 1 / sqrt((ss[r][0] + ... + ss[r][k/128 - 1]) / k + eps), the
+ *     tiles summed in order; k a multiple of 128.
+ *   status  int32 or NULL: MZC_ERR_OVERFLOW when a value stored as fp16 (h,
+ *     or the consumer's output) reaches the fp16 overflow threshold.
+ * Each gives the same bits on every run. */
+mzc_status mzc_k_gemm_norm_out(const uint16_t *a, const uint16_t *w, float *x, int64_t m, int64_t n,
+                               int64_t k, const float *g, uint16_t *h, float *ss, int32_t *status,
+                               void *stream);
+mzc_status mzc_k_gemm_norm_in(const uint16_t *h, const uint16_t *w, void *out, int64_t m, int64_t n,
+                              int64_t k, int32_t epilogue, const float *ss, float eps, int32_t *status,
+                              void *stream);
 
 /* The residual-add GEMM (epilogue 1 of mzc_k_gemm: out fp32 [m][n] += A W^T,
  * the O and down projections of every decoder layer) with the persistent

@@ -18,6 +18,11 @@
 // spans exactly m rows and n columns, so rows >= m (computed on whatever the A
 // buffer holds) are clipped by the TMA unit.
 //
+// Folded RMSNorm (RowNorm, rows <= 256): the persistent kernel's row-scaled
+// form (RS) multiplies row r of the accumulator by its rstd, computed from the
+// producer's per-tile sums of squares before the tile's accumulator is ready,
+// ahead of the fp16 store or SwiGLU.
+//
 // Two kernels: the single-CTA persistent kernel (gemm_persistent_kernel) and,
 // for the tensor-bound projections above 512 rows, the paired-SM kernel
 // (gemm_pair_kernel: 256 x 256 tiles over the two CTAs of a cluster with
@@ -194,7 +199,7 @@ __device__ __forceinline__ bool split_wait(const uint64_t* flag, uint64_t want, 
 // boxes.  Each box goes out as one TMA store (fp16 outputs) or TMA reduce-add
 // into the fp32 residual stream, so the epilogue never reads the output and
 // writes whole 128-byte lines.
-template <int BN, int EPI>
+template <int BN, int EPI, bool RS = false>
 struct EpiWarp {
   uint8_t* box0;      // this warp's two staging boxes
   int lane;
@@ -219,9 +224,10 @@ struct EpiWarp {
   }
 
   // The warp's 32 rows of the tile from TMEM row address trow: rows y..y+31
-  // of the output (none stored when y >= m), columns from n0 (of n).
+  // of the output (none stored when y >= m), columns from n0 (of n).  RS:
+  // the lane's row is scaled by rs first.
   __device__ __forceinline__ void tile(const CUtensorMap* tmo, uint32_t trow, int y, int n0, int m,
-                                       int n) {
+                                       int n, float rs = 1.0f) {
     if constexpr (EPI == EPI_SWIGLU_BF16) {
 #pragma unroll 1
       for (int g = 0; g < BN / (2 * kSwigluGroup); ++g) {
@@ -231,6 +237,13 @@ struct EpiWarp {
           float vg[32], vu[32];
           tmem_ld32w(trow + g * 2 * kSwigluGroup + c, vg);
           tmem_ld32w(trow + g * 2 * kSwigluGroup + kSwigluGroup + c, vu);
+          if constexpr (RS) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              vg[i] *= rs;
+              vu[i] *= rs;
+            }
+          }
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             const float y0 = silu_f(vg[2 * i]) * vu[2 * i], y1 = silu_f(vg[2 * i + 1]) * vu[2 * i + 1];
@@ -254,6 +267,10 @@ struct EpiWarp {
         for (int h = 0; h < 64; h += 32) {
           float v[32];
           tmem_ld32w(trow + c + h, v);
+          if constexpr (RS) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= rs;
+          }
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             amax = fmaxf(amax, fmaxf(fabsf(v[2 * i]), fabsf(v[2 * i + 1])));
@@ -283,11 +300,11 @@ struct EpiWarp {
   }
 };
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, bool RS = false>
 __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw,
     const __grid_constant__ CUtensorMap tmo, int m, int n, int k, int band, int first, int ctas,
-    uint64_t* split_flags, uint32_t epoch, int32_t* status) {
+    uint64_t* split_flags, uint32_t epoch, int32_t* status, const RowNorm rn) {
   using C = PCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -415,11 +432,19 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
   } else {
     // ---- epilogue warps 2-5: TMEM -> registers -> swizzled staging box -> TMA ----
     const int q = warp & 3;
-    EpiWarp<BN, EPI> ew(sOut + q * 2 * kOutBox, lane);
+    EpiWarp<BN, EPI, RS> ew(sOut + q * 2 * kOutBox, lane);
     bool ok = true;
     WorkItem w;
     for (int local = 0; sched_item(sched, local, &w); ++local) {
       const int a = local & 1;
+      float rs = 1.0f;
+      if constexpr (RS) {
+        // folded RMSNorm: the lane's row's rstd before the accumulator is ready
+        int mt_r, nt_r;
+        tile_coords(w.tile, num_m, num_n, band, &mt_r, &nt_r);
+        const int row = mt_r * BM + q * 32 + lane;
+        if (row < m) rs = row_rstd(rn.ss, rn.nt, rn.d, rn.eps, row);
+      }
       ok = ok && pwait(&acc_full[a], (local >> 1) & 1, status, abort_flag);
       __syncwarp();
       if (!__all_sync(0xffffffffu, ok)) break;
@@ -430,7 +455,7 @@ __global__ void __launch_bounds__(192, 1) gemm_persistent_kernel(
       const uint32_t trow = tmem + a * BN + (static_cast<uint32_t>(q * 32) << 16);
       const int n0 = nt * BN;
       if constexpr (EPI != EPI_ADD_F32) {
-        ew.tile(&tmo, trow, y, n0, m, n);
+        ew.tile(&tmo, trow, y, n0, m, n, rs);
       } else {
         uint64_t* flag = w.seg >= 0 ? split_flags + (w.tile - first) : nullptr;
         bool go = true;
@@ -796,15 +821,15 @@ cudaError_t launch_pair(const CUtensorMap& ta, const CUtensorMap& tw128, void* o
   return cudaGetLastError();
 }
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, bool RS = false>
 cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void* out, int64_t m, int64_t n, int64_t k, int32_t* status,
-                              cudaStream_t st, GemmSplit* split) {
+                              cudaStream_t st, GemmSplit* split, const RowNorm* rn = nullptr) {
   using C = PCfg<BN, STAGES>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   static int sms = 0;
   std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_persistent_kernel<BN, STAGES, EPI>,
+    attr_err = cudaFuncSetAttribute(gemm_persistent_kernel<BN, STAGES, EPI, RS>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     int dev = 0;
     if (attr_err == cudaSuccess) attr_err = cudaGetDevice(&dev);
@@ -847,10 +872,11 @@ cudaError_t launch_persistent(const CUtensorMap& ta, const CUtensorMap& tw, void
       split->last_ctas = g;
     }
   }
-  launch_k(gemm_persistent_kernel<BN, STAGES, EPI>, dim3(static_cast<unsigned>(grid)),
+  const RowNorm norm = rn != nullptr ? *rn : RowNorm{};
+  launch_k(gemm_persistent_kernel<BN, STAGES, EPI, RS>, dim3(static_cast<unsigned>(grid)),
       dim3(192), C::SMEM, st, ta, tw, tmo, static_cast<int>(m), static_cast<int>(n),
       static_cast<int>(k), band, static_cast<int>(first), static_cast<int>(ctas), flags, epoch,
-      status);
+      status, norm);
   return cudaGetLastError();
 }
 
@@ -909,8 +935,16 @@ bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k) 
 // deeper ring for the narrower tiles.  The W map passed has the matching box.
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
-                        const uint16_t* a_ptr, GemmSplit* split) {
+                        const uint16_t* a_ptr, GemmSplit* split, const RowNorm* rn) {
   if (m <= 0) return cudaSuccess;
+  const bool norm_out = rn != nullptr && rn->h != nullptr && epilogue == EPI_ADD_F32;
+  const bool norm_in = rn != nullptr && rn->ss != nullptr && epilogue != EPI_ADD_F32;
+  if (norm_out || norm_in) {
+    // a folded RMSNorm: 5 to 256 rows, 128-column tiles of x
+    if (m <= kGemvMaxRows || m > 256 || rn->nt <= 0 || rn->ss == nullptr ||
+        (norm_out && (rn->g == nullptr || static_cast<int64_t>(rn->nt) * 128 != n)))
+      return cudaErrorInvalidValue;
+  }
   if (a_ptr && w.ptr && m <= kGemvMaxRows)
     return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, status, st);
   if (m <= 256) {
@@ -923,10 +957,22 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
       if (sms <= 0) sms = 1;
     }
     bool launched = false;
-    const cudaError_t e = launch_gemm_splitk(ta, w, out, m, n, k, epilogue, sms, status, st, &launched);
+    const cudaError_t e = launch_gemm_splitk(ta, w, out, m, n, k, epilogue, sms, status, st, &launched,
+                                             (norm_out || norm_in) ? rn : nullptr);
     if (launched || e != cudaSuccess) return e;
   }
   const uint32_t bn = gemm_box_n(m, n, epilogue);
+  if (norm_out) return cudaErrorInvalidValue;  // only the split-K kernel writes h and the sums
+  if (norm_in) {
+    // the row-scaled persistent kernel (no paired form)
+    if (epilogue == EPI_SWIGLU_BF16) {
+      if (bn == 256) return launch_persistent<256, 4, EPI_SWIGLU_BF16, true>(ta, w.box256, out, m, n, k, status, st, split, rn);
+      return launch_persistent<128, 6, EPI_SWIGLU_BF16, true>(ta, w.box128, out, m, n, k, status, st, split, rn);
+    }
+    if (bn == 256) return launch_persistent<256, 4, EPI_STORE_BF16, true>(ta, w.box256, out, m, n, k, status, st, split, rn);
+    if (bn == 128) return launch_persistent<128, 6, EPI_STORE_BF16, true>(ta, w.box128, out, m, n, k, status, st, split, rn);
+    return launch_persistent<64, 8, EPI_STORE_BF16, true>(ta, w.box64, out, m, n, k, status, st, split, rn);
+  }
   if (bn == 256 && MZC_GEMM_PAIR && m > BM) {
     // tensor-bound: the paired-SM kernel over 256 x 256 tiles
     static int sms = 0;

@@ -18,6 +18,11 @@
 //     the epilogue (fp16 store, fp32 residual add, SwiGLU) and writes the
 //     rows out; a second cluster barrier keeps every partial alive until all
 //     CTAs have read it.
+// Folded RMSNorm (RowNorm): the residual-add form also writes h = fp16(x * g)
+// and each row's sum of x^2 over the tile (one warp holds a row's 128 columns
+// in the reduction, so a shuffle tree sums them); the fp16-store and SwiGLU
+// forms scale each row by its rstd, which the epilogue warps compute from
+// those sums while the main loop runs.
 // Every thread of every CTA passes both cluster barriers exactly once (no
 // early exit on any path); the pipeline waits are bounded as elsewhere.
 #include <algorithm>
@@ -81,7 +86,7 @@ __device__ __forceinline__ uint32_t part_off(int r, int c) {
 template <int MT, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw, void* __restrict__ out,
-    int m, int n, int k, int32_t* status) {
+    int m, int n, int k, int32_t* status, const RowNorm rn) {
   using C = SKCfg<MT>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -92,6 +97,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   uint64_t* acc_full = empty + STAGES;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
+  __shared__ float s_rs[MT * SBM];  // folded RMSNorm: rstd of rows r_begin ..
   volatile int* abort_flag = &s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -100,6 +106,10 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   const int nkb = (k + SBK - 1) / SBK;
   const int kb0 = static_cast<int>(static_cast<int64_t>(s) * nkb / S);
   const int kb1 = static_cast<int>(static_cast<int64_t>(s + 1) * nkb / S);
+  // the output rows this CTA sums and writes: [r_begin, r_end)
+  const int rows = min(MT * SBM, m);
+  const int RS = (rows + S - 1) / S;
+  const int r_begin = s * RS, r_end = min(rows, r_begin + RS);
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tma);
@@ -180,6 +190,13 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   } else {
     // ---- epilogue warps 2-5: TMEM accumulator -> shared-memory partial ----
     const int q = warp & 3;  // TMEM lane quarter: rows q*32 .. q*32+31 of each M tile
+    if constexpr (EPI != EPI_ADD_F32) {
+      // folded RMSNorm: the rows' rstd while the main loop runs (the sums of
+      // squares come from the previous kernel, complete after pdl_enter)
+      if (rn.ss != nullptr)
+        for (int i = threadIdx.x - 64; r_begin + i < r_end; i += 128)
+          s_rs[i] = row_rstd(rn.ss, rn.nt, rn.d, rn.eps, r_begin + i);
+    }
     bool ok = skwait(acc_full, 0, status, abort_flag);
     __syncwarp();
     ok = __all_sync(0xffffffffu, ok);
@@ -216,16 +233,15 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     // the remote loads (and residual reads) of ITEMS row chunks before it
     // sums any of them: one chunk at a time left every thread waiting out
     // the distributed-shared-memory latency once per chunk ----
-    const int rows = min(MT * SBM, m);
-    const int RS = (rows + S - 1) / S;
-    const int r_begin = s * RS, r_end = min(rows, r_begin + RS);
     const uint32_t part = smem_u32(smem);
     constexpr int CH = EPI == EPI_SWIGLU_BF16 ? 16 : 32;  // float4 chunks handled per row
     constexpr int ITEMS = EPI == EPI_SWIGLU_BF16 ? 2 : MZC_SK_ITEMS;
     const int n_items = max(0, r_end - r_begin) * CH;
     float amax = 0.0f;  // largest |value| this thread stores as fp16
+    const bool norm_out = EPI == EPI_ADD_F32 && rn.h != nullptr;
+    const bool norm_in = EPI != EPI_ADD_F32 && rn.ss != nullptr;
     for (int i0 = threadIdx.x; i0 < n_items; i0 += ITEMS * 192) {
-      float4 v[ITEMS][8], u[ITEMS][8], x[ITEMS];
+      float4 v[ITEMS][8], u[ITEMS][8], x[ITEMS], gv[ITEMS];
 #pragma unroll
       for (int h = 0; h < ITEMS; ++h) {
         const int idx = i0 + h * 192;
@@ -240,7 +256,10 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
           }
           if constexpr (EPI == EPI_ADD_F32) {
             const int col = nt * SBN + c * 4;
-            if (col < n) x[h] = *reinterpret_cast<const float4*>(static_cast<const float*>(out) + static_cast<int64_t>(r) * n + col);
+            if (col < n) {
+              x[h] = *reinterpret_cast<const float4*>(static_cast<const float*>(out) + static_cast<int64_t>(r) * n + col);
+              if (norm_out) gv[h] = *reinterpret_cast<const float4*>(rn.g + col);
+            }
           }
         }
       }
@@ -265,6 +284,17 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
             }
           }
         }
+        if (norm_in) {
+          const float rs = s_rs[r - r_begin];
+          acc.x *= rs;
+          acc.y *= rs;
+          acc.z *= rs;
+          acc.w *= rs;
+          acc2.x *= rs;
+          acc2.y *= rs;
+          acc2.z *= rs;
+          acc2.w *= rs;
+        }
         if constexpr (EPI == EPI_STORE_BF16) {
           const int col = nt * SBN + c * 4;
           if (col < n) {
@@ -281,6 +311,18 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
             y.z += acc.z;
             y.w += acc.w;
             *reinterpret_cast<float4*>(static_cast<float*>(out) + static_cast<int64_t>(r) * n + col) = y;
+            if (norm_out) {
+              // the warp holds the row's 128 columns of this tile (CH = 32
+              // chunks, n a multiple of 128): h = fp16(x * g) and the tile's
+              // sum of x^2 for the consumer's rstd
+              const float h0 = y.x * gv[h].x, h1 = y.y * gv[h].y, h2 = y.z * gv[h].z, h3 = y.w * gv[h].w;
+              amax = fmaxf(amax, fmaxf(fmaxf(fabsf(h0), fabsf(h1)), fmaxf(fabsf(h2), fabsf(h3))));
+              *reinterpret_cast<uint2*>(rn.h + static_cast<int64_t>(r) * n + col) = pack4_f16(h0, h1, h2, h3);
+              float sq = y.x * y.x + y.y * y.y + y.z * y.z + y.w * y.w;
+#pragma unroll
+              for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+              if (lane == 0) rn.ss[static_cast<int64_t>(r) * rn.nt + nt] = sq;
+            }
           }
         } else {
           // gate columns 0..63 of the tile pair with up columns 64..127
@@ -295,7 +337,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
         }
       }
     }
-    if constexpr (EPI != EPI_ADD_F32) note_f16_overflow(status, amax);
+    if (EPI != EPI_ADD_F32 || norm_out) note_f16_overflow(status, amax);
   }
 
   // ---- no CTA leaves while another may still read its partial ----
@@ -310,7 +352,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
 
 template <int MT, int EPI>
 cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out, int64_t m, int64_t n, int64_t k,
-                      int S, int32_t* status, cudaStream_t st) {
+                      int S, int32_t* status, cudaStream_t st, const RowNorm& rn) {
   using C = SKCfg<MT>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -335,7 +377,7 @@ cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out
   cfg.attrs = attr;
   cfg.numAttrs = pdl_enabled() ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<MT, EPI>, ta, tw128, out, static_cast<int>(m),
-                            static_cast<int>(n), static_cast<int>(k), status);
+                            static_cast<int>(n), static_cast<int>(k), status, rn);
 }
 
 // The largest cluster size S <= 8 whose S x num_n CTAs are all resident at
@@ -376,17 +418,18 @@ int pick_splits(int num_n, int num_sms) {
 
 cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m, int64_t n,
                                int64_t k, int epilogue, int num_sms, int32_t* status, cudaStream_t st,
-                               bool* launched) {
+                               bool* launched, const RowNorm* rn) {
   *launched = false;
   if (m <= 0 || m > 2 * SBM || n % SBN != 0 || k % 8 != 0) return cudaSuccess;
   const int num_n = static_cast<int>(n / SBN);
   const bool two = m > SBM;
+  const RowNorm norm = rn != nullptr ? *rn : RowNorm{};
 #define MZC_SK(MTV, EPIV)                                                                   \
   {                                                                                        \
     const int S = pick_splits<MTV, EPIV>(num_n, num_sms);                                  \
     if (S < 2) return cudaSuccess;                                                         \
     *launched = true;                                                                      \
-    return launch_sk<MTV, EPIV>(ta, w.box128, out, m, n, k, S, status, st);                \
+    return launch_sk<MTV, EPIV>(ta, w.box128, out, m, n, k, S, status, st, norm);          \
   }
   switch (epilogue) {
     case EPI_STORE_BF16:
@@ -399,6 +442,22 @@ cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const GemmWeight& w, void*
       return cudaErrorInvalidValue;
   }
 #undef MZC_SK
+}
+
+bool gemm_splitk_launches(int64_t m, int64_t n, int64_t k, int epilogue, int num_sms) {
+  if (m <= 0 || m > 2 * SBM || n % SBN != 0 || k % 8 != 0) return false;
+  const int num_n = static_cast<int>(n / SBN);
+  const bool two = m > SBM;
+  switch (epilogue) {
+    case EPI_STORE_BF16:
+      return (two ? pick_splits<2, EPI_STORE_BF16>(num_n, num_sms) : pick_splits<1, EPI_STORE_BF16>(num_n, num_sms)) >= 2;
+    case EPI_ADD_F32:
+      return (two ? pick_splits<2, EPI_ADD_F32>(num_n, num_sms) : pick_splits<1, EPI_ADD_F32>(num_n, num_sms)) >= 2;
+    case EPI_SWIGLU_BF16:
+      return (two ? pick_splits<2, EPI_SWIGLU_BF16>(num_n, num_sms) : pick_splits<1, EPI_SWIGLU_BF16>(num_n, num_sms)) >= 2;
+    default:
+      return false;
+  }
 }
 
 }  // namespace mzc

@@ -69,12 +69,33 @@ struct GemmWeight {
   CUtensorMap box64, box128, box256;
   const uint16_t* ptr = nullptr;  // W itself, for the few-row GEMV
 };
+// RMSNorm folded into the projections of a short row set (RMSNorm(x) W^T =
+// diag(rstd) ((x * g) W^T) for the decoder layer's pre-norms):
+//   - producer, the split-K residual-add GEMM that finishes x (O or down):
+//     besides x it writes h = fp16(x * g) and, per row r and 128-column tile
+//     t of x, ss[r * nt + t] = the sum of x^2 over the tile's columns;
+//   - consumer, the next projection (QKV or gate/up) with h as its A operand:
+//     row r of its accumulator is scaled by
+//     rstd_r = rsqrt((ss[r * nt + 0] + ... + ss[r * nt + nt - 1]) / d + eps),
+//     summed in tile order, before its epilogue (fp16 store or SwiGLU).
+struct RowNorm {
+  const float* g = nullptr;  // producer: norm weights [d]
+  uint16_t* h = nullptr;     // producer: fp16 x * g, [m][d]
+  float* ss = nullptr;       // producer writes, consumer reads: [m][nt]
+  int nt = 0;                // 128-column tiles of x (d / 128)
+  float d = 0.0f, eps = 0.0f;
+};
+
 // Split-K GEMM over a thread-block cluster for m <= 256 (gemm_splitk.cu):
 // launched (and *launched set) when n is a multiple of 128 and a cluster size
 // of at least 2 fits the grid in one wave; otherwise nothing is launched.
+// `rn`: as the producer (epilogue EPI_ADD_F32, rn->h set) or the consumer
+// (EPI_STORE_BF16 / EPI_SWIGLU_BF16, rn->ss set) of a folded RMSNorm.
 cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const struct GemmWeight& w, void* out, int64_t m,
                                int64_t n, int64_t k, int epilogue, int num_sms, int32_t* status,
-                               cudaStream_t st, bool* launched);
+                               cudaStream_t st, bool* launched, const RowNorm* rn = nullptr);
+// Whether launch_gemm_splitk launches for this shape (the same rule).
+bool gemm_splitk_launches(int64_t m, int64_t n, int64_t k, int epilogue, int num_sms);
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);
 
 // State for splitting the residual-add GEMM's last wave over k: a device
@@ -96,10 +117,15 @@ inline uint32_t next_split_epoch(GemmSplit* s) {
 // C = A W^T; A map [>= m][k] with box rows 128.  The W map used is the one
 // whose box matches the tile width gemm_box_n(m, n, epilogue) selects.  With
 // `split`, the residual-add epilogue splits its last partial wave over k.
+// With `rn` (a folded RMSNorm, m of kGemvMaxRows + 1 .. 256): the producer
+// (EPI_ADD_F32) runs only as the split-K kernel (cudaErrorInvalidValue when
+// gemm_splitk_launches says it would not); a consumer runs as the split-K
+// kernel or the persistent kernel's row-scaled form.
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
-                        const uint16_t* a_ptr = nullptr, GemmSplit* split = nullptr);
+                        const uint16_t* a_ptr = nullptr, GemmSplit* split = nullptr,
+                        const RowNorm* rn = nullptr);
 
 // Few-row projections (decode steps; gemv.cu): A fp16 [m][k], W fp16 [n][k],
 // same epilogues as the GEMM; launch_gemm takes this path for m <= kGemvMaxRows

@@ -29,6 +29,16 @@ __device__ __forceinline__ void set_status(int32_t* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
 
+// 1 / RMS of row r from its per-tile sums of squares ss[r * nt + t] (a folded
+// RMSNorm): rsqrt(sum / d + eps), the tiles summed in order t = 0, 1, ...
+__device__ __forceinline__ float row_rstd(const float* ss, int nt, float d, float eps, int r) {
+  const float* p = ss + static_cast<int64_t>(r) * nt;
+  float s = 0.0f;
+#pragma unroll 8
+  for (int t = 0; t < nt; ++t) s += p[t];
+  return rsqrtf(s / d + eps);
+}
+
 // Records MZC_ERR_OVERFLOW when any lane of the (fully active) warp is about
 // to store, or has stored, a value of magnitude >= 65520 as fp16.  amax is the
 // lane's running maximum of |value| (fmaxf, so NaN inputs are not counted).

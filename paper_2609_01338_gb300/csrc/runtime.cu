@@ -73,6 +73,12 @@ struct mzc_ctx {
   uint8_t* d_weights = nullptr;
   uint16_t *d_embed = nullptr, *d_lm = nullptr;
   float* d_fnorm = nullptr;
+  // folded RMSNorm of row sets of 5-256 rows: resident copies of the layers'
+  // norm weights ([L][attn, ffn][d]; a producer GEMM reads the next layer's
+  // before that layer's streamed weights are waited for) and the per-row,
+  // per-128-column-tile sums of squares [256][d / 128]
+  float* d_gnorm = nullptr;
+  float* d_ss = nullptr;
   uint8_t* d_pool = nullptr;
   float *d_cos = nullptr, *d_sin = nullptr;
   float* d_x = nullptr;
@@ -163,7 +169,8 @@ mzc_status destroy_impl(mzc_ctx* ctx) {
                  ctx->d_cos,     ctx->d_sin,   ctx->d_x,       ctx->d_h,       ctx->d_qkv,
                  ctx->d_q,       ctx->d_attn,  ctx->d_act,     ctx->d_meta,    ctx->d_logits,
                  ctx->d_scratch, ctx->d_status, ctx->d_staging, ctx->d_list,
-                 ctx->d_rstage[0], ctx->d_rstage[1], ctx->d_flags, ctx->gsplit.flags};
+                 ctx->d_rstage[0], ctx->d_rstage[1], ctx->d_flags, ctx->gsplit.flags,
+                 ctx->d_gnorm,   ctx->d_ss};
   for (void* p : dev)
     if (p) cudaFree(p);
   void* host[] = {ctx->h_meta, ctx->h_logits, ctx->h_store, ctx->h_list, ctx->h_staging, ctx->h_ones};
@@ -338,6 +345,14 @@ mzc_status create_impl(const mzc_model_shape* shape, const mzc_options* options,
   CK(cudaMemcpy(ctx->d_embed, weights->embed, V * d * 2, cudaMemcpyHostToDevice));
   CK(cudaMemcpy(ctx->d_lm, weights->lm_head, V * d * 2, cudaMemcpyHostToDevice));
   CK(cudaMemcpy(ctx->d_fnorm, weights->final_norm, d * 4, cudaMemcpyHostToDevice));
+  if (d % 128 == 0) {
+    CK(cudaMalloc(&ctx->d_gnorm, static_cast<size_t>(L) * 2 * d * 4));
+    CK(cudaMalloc(&ctx->d_ss, static_cast<size_t>(256) * (d / 128) * 4));
+    for (int64_t l = 0; l < L; ++l) {
+      CK(cudaMemcpy(ctx->d_gnorm + (2 * l) * d, weights->layers[l].attn_norm, d * 4, cudaMemcpyHostToDevice));
+      CK(cudaMemcpy(ctx->d_gnorm + (2 * l + 1) * d, weights->layers[l].ffn_norm, d * 4, cudaMemcpyHostToDevice));
+    }
+  }
 
   // ---- KV pool (zeroed: never-written slots hold finite values) ----
   const size_t pool_bytes = static_cast<size_t>(ctx->st.pool_blocks()) * ctx->block_bytes;
@@ -630,13 +645,29 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
       return mzc::launch_embed(ctok, cr, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
     }));
+    // RMSNorm folded into the projections for row sets of 5-256 rows (the
+    // split-K kernels): each residual-add GEMM also writes x * g of the next
+    // norm and the rows' per-tile sums of squares, and the next QKV or gate/up
+    // projection scales its rows by rstd, so no norm runs as its own launch
+    // but the first layer's attention norm (after the embedding).
+    const bool fold = !ctx->opt.separate_norm && ctx->d_ss != nullptr && cr > mzc::kGemvMaxRows && cr <= 256 &&
+                      mzc::gemm_splitk_launches(cr, d, hq * hd, mzc::EPI_ADD_F32, ctx->num_sms) &&
+                      mzc::gemm_splitk_launches(cr, d, ctx->f_pad, mzc::EPI_ADD_F32, ctx->num_sms);
+    mzc::RowNorm rn_in;  // consumer: scales its rows by rstd
+    rn_in.ss = ctx->d_ss;
+    rn_in.nt = static_cast<int>(d / 128);
+    rn_in.d = static_cast<float>(d);
+    rn_in.eps = s.rms_eps;
+    mzc::RowNorm rn_out = rn_in;  // producer: writes h and the sums
+    rn_out.h = ctx->d_h;
     auto gemm = [&](const CUtensorMap& ta, const void* a_ptr, const mzc::GemmWeight& w, void* out,
-                    int64_t N, int64_t K, int epi) {
-      const double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
+                    int64_t N, int64_t K, int epi, const mzc::RowNorm* rn = nullptr) {
+      double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
+      if (rn != nullptr) out_b += epi == mzc::EPI_ADD_F32 ? R * N * 2.0 : R * (N / 128) * 4.0;
       return klaunch(ctx, MZC_K_GEMM, 2.0 * R * N * K, 2.0 * (R * K + static_cast<double>(N) * K) + out_b, 1,
                      [&] {
                        return mzc::launch_gemm(ta, w, out, cr, N, K, epi, ctx->d_status, cs,
-                                               static_cast<const uint16_t*>(a_ptr), &ctx->gsplit);
+                                               static_cast<const uint16_t*>(a_ptr), &ctx->gsplit, rn);
                      });
     };
     // attention of chunk rows [r0, r0 + nr) (r0 relative to the chunk)
@@ -661,11 +692,14 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
       const LayerDev& W = ctx->layers[l];
       const int32_t* ltab = dtab + l * ctx->nblk;
       if (P.w_wait[l]) CKP(cudaStreamWaitEvent(cs, ctx->ev_w[l], 0));
-      CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-        return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
-                                   ctx->d_status);
-      }));
-      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16));
+      const bool fold_in = fold && l > 0;  // h and the sums come from layer l-1's down projection
+      if (!fold_in)
+        CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+          return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
+                                     ctx->d_status);
+        }));
+      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16,
+               fold_in ? &rn_in : nullptr));
       if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
       CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
         return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
@@ -730,13 +764,21 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         if (wait_rec || wait_prm) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
         CKP(attention(0, cr, max_keys, ltab));
       }
-      CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
-      CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
-        return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
-                                   ctx->d_status);
-      }));
-      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16));
-      CKP(gemm(ctx->tm_act, ctx->d_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32));
+      if (fold) {
+        rn_out.g = ctx->d_gnorm + (2 * l + 1) * d;  // this layer's MLP norm
+        CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32, &rn_out));
+      } else {
+        CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
+        CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
+          return mzc::launch_rmsnorm(ctx->d_x, W.ffn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
+                                     ctx->d_status);
+        }));
+      }
+      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16,
+               fold ? &rn_in : nullptr));
+      if (fold) rn_out.g = ctx->d_gnorm + (2 * (l + 1)) * d;  // the next layer's attention norm
+      CKP(gemm(ctx->tm_act, ctx->d_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32,
+               fold ? &rn_out : nullptr));
       if (ctx->opt.debug_checks) {
         // name the first layer whose kernels recorded a device error
         CKP(cudaStreamSynchronize(cs));
@@ -1528,6 +1570,60 @@ mzc_status mzc_k_gemm(const uint16_t* a, const uint16_t* w, void* out, int64_t m
       !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
     return MZC_ERR_CUDA;
   KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, nullptr, static_cast<cudaStream_t>(stream), a));
+}
+
+static int device_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return sms;
+}
+
+mzc_status mzc_k_gemm_norm_out(const uint16_t* a, const uint16_t* w, float* x, int64_t m, int64_t n,
+                               int64_t k, const float* g, uint16_t* h, float* ss, int32_t* status,
+                               void* stream) {
+  if (!a || !w || !x || !g || !h || !ss || m <= mzc::kGemvMaxRows || m > 256 || n <= 0 || n % 128 != 0 ||
+      k <= 0 || k % 8 != 0)
+    return MZC_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return MZC_ERR_CUDA;
+  if (!mzc::gemm_splitk_launches(m, n, k, mzc::EPI_ADD_F32, sms)) return MZC_ERR_INVALID;
+  CUtensorMap ta;
+  mzc::GemmWeight tw;
+  if (!mzc::make_tmap_f16(&ta, a, static_cast<uint64_t>(m), static_cast<uint64_t>(k), 128) ||
+      !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
+    return MZC_ERR_CUDA;
+  mzc::RowNorm rn;
+  rn.g = g;
+  rn.h = h;
+  rn.ss = ss;
+  rn.nt = static_cast<int>(n / 128);
+  rn.d = static_cast<float>(n);
+  KCK(mzc::launch_gemm(ta, tw, x, m, n, k, mzc::EPI_ADD_F32, status, static_cast<cudaStream_t>(stream), a,
+                       nullptr, &rn));
+}
+
+mzc_status mzc_k_gemm_norm_in(const uint16_t* h, const uint16_t* w, void* out, int64_t m, int64_t n,
+                              int64_t k, int32_t epilogue, const float* ss, float eps, int32_t* status,
+                              void* stream) {
+  if (!h || !w || !out || !ss || m <= mzc::kGemvMaxRows || m > 256 || n <= 0 || n % 16 != 0 || k <= 0 ||
+      k % 128 != 0)
+    return MZC_ERR_INVALID;
+  if (epilogue != mzc::EPI_STORE_BF16 && epilogue != mzc::EPI_SWIGLU_BF16) return MZC_ERR_INVALID;
+  if (epilogue == mzc::EPI_SWIGLU_BF16 && n % (2 * mzc::kSwigluGroup) != 0) return MZC_ERR_INVALID;
+  CUtensorMap ta;
+  mzc::GemmWeight tw;
+  if (!mzc::make_tmap_f16(&ta, h, static_cast<uint64_t>(m), static_cast<uint64_t>(k), 128) ||
+      !mzc::make_gemm_weight(&tw, w, static_cast<uint64_t>(n), static_cast<uint64_t>(k)))
+    return MZC_ERR_CUDA;
+  mzc::RowNorm rn;
+  rn.ss = const_cast<float*>(ss);
+  rn.nt = static_cast<int>(k / 128);
+  rn.d = static_cast<float>(k);
+  rn.eps = eps;
+  KCK(mzc::launch_gemm(ta, tw, out, m, n, k, epilogue, status, static_cast<cudaStream_t>(stream), h,
+                       nullptr, &rn));
 }
 
 mzc_status mzc_k_gemm_split(const uint16_t* a, const uint16_t* w, float* out, int64_t m, int64_t n,

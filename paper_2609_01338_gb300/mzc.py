@@ -41,7 +41,7 @@ class mzc_options(ctypes.Structure):
     _fields_ = [("pool_blocks", c_i64), ("max_rows", c_i64), ("host_store_bytes", c_i64),
                 ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32),
                 ("wait_mode", c_i32), ("debug_checks", c_i32), ("read_swapped", c_i32),
-                ("compute_stream", c_vp), ("copy_stream", c_vp)]
+                ("compute_stream", c_vp), ("copy_stream", c_vp), ("separate_norm", c_i32)]
 
 
 class mzc_layer_weights(ctypes.Structure):
@@ -129,6 +129,8 @@ _SIGS = {
     "mzc_k_gemm": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_vp],
     "mzc_k_gemm_split": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_vp, c_i64, ctypes.c_uint32, c_vp,
                          c_vp, c_vp],
+    "mzc_k_gemm_norm_out": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_vp, c_vp, c_vp, c_vp, c_vp],
+    "mzc_k_gemm_norm_in": [c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_vp, c_f32, c_vp, c_vp],
     "mzc_k_swiglu_pack": [c_vp, c_vp, c_i64, c_i64, c_vp],
     "mzc_k_rope_kv_write": [c_vp, c_vp, c_i64, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_i64,
                             c_vp, c_i64, c_i32, c_vp, c_vp, c_vp],
@@ -241,12 +243,13 @@ def make_weights(weights: dict):
 
 def mzc_create(shape: dict, weights: dict, pool_blocks=0, max_rows=0, host_store_bytes=0,
                overlap=1, device=0, swap_codec=MZC_CODEC_NONE, wait_mode=MZC_WAIT_LAYER_EVENT,
-               debug_checks=0, compute_stream=None, copy_stream=None, read_swapped=0):
+               debug_checks=0, compute_stream=None, copy_stream=None, read_swapped=0, separate_norm=0):
     """compute_stream / copy_stream: cudaStream_t handles (ints, e.g. a torch
     stream's cuda_stream) owned by the caller, or None."""
     sh = make_shape(shape)
     opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec,
-                      wait_mode, debug_checks, read_swapped, compute_stream, copy_stream)
+                      wait_mode, debug_checks, read_swapped, compute_stream, copy_stream,
+                      separate_norm)
     w, keep = make_weights(weights)
     out = c_vp()
     _call("mzc_create", ctypes.byref(sh), ctypes.byref(opt), ctypes.byref(w), ctypes.byref(out))
@@ -441,6 +444,19 @@ def mzc_k_gemm_split(a, w, out, m, n, k, flags, epoch, status=None, stream=None)
     _call("mzc_k_gemm_split", _ptr(a), _ptr(w), _ptr(out), m, n, k, _ptr(flags), flags.numel(),
           epoch, _ptr(status), ctypes.byref(ctas), stream)
     return ctas.value
+
+
+def mzc_k_gemm_norm_out(a, w, x, m, n, k, g, h, ss, status=None, stream=None):
+    """x += A W^T, also writing h = fp16(x * g) and the per-128-column sums
+    of squares ss [m][n / 128] (the producer side of a folded RMSNorm)."""
+    return _call("mzc_k_gemm_norm_out", _ptr(a), _ptr(w), _ptr(x), m, n, k, _ptr(g), _ptr(h), _ptr(ss),
+                 _ptr(status), stream)
+
+
+def mzc_k_gemm_norm_in(h, w, out, m, n, k, epilogue, ss, eps, status=None, stream=None):
+    """Epilogue 0 / 2 of mzc_k_gemm on diag(rstd) (h W^T), rstd from ss."""
+    return _call("mzc_k_gemm_norm_in", _ptr(h), _ptr(w), _ptr(out), m, n, k, epilogue, _ptr(ss), eps,
+                 _ptr(status), stream)
 
 
 def mzc_k_swiglu_pack(gate, up):

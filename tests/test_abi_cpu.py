@@ -34,7 +34,7 @@ def test_library_exports_every_declared_symbol():
 
 def test_struct_sizes_match_c_layout():
     assert ctypes.sizeof(M.mzc_model_shape) == 56
-    assert ctypes.sizeof(M.mzc_options) == 64
+    assert ctypes.sizeof(M.mzc_options) == 72
     assert ctypes.sizeof(M.mzc_copy_run) == 24
     assert ctypes.sizeof(M.mzc_stats_t) == 80
 
