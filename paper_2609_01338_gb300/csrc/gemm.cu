@@ -939,6 +939,8 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
   if (m <= 0) return cudaSuccess;
   const bool norm_out = rn != nullptr && rn->h != nullptr && epilogue == EPI_ADD_F32;
   const bool norm_in = rn != nullptr && rn->ss != nullptr && epilogue != EPI_ADD_F32;
+  if ((norm_out || norm_in) && m == 1 && a_ptr && w.ptr)
+    return launch_gemv(a_ptr, w.ptr, out, m, n, k, epilogue, status, st, rn);  // one-row fold
   if (norm_out || norm_in) {
     // a folded RMSNorm: 5 to 256 rows, 128-column tiles of x
     if (m <= kGemvMaxRows || m > 256 || rn->nt <= 0 || rn->ss == nullptr ||

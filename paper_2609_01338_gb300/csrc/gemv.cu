@@ -7,6 +7,15 @@
 // non-caching loads, several in flight per lane, and reduces with shuffles;
 // the few activation rows come through L1.  fp32 accumulation; the
 // epilogues are the GEMM's (fp16 store, fp32 residual add, SwiGLU).
+//
+// Folded RMSNorm for one row (RowNorm; decode steps and the last layer's
+// logits row): the residual-add form (NORM = 1) also writes h = fp16(x * g)
+// for its outputs and one partial sum of x^2 per CTA (its outputs summed in
+// slot order) at ss[blockIdx.x]; the fp16-store and SwiGLU forms (NORM = 2)
+// load the producer's nt partials at their start (at most kGemvNormMax), sum
+// them after the main loop in a fixed order (per thread, then a shuffle tree,
+// then the warps in order; every CTA gets the same bits) and scale their
+// outputs by rsqrt(sum / d + eps).
 #include <cuda_fp16.h>
 
 #include "kernels.hpp"
@@ -44,16 +53,29 @@ __device__ __forceinline__ float silu_g(float g) { return g / (1.0f + __expf(-g)
 // 8 / KS outputs, and the KS partial sums meet in shared memory, added in
 // warp order (the same sum on every run).  Splitting K keeps each warp's chain
 // of dependent load rounds short and puts more weight bytes in flight.
-template <int EPI, int MR, int KS>
+template <int EPI, int MR, int KS, int NORM = 0>
 __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ a,
                                                    const uint16_t* __restrict__ w,
                                                    void* __restrict__ out, int m, int n, int k,
-                                                   int32_t* status) {
+                                                   int32_t* status, const RowNorm rn) {
   pdl_enter();
   constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
   constexpr int OUTS = 8 / KS;  // outputs per CTA
+  static_assert(NORM == 0 || MR == 1, "the folded norm is for one row");
+  constexpr int NQ = kGemvNormMax / 256;  // partials per thread (consumer)
   __shared__ float part[8][R][MR];
+  __shared__ float s_norm[8];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float pv[NORM == 2 ? NQ : 1];
+  if constexpr (NORM == 2) {
+    // the producer's partial sums of squares, loaded now, summed after the
+    // main loop (their latency hides under the weight stream)
+#pragma unroll
+    for (int q = 0; q < NQ; ++q) {
+      const int idx = threadIdx.x + 256 * q;
+      pv[q] = idx < rn.nt ? rn.ss[idx] : 0.0f;
+    }
+  }
   const int slot = warp / KS, ks = warp % KS;
   const int j = blockIdx.x * OUTS + slot;
   const int n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
@@ -103,6 +125,52 @@ __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ 
     for (int i = 0; i < MR; ++i)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) acc[r][i] += __shfl_xor_sync(0xffffffffu, acc[r][i], o);
+  if constexpr (NORM == 2) {
+    float t = 0.0f;
+#pragma unroll
+    for (int q = 0; q < NQ; ++q) t += pv[q];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) s_norm[warp] = t;
+    __syncthreads();
+    float sum = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) sum += s_norm[q];
+    const float rs = rsqrtf(sum / rn.d + rn.eps);
+#pragma unroll
+    for (int r = 0; r < R; ++r) acc[r][0] *= rs;  // the per-warp K parts scale alike
+  }
+  if constexpr (NORM == 1) {
+    // residual add with the folded norm's outputs: every thread reaches the
+    // CTA barrier below, so no thread leaves early
+    if constexpr (KS > 1) {
+      if (lane == 0) part[warp][0][0] = acc[0][0];
+      __syncthreads();
+    }
+    const bool writer = ks == 0 && lane == 0;
+    float ysq = 0.0f;
+    if (writer && valid) {
+      float t = acc[0][0];
+#pragma unroll
+      for (int q = 1; q < KS; ++q) t += part[warp + q][0][0];
+      float* o = static_cast<float*>(out) + j;
+      const float y = *o + t;
+      *o = y;
+      const float hv = y * rn.g[j];
+      if (fabsf(hv) >= kF16Overflow) set_status(status, kStatusOverflow);
+      reinterpret_cast<__half*>(rn.h)[j] = __float2half_rn(hv);
+      ysq = y * y;
+    }
+    if (writer) s_norm[slot] = ysq;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float sum = 0.0f;
+#pragma unroll
+      for (int q = 0; q < OUTS; ++q) sum += s_norm[q];
+      rn.ss[blockIdx.x] = sum;
+    }
+    return;
+  }
   if constexpr (KS > 1) {
     if (lane == 0) {
 #pragma unroll
@@ -141,48 +209,67 @@ __global__ void __launch_bounds__(256) gemv_kernel(const uint16_t* __restrict__ 
   }
 }
 
-template <int EPI, int MR, int KS>
+template <int EPI, int MR, int KS, int NORM = 0>
 cudaError_t launch_mrk(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                       int64_t k, int32_t* status, cudaStream_t st) {
+                       int64_t k, int32_t* status, cudaStream_t st, const RowNorm& rn) {
   const int64_t n_out = EPI == EPI_SWIGLU_BF16 ? n / 2 : n;
   constexpr int OUTS = 8 / KS;
-  launch_k(gemv_kernel<EPI, MR, KS>, dim3(static_cast<unsigned>((n_out + OUTS - 1) / OUTS)), dim3(256), 0, st,
-           a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status);
+  launch_k(gemv_kernel<EPI, MR, KS, NORM>, dim3(static_cast<unsigned>((n_out + OUTS - 1) / OUTS)), dim3(256), 0,
+           st, a, w, out, static_cast<int>(m), static_cast<int>(n), static_cast<int>(k), status, rn);
   return cudaGetLastError();
 }
 
 // K split per output: outputs of 6 KB of weights and more take two warps
 // (3B decode step: 2.68 -> 2.58 ms on one box; four warps for the 16 KB down
 // rows measured 2.64).
-template <int EPI, int MR>
+int gemv_ks(int64_t k, int epilogue) {
+  const int64_t bytes = k * 2 * (epilogue == EPI_SWIGLU_BF16 ? 2 : 1);  // weight bytes of one output
+  return bytes >= 6144 ? 2 : 1;
+}
+
+template <int EPI, int MR, int NORM = 0>
 cudaError_t launch_mr(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                      int64_t k, int32_t* status, cudaStream_t st) {
-  constexpr int R = EPI == EPI_SWIGLU_BF16 ? 2 : 1;
-  const int64_t bytes = k * 2 * R;  // weight bytes of one output
-  if (bytes >= 6144) return launch_mrk<EPI, MR, 2>(a, w, out, m, n, k, status, st);
-  return launch_mrk<EPI, MR, 1>(a, w, out, m, n, k, status, st);
+                      int64_t k, int32_t* status, cudaStream_t st, const RowNorm& rn) {
+  if (gemv_ks(k, EPI) == 2) return launch_mrk<EPI, MR, 2, NORM>(a, w, out, m, n, k, status, st, rn);
+  return launch_mrk<EPI, MR, 1, NORM>(a, w, out, m, n, k, status, st, rn);
 }
 
 template <int EPI>
 cudaError_t launch_epi(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                       int64_t k, int32_t* status, cudaStream_t st) {
-  return m == 1 ? launch_mr<EPI, 1>(a, w, out, m, n, k, status, st)
-                : launch_mr<EPI, 4>(a, w, out, m, n, k, status, st);
+                       int64_t k, int32_t* status, cudaStream_t st, const RowNorm* rn) {
+  if (rn != nullptr) {
+    // one row, with the folded norm: producer (residual add) or consumer
+    if constexpr (EPI == EPI_ADD_F32) return launch_mr<EPI, 1, 1>(a, w, out, m, n, k, status, st, *rn);
+    else return launch_mr<EPI, 1, 2>(a, w, out, m, n, k, status, st, *rn);
+  }
+  const RowNorm none{};
+  return m == 1 ? launch_mr<EPI, 1>(a, w, out, m, n, k, status, st, none)
+                : launch_mr<EPI, 4>(a, w, out, m, n, k, status, st, none);
 }
 
 }  // namespace
 
+int64_t gemv_norm_tiles(int64_t n, int64_t k) {
+  return (n + 8 / gemv_ks(k, EPI_ADD_F32) - 1) / (8 / gemv_ks(k, EPI_ADD_F32));
+}
+
 cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                        int64_t k, int epilogue, int32_t* status, cudaStream_t st) {
+                        int64_t k, int epilogue, int32_t* status, cudaStream_t st, const RowNorm* rn) {
   if (m <= 0) return cudaSuccess;
   if (m > kGemvMaxRows || k % 8 != 0) return cudaErrorInvalidValue;
+  if (rn != nullptr) {
+    // the folded norm takes one row; the producer's partials are one per CTA
+    if (m != 1 || rn->ss == nullptr || rn->nt <= 0 || rn->nt > kGemvNormMax) return cudaErrorInvalidValue;
+    if (epilogue == EPI_ADD_F32 && (rn->h == nullptr || rn->g == nullptr || rn->nt != gemv_norm_tiles(n, k)))
+      return cudaErrorInvalidValue;
+  }
   switch (epilogue) {
     case EPI_STORE_BF16:
-      return launch_epi<EPI_STORE_BF16>(a, w, out, m, n, k, status, st);
+      return launch_epi<EPI_STORE_BF16>(a, w, out, m, n, k, status, st, rn);
     case EPI_ADD_F32:
-      return launch_epi<EPI_ADD_F32>(a, w, out, m, n, k, status, st);
+      return launch_epi<EPI_ADD_F32>(a, w, out, m, n, k, status, st, rn);
     case EPI_SWIGLU_BF16:
-      return launch_epi<EPI_SWIGLU_BF16>(a, w, out, m, n, k, status, st);
+      return launch_epi<EPI_SWIGLU_BF16>(a, w, out, m, n, k, status, st, rn);
     default:
       return cudaErrorInvalidValue;
   }

@@ -120,7 +120,8 @@ inline uint32_t next_split_epoch(GemmSplit* s) {
 // With `rn` (a folded RMSNorm, m of kGemvMaxRows + 1 .. 256): the producer
 // (EPI_ADD_F32) runs only as the split-K kernel (cudaErrorInvalidValue when
 // gemm_splitk_launches says it would not); a consumer runs as the split-K
-// kernel or the persistent kernel's row-scaled form.
+// kernel or the persistent kernel's row-scaled form.  For m = 1 with a_ptr,
+// the GEMV's one-row form (launch_gemv); m of 2..4 with `rn` is refused.
 uint32_t gemm_box_n(int64_t m, int64_t n, int epilogue);
 cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m,
                         int64_t n, int64_t k, int epilogue, int32_t* status, cudaStream_t st,
@@ -129,10 +130,16 @@ cudaError_t launch_gemm(const CUtensorMap& ta, const GemmWeight& w, void* out, i
 
 // Few-row projections (decode steps; gemv.cu): A fp16 [m][k], W fp16 [n][k],
 // same epilogues as the GEMM; launch_gemm takes this path for m <= kGemvMaxRows
-// when it is given the activation pointer.
+// when it is given the activation pointer.  `rn`: the folded RMSNorm for one
+// row (m = 1): the residual add writes h and one partial sum of squares per
+// CTA (gemv_norm_tiles(n, k) of them, at most kGemvNormMax); the fp16-store or
+// SwiGLU consumer sums rn->nt partials and scales its outputs by rstd.
 constexpr int kGemvMaxRows = 4;
+constexpr int kGemvNormMax = 2048;
+int64_t gemv_norm_tiles(int64_t n, int64_t k);
 cudaError_t launch_gemv(const uint16_t* a, const uint16_t* w, void* out, int64_t m, int64_t n,
-                        int64_t k, int epilogue, int32_t* status, cudaStream_t st);
+                        int64_t k, int epilogue, int32_t* status, cudaStream_t st,
+                        const RowNorm* rn = nullptr);
 
 // 8-bit swap codec (codec.cu).  block_elems = 2 * hkv * 16 * hd.
 int64_t q8_block_bytes(int64_t block_elems);

@@ -645,21 +645,30 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     CKP(klaunch(ctx, MZC_K_EMBED, 0.0, R * dd * 6.0, 1, [&] {
       return mzc::launch_embed(ctok, cr, ctx->d_embed, static_cast<int32_t>(d), s.vocab, ctx->d_x, ctx->d_status, cs);
     }));
-    // RMSNorm folded into the projections for row sets of 5-256 rows (the
-    // split-K kernels): each residual-add GEMM also writes x * g of the next
-    // norm and the rows' per-tile sums of squares, and the next QKV or gate/up
-    // projection scales its rows by rstd, so no norm runs as its own launch
-    // but the first layer's attention norm (after the embedding).
-    const bool fold = !ctx->opt.separate_norm && ctx->d_ss != nullptr && cr > mzc::kGemvMaxRows && cr <= 256 &&
-                      mzc::gemm_splitk_launches(cr, d, hq * hd, mzc::EPI_ADD_F32, ctx->num_sms) &&
-                      mzc::gemm_splitk_launches(cr, d, ctx->f_pad, mzc::EPI_ADD_F32, ctx->num_sms);
-    mzc::RowNorm rn_in;  // consumer: scales its rows by rstd
-    rn_in.ss = ctx->d_ss;
-    rn_in.nt = static_cast<int>(d / 128);
-    rn_in.d = static_cast<float>(d);
-    rn_in.eps = s.rms_eps;
-    mzc::RowNorm rn_out = rn_in;  // producer: writes h and the sums
-    rn_out.h = ctx->d_h;
+    // RMSNorm folded into the projections: each residual-add projection also
+    // writes x * g of the next norm and partial sums of squares of x, and the
+    // next QKV or gate/up projection scales its rows by rstd, so no norm runs
+    // as its own launch but the first layer's attention norm (after the
+    // embedding).  Row sets of 5-256 rows: the split-K kernels, one partial
+    // per row and 128-column tile.  One row (decode steps, and the last
+    // layer's logits row of every prefill): the GEMV kernels, one partial per
+    // producer CTA.
+    const bool fold_rows = !ctx->opt.separate_norm && ctx->d_ss != nullptr && cr > mzc::kGemvMaxRows &&
+                           cr <= 256 && mzc::gemm_splitk_launches(cr, d, hq * hd, mzc::EPI_ADD_F32, ctx->num_sms) &&
+                           mzc::gemm_splitk_launches(cr, d, ctx->f_pad, mzc::EPI_ADD_F32, ctx->num_sms);
+    const int64_t np_o = mzc::gemv_norm_tiles(d, hq * hd), np_d = mzc::gemv_norm_tiles(d, ctx->f_pad);
+    const bool fold_one = !ctx->opt.separate_norm && ctx->d_ss != nullptr && np_o <= mzc::kGemvNormMax &&
+                          np_d <= mzc::kGemvNormMax;
+    const bool fold = fold_rows || (cr == 1 && fold_one);
+    mzc::RowNorm rn_qkv;  // consumer of the previous layer's down projection
+    rn_qkv.ss = ctx->d_ss;
+    rn_qkv.nt = static_cast<int>(fold_rows ? d / 128 : np_d);
+    rn_qkv.d = static_cast<float>(d);
+    rn_qkv.eps = s.rms_eps;
+    mzc::RowNorm rn_mlp = rn_qkv;  // consumer of the O projection
+    rn_mlp.nt = static_cast<int>(fold_rows ? d / 128 : np_o);
+    mzc::RowNorm rn_o = rn_mlp, rn_down = rn_qkv;  // producers: write h and the sums
+    rn_o.h = rn_down.h = ctx->d_h;
     auto gemm = [&](const CUtensorMap& ta, const void* a_ptr, const mzc::GemmWeight& w, void* out,
                     int64_t N, int64_t K, int epi, const mzc::RowNorm* rn = nullptr) {
       double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
@@ -699,7 +708,7 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
                                      ctx->d_status);
         }));
       CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16,
-               fold_in ? &rn_in : nullptr));
+               fold_in ? &rn_qkv : nullptr));
       if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
       CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
         return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
@@ -722,21 +731,27 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
             CKP(attention(r, 1, max_keys, ltab));
           }
           auto row_gemm = [&](const void* a_row, const mzc::GemmWeight& w, void* out_row, int64_t N, int64_t K,
-                              int epi) {
+                              int epi, const mzc::RowNorm* rn = nullptr) {
             const double out_b = epi == mzc::EPI_ADD_F32 ? N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? N * 1.0 : N * 2.0);
             return klaunch(ctx, MZC_K_GEMM, 2.0 * N * K, 2.0 * (K + static_cast<double>(N) * K) + out_b, 1, [&] {
               return mzc::launch_gemm(ctx->tm_h, w, out_row, 1, N, K, epi, ctx->d_status, cs,
-                                      static_cast<const uint16_t*>(a_row));
+                                      static_cast<const uint16_t*>(a_row), nullptr, rn);
             });
           };
+          // the row's MLP norm folded into its O and gate/up GEMVs
+          mzc::RowNorm rn_o1 = rn_o, rn_m1 = rn_mlp;
+          rn_o1.nt = rn_m1.nt = static_cast<int>(np_o);
+          rn_o1.h = ctx->d_h + r * d;
+          rn_o1.g = ctx->d_gnorm != nullptr ? ctx->d_gnorm + (2 * l + 1) * d : nullptr;
           CKP(row_gemm(ctx->d_attn + r * hq * hd, W.tm_o, ctx->d_x + r * d, d, static_cast<int64_t>(f),
-                       mzc::EPI_ADD_F32));
-          CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, dd * 10.0, 1, [&] {
-            return mzc::launch_rmsnorm(ctx->d_x + r * d, W.ffn_norm, 1, static_cast<int32_t>(d), s.rms_eps,
-                                       ctx->d_h + r * d, cs, ctx->d_status);
-          }));
+                       mzc::EPI_ADD_F32, fold_one ? &rn_o1 : nullptr));
+          if (!fold_one)
+            CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, dd * 10.0, 1, [&] {
+              return mzc::launch_rmsnorm(ctx->d_x + r * d, W.ffn_norm, 1, static_cast<int32_t>(d), s.rms_eps,
+                                         ctx->d_h + r * d, cs, ctx->d_status);
+            }));
           CKP(row_gemm(ctx->d_h + r * d, W.tm_13, ctx->d_act + r * ctx->f_pad, 2 * ctx->f_pad, d,
-                       mzc::EPI_SWIGLU_BF16));
+                       mzc::EPI_SWIGLU_BF16, fold_one ? &rn_m1 : nullptr));
           CKP(row_gemm(ctx->d_act + r * ctx->f_pad, W.tm_2, ctx->d_x + r * d, d, ctx->f_pad, mzc::EPI_ADD_F32));
         }
         if (ctx->opt.debug_checks) {
@@ -765,8 +780,8 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         CKP(attention(0, cr, max_keys, ltab));
       }
       if (fold) {
-        rn_out.g = ctx->d_gnorm + (2 * l + 1) * d;  // this layer's MLP norm
-        CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32, &rn_out));
+        rn_o.g = ctx->d_gnorm + (2 * l + 1) * d;  // this layer's MLP norm
+        CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32, &rn_o));
       } else {
         CKP(gemm(ctx->tm_attn, ctx->d_attn, W.tm_o, ctx->d_x, d, hq * hd, mzc::EPI_ADD_F32));
         CKP(klaunch(ctx, MZC_K_RMSNORM, 0.0, norm_bytes, 1, [&] {
@@ -775,10 +790,10 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
         }));
       }
       CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_13, ctx->d_act, 2 * ctx->f_pad, d, mzc::EPI_SWIGLU_BF16,
-               fold ? &rn_in : nullptr));
-      if (fold) rn_out.g = ctx->d_gnorm + (2 * (l + 1)) * d;  // the next layer's attention norm
+               fold ? &rn_mlp : nullptr));
+      if (fold) rn_down.g = ctx->d_gnorm + (2 * (l + 1)) * d;  // the next layer's attention norm
       CKP(gemm(ctx->tm_act, ctx->d_act, W.tm_2, ctx->d_x, d, ctx->f_pad, mzc::EPI_ADD_F32,
-               fold ? &rn_out : nullptr));
+               fold ? &rn_down : nullptr));
       if (ctx->opt.debug_checks) {
         // name the first layer whose kernels recorded a device error
         CKP(cudaStreamSynchronize(cs));

@@ -8,9 +8,10 @@ rstd.  What is fixed exactly is checked exactly (h is the fp16 rounding of the
 returned x times g); the projection is checked against the oracle's
 RMSNorm + linear (+ SwiGLU) with the bound that the fp16 rounding of h and of
 the output gives, element by element.  End to end, prefills of 200 and 37 rows
-with the fold match the oracle's full prefill as the separate-norm path does,
-and run the RMSNorm kernel only where the fold cannot (the first layer's
-attention norm and the last row's MLP norm)."""
+and two one-token steps (the GEMV kernels' one-row fold, also taken by the
+last layer's logits row of every prefill) match the oracle's prefill of the
+same tokens as the separate-norm path does, and run the RMSNorm kernel only
+for the first layer's attention norm."""
 import numpy as np
 import pytest
 
@@ -131,10 +132,11 @@ CASES = {
 
 @pytest.mark.parametrize("name", list(CASES))
 def test_folded_norm_prefill_matches_the_oracle(name):
-    """A 200-row context prefill and a 37-row prompt prefill (both folded)
-    against the oracle's prefill of the same tokens: logits max-abs <= 2e-2,
-    K/V max|d| / max|ref| <= 1e-2 per layer, as for the separate-norm path,
-    which runs beside it; the fold leaves two RMSNorm launches a prefill."""
+    """A 200-row context prefill, a 37-row prompt prefill and two one-token
+    steps (all folded) against the oracle's prefill of the same tokens: logits
+    max-abs <= 2e-2, K/V max|d| / max|ref| <= 1e-2 per layer, as for the
+    separate-norm path, which runs beside it; the fold leaves one RMSNorm
+    launch a prefill."""
     sh = CASES[name]
     L = sh["n_layers"]
     w = synth.model_weights(sh)
@@ -149,12 +151,15 @@ def test_folded_norm_prefill_matches_the_oracle(name):
     kv_ref = oracle.KVState(sh, sh["max_ctx"])
     lg_ctx = oracle.prefill(sh, w, kv_ref, ctx, 0)
     lg_prm = oracle.prefill(sh, w, kv_ref, prm, 200)
+    steps = synth.tokens(synth.SEED_PROMPT, 22, 2, sh["vocab"])
+    lg_steps = [oracle.prefill(sh, w, kv_ref, steps[i:i + 1], 237 + i) for i in range(2)]
+    n_tok = 239
     for sep in (0, 1):
         c = m.mzc_create(sh, w, separate_norm=sep)
         try:
             norms = []
             lgs = []
-            for toks in (ctx, prm):
+            for toks in (ctx, prm, steps[:1], steps[1:]):
                 m.mzc_set_kernel_timing(c, 0)  # resets the launch counters
                 out = np.empty(sh["vocab"], np.float32)
                 m.mzc_prefill(c, toks, out)
@@ -162,12 +167,14 @@ def test_folded_norm_prefill_matches_the_oracle(name):
                 norms.append(m.mzc_kernel_stats(c, m.MZC_K_RMSNORM).launches)
             assert np.max(np.abs(lgs[0] - lg_ctx)) < 2e-2
             assert np.max(np.abs(lgs[1] - lg_prm)) < 2e-2
-            k, v = m.mzc_read_kv_all(c, 237, sh)
+            for i in range(2):
+                assert np.max(np.abs(lgs[2 + i] - lg_steps[i])) < 2e-2
+            k, v = m.mzc_read_kv_all(c, n_tok, sh)
             for l in range(L):
-                assert rel_err(k[l], kv_ref.k[l, :237]) < 1e-2
-                assert rel_err(v[l], kv_ref.v[l, :237]) < 1e-2
+                assert rel_err(k[l], kv_ref.k[l, :n_tok]) < 1e-2
+                assert rel_err(v[l], kv_ref.v[l, :n_tok]) < 1e-2
             # separate: every layer's attention norm, the MLP norms of the first
             # L - 1 layers over all rows, the last layer's over the logits row
-            assert norms == ([2, 2] if sep == 0 else [2 * L, 2 * L])
+            assert norms == ([1] * 4 if sep == 0 else [2 * L] * 4)
         finally:
             m.mzc_destroy(c)
