@@ -151,7 +151,8 @@ class Runner:
     """Owns one ctx on one GPU and knows how to put the evicted state at rest
     (untimed) and run one timed restore + prefill."""
 
-    def __init__(self, name, sc, device, codec=0, read_swapped=0, wait_mode=0, separate_norm=0):
+    def __init__(self, name, sc, device, codec=0, read_swapped=0, wait_mode=0, separate_norm=0,
+                 fused_rope=0):
         import synth
         import paper_2609_01338_gb300 as m
         self.m, self.name, self.sc = m, name, sc
@@ -166,7 +167,7 @@ class Runner:
         t = time.time()
         self.c = m.mzc_create(sh, self.w, max_rows=max_rows, device=device, swap_codec=codec,
                               read_swapped=read_swapped, wait_mode=wait_mode,
-                              separate_norm=separate_norm)
+                              separate_norm=separate_norm, fused_rope=fused_rope)
         self.t_create = time.time() - t
         t = time.time()
         m.mzc_prefill(self.c, self.ctx_tokens)  # long contexts run in causal chunks
@@ -246,10 +247,11 @@ class Runner:
 HEADLINE = (1.0, "hybrid")
 
 
-def _config(name, sc, codec, n_gpus, wait_mode="event", separate_norm=False):
+def _config(name, sc, codec, n_gpus, wait_mode="event", separate_norm=False, fused_rope=False):
     """The `config` object; both arms print the same one."""
     cfg = {"workload": _describe(name, sc), "swap_codec": codec, "wait_mode": wait_mode,
-           "rmsnorm": "separate launches" if separate_norm else "folded into the projections at 5-256 rows",
+           "rmsnorm": "separate launches" if separate_norm else "folded into the projections at 1 and 5-256 rows",
+           "rope_kv_write": "inside the QKV projection at 5-256 rows" if fused_rope else "its own launch",
            "l2": "inputs larger than L2 (weights + KV >> 129 MB)",
            "parallelism": f"replicas x{n_gpus}" if n_gpus > 1 else "single GPU",
            "timed": "restore + recompute + prompt prefill + logits D2H per step; eviction between steps untimed"}
@@ -432,7 +434,7 @@ def run_reference(args, name, sc, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(statistics.mean(walls) * 1e3, 3), "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": _config(name, sc, args.codec, args.gpus, args.wait_mode, args.separate_norm),
+            "config": _config(name, sc, args.codec, args.gpus, args.wait_mode, args.separate_norm, args.fused_rope),
             "extrapolated": {"rows_per_timed_step": int(per), "rows_per_step": int(total),
                              "note": "value scales each step's sampled rows to the whole step; "
                                      "ms_per_step is the sampled step's own wall time"},
@@ -571,7 +573,10 @@ def main():
                     help="swap codec of the pinned store: none, or 8-bit groups (q8)")
     ap.add_argument("--separate-norm", action="store_true",
                     help="ablation: every RMSNorm as its own launch (no fold into the projections "
-                         "for row sets of 5-256 rows)")
+                         "for row sets of 1 or 5-256 rows)")
+    ap.add_argument("--fused-rope", action="store_true",
+                    help="the rotary embedding and KV-block write inside the QKV projection for row "
+                         "sets of 5-256 rows (option fused_rope; measured no faster)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mzc":
         args.warmup = 3
@@ -614,7 +619,8 @@ def main():
     r = Runner(name, sc, local, codec=1 if args.codec == "q8" else 0,
                read_swapped=1 if name == "3b_read_swapped" else 0,
                wait_mode=1 if args.wait_mode == "flag" else 0,
-               separate_norm=1 if args.separate_norm else 0)
+               separate_norm=1 if args.separate_norm else 0,
+               fused_rope=1 if args.fused_rope else 0)
     if name == "3b_sweep":
         run_headline(r, args, rank, world, local, dist)
         if dist:
@@ -666,7 +672,7 @@ def _single_line(r, args, world, name, sc, res, dist, clocks, wall):
         "ms_per_step": round(statistics.mean(res["dev"]), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": _config(name, sc, args.codec, world, args.wait_mode, args.separate_norm),
+        "config": _config(name, sc, args.codec, world, args.wait_mode, args.separate_norm, args.fused_rope),
         "recompute_tok_s": round(rec_rows / (v * 1e-3), 1) if rec_rows else None,
         "rows_per_step": rows,
         "gemm_tflops": round(gemm_tfs, 1) if gemm_tfs else None,
@@ -781,7 +787,7 @@ def run_headline(r, args, rank, world, local, dist):
         "ms_per_step": round(statistics.mean(head["dev"]), 3), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16",
         "data": "synthetic (seeded N(0,0.02) bf16 weights, uniform token ids)",
-        "config": {**_config(name, sc, args.codec, world, args.wait_mode, args.separate_norm),
+        "config": {**_config(name, sc, args.codec, world, args.wait_mode, args.separate_norm, args.fused_rope),
                    "value_point": {"fraction": vp[0], "policy": vp[1]}},
         "sweep": sweep, "hybrid_vs_policies": vs, "points": pts, "profile": prof,
         "roofline": _roofline(head["ks"], head["dom"], peaks, src, name),

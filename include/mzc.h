@@ -130,6 +130,13 @@ typedef struct {
                                1 / RMS); 1: every RMSNorm runs as its own kernel, as for
                                larger row sets (ablation).  Results agree within the
                                fp16 rounding of the projection inputs */
+  int32_t fused_rope;       /* 1: for row sets of 5-256 rows the rotary embedding and
+                               KV-block write run inside the QKV projection (its split-K
+                               reduction rotates the fp32 sums and writes q and the K/V
+                               blocks), except in a layer whose KV writes wait for a copy;
+                               0 (default): as their own kernel after an fp16 QKV output,
+                               which measured as fast or faster (the 3B 128-row prompt
+                               step: 3.842-3.845 ms against 3.852-3.862 fused) */
 } mzc_options;
 
 /* Weights, host memory, bf16 bit patterns, row-major [out_features][in_features]

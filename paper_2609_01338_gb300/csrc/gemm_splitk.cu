@@ -23,6 +23,11 @@
 // in the reduction, so a shuffle tree sums them); the fp16-store and SwiGLU
 // forms scale each row by its rstd, which the epilogue warps compute from
 // those sums while the main loop runs.
+// EPI_QKV_ROPE (the QKV projection of a short row set): the summed rows go
+// through the rotary embedding and the KV-block write in the reduction, so
+// no separate rotary launch and no fp16 QKV round trip.  A warp holds a row's
+// 128 columns, i.e. whole heads (hd 64 or 128), so the other half of each
+// rotary pair comes from lane ^ (hd / 8) by shuffle.
 // Every thread of every CTA passes both cluster barriers exactly once (no
 // early exit on any path); the pipeline waits are bounded as elsewhere.
 #include <algorithm>
@@ -76,6 +81,8 @@ __device__ __forceinline__ uint2 pack4_f16(float a, float b, float c, float d) {
   return make_uint2(pack2<true>(a, b), pack2<true>(c, d));
 }
 
+__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
 // Partial layout: row r (0 .. MT*128) of 32 float4 chunks, chunk c stored at
 // c ^ (r & 7) so that eight lanes writing one chunk of eight rows hit eight
 // different bank groups.
@@ -86,7 +93,7 @@ __device__ __forceinline__ uint32_t part_off(int r, int c) {
 template <int MT, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmw, void* __restrict__ out,
-    int m, int n, int k, int32_t* status, const RowNorm rn) {
+    int m, int n, int k, int32_t* status, const RowNorm rn, const RopeKV rk) {
   using C = SKCfg<MT>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -98,6 +105,9 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
   __shared__ float s_rs[MT * SBM];  // folded RMSNorm: rstd of rows r_begin ..
+  // EPI_QKV_ROPE: position and physical block of rows r_begin .. (-2: the
+  // position is outside the rotary tables and the block table)
+  __shared__ int s_pos[MT * SBM], s_phys[MT * SBM];
   volatile int* abort_flag = &s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -197,6 +207,16 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
         for (int i = threadIdx.x - 64; r_begin + i < r_end; i += 128)
           s_rs[i] = row_rstd(rn.ss, rn.nt, rn.d, rn.eps, r_begin + i);
     }
+    if constexpr (EPI == EPI_QKV_ROPE) {
+      // the rows' positions and KV blocks, looked up while the main loop runs
+      for (int i = threadIdx.x - 64; r_begin + i < r_end; i += 128) {
+        const int p = rk.pos[r_begin + i];
+        int ph = -2;
+        if (p >= 0 && (p >> 4) < rk.n_logical) ph = rk.table[p >> 4];
+        s_pos[i] = p;
+        s_phys[i] = ph;
+      }
+    }
     bool ok = skwait(acc_full, 0, status, abort_flag);
     __syncwarp();
     ok = __all_sync(0xffffffffu, ok);
@@ -241,7 +261,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
     const bool norm_out = EPI == EPI_ADD_F32 && rn.h != nullptr;
     const bool norm_in = EPI != EPI_ADD_F32 && rn.ss != nullptr;
     for (int i0 = threadIdx.x; i0 < n_items; i0 += ITEMS * 192) {
-      float4 v[ITEMS][8], u[ITEMS][8], x[ITEMS], gv[ITEMS];
+      float4 v[ITEMS][8], u[ITEMS][8], x[ITEMS], gv[ITEMS], rc[ITEMS], rsn[ITEMS];
 #pragma unroll
       for (int h = 0; h < ITEMS; ++h) {
         const int idx = i0 + h * 192;
@@ -259,6 +279,17 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
             if (col < n) {
               x[h] = *reinterpret_cast<const float4*>(static_cast<const float*>(out) + static_cast<int64_t>(r) * n + col);
               if (norm_out) gv[h] = *reinterpret_cast<const float4*>(rn.g + col);
+            }
+          }
+          if constexpr (EPI == EPI_QKV_ROPE) {
+            // the rotary angles of q and k columns, loaded with the partials
+            const int col = nt * SBN + c * 4;
+            const int head = col / rk.hd, e = col - head * rk.hd, half = rk.hd >> 1;
+            const int p = s_pos[r - r_begin];
+            if (head < rk.hq + rk.hkv && s_phys[r - r_begin] != -2) {
+              const int64_t t = static_cast<int64_t>(p) * half + (e < half ? e : e - half);
+              rc[h] = *reinterpret_cast<const float4*>(rk.cos_t + t);
+              rsn[h] = *reinterpret_cast<const float4*>(rk.sin_t + t);
             }
           }
         }
@@ -295,7 +326,54 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
           acc2.z *= rs;
           acc2.w *= rs;
         }
-        if constexpr (EPI == EPI_STORE_BF16) {
+        if constexpr (EPI == EPI_QKV_ROPE) {
+          // every lane of the warp is here (n_items is a multiple of 32, and
+          // a warp's items are one row): the rotary partner by shuffle first
+          const int pl = rk.hd >> 3;  // chunks between the two halves of a pair
+          float4 pr;
+          pr.x = __shfl_xor_sync(0xffffffffu, acc.x, pl);
+          pr.y = __shfl_xor_sync(0xffffffffu, acc.y, pl);
+          pr.z = __shfl_xor_sync(0xffffffffu, acc.z, pl);
+          pr.w = __shfl_xor_sync(0xffffffffu, acc.w, pl);
+          const int col = nt * SBN + c * 4;
+          const int head = col / rk.hd, e = col - head * rk.hd, half = rk.hd >> 1;
+          const int p = s_pos[r - r_begin], phys = s_phys[r - r_begin];
+          if (phys == -2) {
+            set_status(status, kStatusDevice);  // outside the rotary tables and the block table
+          } else {
+            float y0 = acc.x, y1 = acc.y, y2 = acc.z, y3 = acc.w;
+            if (head < rk.hq + rk.hkv) {
+              const float4 cs = rc[h], sn = rsn[h];
+              const float sg = e < half ? -1.0f : 1.0f;  // x1 c - x2 s, or x2 c + x1 s
+              y0 = acc.x * cs.x + sg * (pr.x * sn.x);
+              y1 = acc.y * cs.y + sg * (pr.y * sn.y);
+              y2 = acc.z * cs.z + sg * (pr.z * sn.z);
+              y3 = acc.w * cs.w + sg * (pr.w * sn.w);
+            }
+            uint16_t* dst = nullptr;
+            if (head < rk.hq) {
+              dst = rk.q_out + (static_cast<int64_t>(r) * rk.hq + head) * rk.hd + e;
+            } else {
+              if (phys < 0 || phys >= rk.pool_blocks) {
+                set_status(status, kStatusDevice);
+              } else {
+                if (!rk.f16kv) {
+                  y0 = bf16_round(y0);
+                  y1 = bf16_round(y1);
+                  y2 = bf16_round(y2);
+                  y3 = bf16_round(y3);
+                }
+                // K heads then V heads: head - hq indexes [2 hkv][16][hd] of the block
+                dst = rk.pool + static_cast<int64_t>(phys) * (2LL * rk.hkv * 16 * rk.hd) +
+                      (static_cast<int64_t>(head - rk.hq) * 16 + (p & 15)) * rk.hd + e;
+              }
+            }
+            if (dst != nullptr) {
+              amax = fmaxf(amax, fmaxf(fmaxf(fabsf(y0), fabsf(y1)), fmaxf(fabsf(y2), fabsf(y3))));
+              *reinterpret_cast<uint2*>(dst) = pack4_f16(y0, y1, y2, y3);
+            }
+          }
+        } else if constexpr (EPI == EPI_STORE_BF16) {
           const int col = nt * SBN + c * 4;
           if (col < n) {
             amax = fmaxf(amax, fmaxf(fmaxf(fabsf(acc.x), fabsf(acc.y)), fmaxf(fabsf(acc.z), fabsf(acc.w))));
@@ -352,7 +430,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
 
 template <int MT, int EPI>
 cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out, int64_t m, int64_t n, int64_t k,
-                      int S, int32_t* status, cudaStream_t st, const RowNorm& rn) {
+                      int S, int32_t* status, cudaStream_t st, const RowNorm& rn, const RopeKV& rk) {
   using C = SKCfg<MT>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -377,7 +455,7 @@ cudaError_t launch_sk(const CUtensorMap& ta, const CUtensorMap& tw128, void* out
   cfg.attrs = attr;
   cfg.numAttrs = pdl_enabled() ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, gemm_splitk_kernel<MT, EPI>, ta, tw128, out, static_cast<int>(m),
-                            static_cast<int>(n), static_cast<int>(k), status, rn);
+                            static_cast<int>(n), static_cast<int>(k), status, rn, rk);
 }
 
 // The largest cluster size S <= 8 whose S x num_n CTAs are all resident at
@@ -418,18 +496,24 @@ int pick_splits(int num_n, int num_sms) {
 
 cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const GemmWeight& w, void* out, int64_t m, int64_t n,
                                int64_t k, int epilogue, int num_sms, int32_t* status, cudaStream_t st,
-                               bool* launched, const RowNorm* rn) {
+                               bool* launched, const RowNorm* rn, const RopeKV* rk) {
   *launched = false;
   if (m <= 0 || m > 2 * SBM || n % SBN != 0 || k % 8 != 0) return cudaSuccess;
   const int num_n = static_cast<int>(n / SBN);
   const bool two = m > SBM;
   const RowNorm norm = rn != nullptr ? *rn : RowNorm{};
+  const RopeKV rope = rk != nullptr ? *rk : RopeKV{};
+  if (epilogue == EPI_QKV_ROPE &&
+      (rk == nullptr || (rope.hd != 64 && rope.hd != 128) || static_cast<int64_t>(rope.hq + 2 * rope.hkv) * rope.hd != n ||
+       rope.pos == nullptr || rope.cos_t == nullptr || rope.sin_t == nullptr || rope.table == nullptr ||
+       rope.pool == nullptr || rope.q_out == nullptr))
+    return cudaErrorInvalidValue;
 #define MZC_SK(MTV, EPIV)                                                                   \
   {                                                                                        \
     const int S = pick_splits<MTV, EPIV>(num_n, num_sms);                                  \
     if (S < 2) return cudaSuccess;                                                         \
     *launched = true;                                                                      \
-    return launch_sk<MTV, EPIV>(ta, w.box128, out, m, n, k, S, status, st, norm);          \
+    return launch_sk<MTV, EPIV>(ta, w.box128, out, m, n, k, S, status, st, norm, rope);    \
   }
   switch (epilogue) {
     case EPI_STORE_BF16:
@@ -438,6 +522,8 @@ cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const GemmWeight& w, void*
       if (two) MZC_SK(2, EPI_ADD_F32) else MZC_SK(1, EPI_ADD_F32)
     case EPI_SWIGLU_BF16:
       if (two) MZC_SK(2, EPI_SWIGLU_BF16) else MZC_SK(1, EPI_SWIGLU_BF16)
+    case EPI_QKV_ROPE:
+      if (two) MZC_SK(2, EPI_QKV_ROPE) else MZC_SK(1, EPI_QKV_ROPE)
     default:
       return cudaErrorInvalidValue;
   }
@@ -455,6 +541,8 @@ bool gemm_splitk_launches(int64_t m, int64_t n, int64_t k, int epilogue, int num
       return (two ? pick_splits<2, EPI_ADD_F32>(num_n, num_sms) : pick_splits<1, EPI_ADD_F32>(num_n, num_sms)) >= 2;
     case EPI_SWIGLU_BF16:
       return (two ? pick_splits<2, EPI_SWIGLU_BF16>(num_n, num_sms) : pick_splits<1, EPI_SWIGLU_BF16>(num_n, num_sms)) >= 2;
+    case EPI_QKV_ROPE:
+      return (two ? pick_splits<2, EPI_QKV_ROPE>(num_n, num_sms) : pick_splits<1, EPI_QKV_ROPE>(num_n, num_sms)) >= 2;
     default:
       return false;
   }

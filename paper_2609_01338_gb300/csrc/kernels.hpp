@@ -52,7 +52,27 @@ cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, si
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
+enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2, EPI_QKV_ROPE = 3 };
+
+// EPI_QKV_ROPE (split-K GEMM only): the QKV projection's rows go straight to
+// the rotary embedding and the KV-block write (as rope_kv_kernel, from the
+// fp32 sums instead of fp16 outputs): q and k rotated (half-split pairs,
+// fp32 tables), q to q_out [m][hq][hd] in fp16, K and V rounded to the KV
+// precision into pool[table[pos / 16]] slot pos % 16 (K [hkv][16][hd], then V).
+// Needs n = (hq + 2 hkv) hd a multiple of 128 and hd 64 or 128, so that a
+// 128-column tile holds whole heads.
+struct RopeKV {
+  const int32_t* pos = nullptr;    // [m]
+  const float* cos_t = nullptr;    // [positions][hd / 2]
+  const float* sin_t = nullptr;
+  const int32_t* table = nullptr;  // logical block -> physical block
+  int64_t n_logical = 0;           // table entries: positions < n_logical * 16
+  uint16_t* pool = nullptr;
+  int64_t pool_blocks = 0;
+  uint16_t* q_out = nullptr;
+  int hq = 0, hkv = 0, hd = 0;
+  int f16kv = 1;  // 0: K and V rounded to bf16 precision before the fp16 encoding
+};
 
 // Row group of the SwiGLU weight interleave: 64 gate rows, then the matching
 // 64 up rows, repeated.  The fused epilogue needs both halves in one tile.
@@ -91,9 +111,11 @@ struct RowNorm {
 // of at least 2 fits the grid in one wave; otherwise nothing is launched.
 // `rn`: as the producer (epilogue EPI_ADD_F32, rn->h set) or the consumer
 // (EPI_STORE_BF16 / EPI_SWIGLU_BF16, rn->ss set) of a folded RMSNorm.
+// `rk`: the rotary / KV-write targets of EPI_QKV_ROPE.
 cudaError_t launch_gemm_splitk(const CUtensorMap& ta, const struct GemmWeight& w, void* out, int64_t m,
                                int64_t n, int64_t k, int epilogue, int num_sms, int32_t* status,
-                               cudaStream_t st, bool* launched, const RowNorm* rn = nullptr);
+                               cudaStream_t st, bool* launched, const RowNorm* rn = nullptr,
+                               const RopeKV* rk = nullptr);
 // Whether launch_gemm_splitk launches for this shape (the same rule).
 bool gemm_splitk_launches(int64_t m, int64_t n, int64_t k, int epilogue, int num_sms);
 bool make_gemm_weight(GemmWeight* gw, const void* base, uint64_t n, uint64_t k);

@@ -669,6 +669,25 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
     rn_mlp.nt = static_cast<int>(fold_rows ? d / 128 : np_o);
     mzc::RowNorm rn_o = rn_mlp, rn_down = rn_qkv;  // producers: write h and the sums
     rn_o.h = rn_down.h = ctx->d_h;
+    // Option fused_rope: the rotary embedding and KV-block write inside the
+    // QKV projection's split-K reduction for row sets of 5-256 rows (no rotary
+    // launch, no fp16 QKV round trip), unless the layer's writes must wait for
+    // a copy.
+    const bool rope_rows = ctx->opt.fused_rope && cr > mzc::kGemvMaxRows && cr <= 256 &&
+                           (hd == 64 || hd == 128) &&
+                           mzc::gemm_splitk_launches(cr, ctx->qkv_dim, d, mzc::EPI_QKV_ROPE, ctx->num_sms);
+    mzc::RopeKV rk;
+    rk.pos = cpos;
+    rk.cos_t = ctx->d_cos;
+    rk.sin_t = ctx->d_sin;
+    rk.n_logical = ctx->nblk;
+    rk.pool = reinterpret_cast<uint16_t*>(ctx->d_pool);
+    rk.pool_blocks = ctx->st.pool_blocks();
+    rk.q_out = ctx->d_q;
+    rk.hq = static_cast<int>(hq);
+    rk.hkv = static_cast<int>(hkv);
+    rk.hd = static_cast<int>(hd);
+    rk.f16kv = s.kv_dtype == MZC_KV_FP16 ? 1 : 0;
     auto gemm = [&](const CUtensorMap& ta, const void* a_ptr, const mzc::GemmWeight& w, void* out,
                     int64_t N, int64_t K, int epi, const mzc::RowNorm* rn = nullptr) {
       double out_b = epi == mzc::EPI_ADD_F32 ? R * N * 8.0 : (epi == mzc::EPI_SWIGLU_BF16 ? R * N : R * N * 2.0);
@@ -707,14 +726,28 @@ mzc_status run_prefill(mzc_ctx* ctx, const int32_t* tokens, int64_t n, float* lo
           return mzc::launch_rmsnorm(ctx->d_x, W.attn_norm, cr, static_cast<int32_t>(d), s.rms_eps, ctx->d_h, cs,
                                      ctx->d_status);
         }));
-      CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16,
-               fold_in ? &rn_qkv : nullptr));
-      if (P.kv_wait_write[l] && n_prm_c > 0) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
-      CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
-        return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
-                                         ctx->d_cos, ctx->d_sin, ltab, ctx->nblk, ctx->d_pool,
-                                         ctx->st.pool_blocks(), s.kv_dtype, ctx->d_q, ctx->d_status, cs);
-      }));
+      const bool kv_wait = P.kv_wait_write[l] && n_prm_c > 0;
+      if (rope_rows && !kv_wait) {
+        rk.table = ltab;
+        bool launched = false;
+        const double qn = static_cast<double>(ctx->qkv_dim);
+        CKP(klaunch(ctx, MZC_K_GEMM, 2.0 * R * qn * dd, 2.0 * (R * dd + qn * dd) + rope_bytes / 2.0, 1, [&] {
+          return mzc::launch_gemm_splitk(ctx->tm_h, W.tm_qkv, ctx->d_qkv, cr, ctx->qkv_dim, d, mzc::EPI_QKV_ROPE,
+                                         ctx->num_sms, ctx->d_status, cs, &launched, fold_in ? &rn_qkv : nullptr,
+                                         &rk);
+        }));
+        if (!launched)
+          return bail(ctx->fail(MZC_ERR_CUDA, "the QKV projection with the rotary write did not launch"));
+      } else {
+        CKP(gemm(ctx->tm_h, ctx->d_h, W.tm_qkv, ctx->d_qkv, ctx->qkv_dim, d, mzc::EPI_STORE_BF16,
+                 fold_in ? &rn_qkv : nullptr));
+        if (kv_wait) CKP(cudaStreamWaitEvent(cs, ctx->ev_kv[l], 0));
+        CKP(klaunch(ctx, MZC_K_ROPE_KV, 0.0, rope_bytes, 1, [&] {
+          return mzc::launch_rope_kv_write(ctx->d_qkv, cpos, cr, s.n_q_heads, s.n_kv_heads, s.head_dim,
+                                           ctx->d_cos, ctx->d_sin, ltab, ctx->nblk, ctx->d_pool,
+                                           ctx->st.pool_blocks(), s.kv_dtype, ctx->d_q, ctx->d_status, cs);
+        }));
+      }
       const bool wait_rec = n_rec_c > 0 && P.kv_wait_rec[l];
       const bool wait_prm = n_prm_c > 0 && P.kv_wait_prompt[l];
       if (l == L - 1) {

@@ -41,7 +41,8 @@ class mzc_options(ctypes.Structure):
     _fields_ = [("pool_blocks", c_i64), ("max_rows", c_i64), ("host_store_bytes", c_i64),
                 ("overlap", c_i32), ("device", c_i32), ("swap_codec", c_i32),
                 ("wait_mode", c_i32), ("debug_checks", c_i32), ("read_swapped", c_i32),
-                ("compute_stream", c_vp), ("copy_stream", c_vp), ("separate_norm", c_i32)]
+                ("compute_stream", c_vp), ("copy_stream", c_vp), ("separate_norm", c_i32),
+                ("fused_rope", c_i32)]
 
 
 class mzc_layer_weights(ctypes.Structure):
@@ -243,13 +244,14 @@ def make_weights(weights: dict):
 
 def mzc_create(shape: dict, weights: dict, pool_blocks=0, max_rows=0, host_store_bytes=0,
                overlap=1, device=0, swap_codec=MZC_CODEC_NONE, wait_mode=MZC_WAIT_LAYER_EVENT,
-               debug_checks=0, compute_stream=None, copy_stream=None, read_swapped=0, separate_norm=0):
+               debug_checks=0, compute_stream=None, copy_stream=None, read_swapped=0, separate_norm=0,
+               fused_rope=0):
     """compute_stream / copy_stream: cudaStream_t handles (ints, e.g. a torch
     stream's cuda_stream) owned by the caller, or None."""
     sh = make_shape(shape)
     opt = mzc_options(pool_blocks, max_rows, host_store_bytes, overlap, device, swap_codec,
                       wait_mode, debug_checks, read_swapped, compute_stream, copy_stream,
-                      separate_norm)
+                      separate_norm, fused_rope)
     w, keep = make_weights(weights)
     out = c_vp()
     _call("mzc_create", ctypes.byref(sh), ctypes.byref(opt), ctypes.byref(w), ctypes.byref(out))

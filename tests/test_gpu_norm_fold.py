@@ -135,8 +135,10 @@ def test_folded_norm_prefill_matches_the_oracle(name):
     """A 200-row context prefill, a 37-row prompt prefill and two one-token
     steps (all folded) against the oracle's prefill of the same tokens: logits
     max-abs <= 2e-2, K/V max|d| / max|ref| <= 1e-2 per layer, as for the
-    separate-norm path, which runs beside it; the fold leaves one RMSNorm
-    launch a prefill."""
+    separate norm launches, which run beside it; the fold leaves one RMSNorm
+    launch a prefill.  The same with the rotary write inside the QKV
+    projection (option fused_rope): no rotary launch for the 5-256-row sets,
+    and every position it wrote matches."""
     sh = CASES[name]
     L = sh["n_layers"]
     w = synth.model_weights(sh)
@@ -154,10 +156,10 @@ def test_folded_norm_prefill_matches_the_oracle(name):
     steps = synth.tokens(synth.SEED_PROMPT, 22, 2, sh["vocab"])
     lg_steps = [oracle.prefill(sh, w, kv_ref, steps[i:i + 1], 237 + i) for i in range(2)]
     n_tok = 239
-    for sep in (0, 1):
-        c = m.mzc_create(sh, w, separate_norm=sep)
+    for sep, fused_rope in ((0, 0), (0, 1), (1, 0)):
+        c = m.mzc_create(sh, w, separate_norm=sep, fused_rope=fused_rope)
         try:
-            norms = []
+            norms, ropes = [], []
             lgs = []
             for toks in (ctx, prm, steps[:1], steps[1:]):
                 m.mzc_set_kernel_timing(c, 0)  # resets the launch counters
@@ -165,6 +167,7 @@ def test_folded_norm_prefill_matches_the_oracle(name):
                 m.mzc_prefill(c, toks, out)
                 lgs.append(out)
                 norms.append(m.mzc_kernel_stats(c, m.MZC_K_RMSNORM).launches)
+                ropes.append(m.mzc_kernel_stats(c, m.MZC_K_ROPE_KV).launches)
             assert np.max(np.abs(lgs[0] - lg_ctx)) < 2e-2
             assert np.max(np.abs(lgs[1] - lg_prm)) < 2e-2
             for i in range(2):
@@ -176,5 +179,8 @@ def test_folded_norm_prefill_matches_the_oracle(name):
             # separate: every layer's attention norm, the MLP norms of the first
             # L - 1 layers over all rows, the last layer's over the logits row
             assert norms == ([1] * 4 if sep == 0 else [2 * L] * 4)
+            # fused_rope: the rotary write runs inside the QKV projection for the
+            # 200- and 37-row prefills; one-row steps keep their rotary launch
+            assert ropes == ([0, 0, L, L] if fused_rope else [L] * 4)
         finally:
             m.mzc_destroy(c)
