@@ -31,7 +31,8 @@
  *     range: zero and magnitudes in [2^-14, 65504].  A bf16 K/V value below
  *     2^-14 keeps only fp16-subnormal precision, and one of 65520 or more
  *     does not fit at all: the prefill then fails with MZC_ERR_OVERFLOW.
- *     The activations the projections read (RMSNorm outputs, SwiGLU
+ *     The activations the projections read (RMSNorm outputs, or x * g where
+ *     the norm is folded into the projections: see separate_norm; SwiGLU
  *     outputs) and the q/k/v projection outputs are fp16 too, with the same
  *     check.
  */
@@ -54,8 +55,8 @@ typedef enum {
   MZC_ERR_CUDA = 5,    /* a CUDA runtime call failed; the text names it */
   MZC_ERR_TIMEOUT = 6, /* a bounded device wait gave up (kernel status word) */
   MZC_ERR_DEVICE = 7,  /* a device-side bounds check failed (kernel status word) */
-  MZC_ERR_OVERFLOW = 8 /* a device-side range check: an fp16 activation (RMSNorm output,
-                          q/k/v projection, SwiGLU output) or fp16-encoded K/V value reached
+  MZC_ERR_OVERFLOW = 8 /* a device-side range check: an fp16 activation (RMSNorm output or
+                          folded x * g, q/k/v projection, SwiGLU output) or fp16-encoded K/V value reached
                           65520 in magnitude and was stored as infinity (kernel status word);
                           the results of that call are not to be used */
 } mzc_status;
