@@ -39,6 +39,35 @@ def test_struct_sizes_match_c_layout():
     assert ctypes.sizeof(M.mzc_stats_t) == 80
 
 
+def test_binding_structs_match_the_header(tmp_path):
+    """The ctypes mirrors have the sizes and field offsets a C compiler gives
+    the structs of include/mzc.h (a field added on one side only shows)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    structs = {"mzc_model_shape": M.mzc_model_shape, "mzc_options": M.mzc_options,
+               "mzc_copy_run": M.mzc_copy_run, "mzc_stats_t": M.mzc_stats_t}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "mzc.h"', 'int main(void) {']
+    for name, cls in structs.items():
+        lines.append(f'  printf("{name} %zu\\n", sizeof({name}));')
+        for f in cls._fields_:
+            lines.append(f'  printf("{name}.{f[0]} %zu\\n", offsetof({name}, {f[0]}));')
+    lines += ['  return 0;', '}']
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-std=c99", "-I", inc, str(src), "-o", str(exe)], check=True)
+    got = dict(l.split() for l in subprocess.run([str(exe)], check=True, capture_output=True,
+                                                  text=True).stdout.splitlines())
+    for name, cls in structs.items():
+        assert int(got[name]) == ctypes.sizeof(cls), name
+        for f in cls._fields_:
+            assert int(got[f"{name}.{f[0]}"]) == getattr(cls, f[0]).offset, f"{name}.{f[0]}"
+
+
 SMALL = W.scaled(W.TINY, n_layers=3, max_ctx=640)
 
 
