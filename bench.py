@@ -929,9 +929,22 @@ def run_kernels(args):
         return fn, 4.0 * hd_ * hq_ * pairs, 2.0 * ctx * hkv_ * hd_ * 2 + 2.0 * n_rows * hq_ * hd_ * 2
     at_fn, at_fl, at_by = attn_case(4224, 8320, 32, 8, 64, 1)
     ad_fn, ad_fl, ad_by = attn_case(1, 32768, 24, 8, 128, 0)
+    # the folded RMSNorm's two halves at the same 128 rows: the down projection
+    # writing x * g and the per-tile sums of squares, then the QKV projection
+    # (3072 -> 5120) scaling its rows by rstd
+    h_sk = torch.empty((128, d), dtype=torch.int16, device="cuda")
+    ss_sk = torch.zeros((128, d // 128), device="cuda")
+    w_q = (torch.randn((5120, d), device="cuda", generator=gen) * 0.02).half().view(torch.int16)
+    o_q = torch.empty((128, 5120), dtype=torch.int16, device="cuda")
     cases = {
         "gemm_splitk_kernel": (lambda: m.mzc_k_gemm(a_sk, w_sk, o_sk, 128, d, 8192, 1),
                                2.0 * (128 * 8192 + d * 8192) + 128 * d * 8.0, 2.0 * 128 * d * 8192),
+        "gemm_splitk_kernel_norm_out": (
+            lambda: m.mzc_k_gemm_norm_out(a_sk, w_sk, o_sk, 128, d, 8192, g, h_sk, ss_sk, status),
+            2.0 * (128 * 8192 + d * 8192) + 128 * d * 10.0 + 128 * (d // 128) * 4.0, 2.0 * 128 * d * 8192),
+        "gemm_splitk_kernel_norm_in": (
+            lambda: m.mzc_k_gemm_norm_in(h_sk, w_q, o_q, 128, 5120, d, 0, ss_sk, 1e-5, status),
+            2.0 * (128 * d + 5120 * d) + 128 * 5120 * 2.0 + 128 * (d // 128) * 4.0, 2.0 * 128 * 5120 * d),
         "gemm_persistent_kernel": (lambda: m.mzc_k_gemm(a_p, w_p, o_p, M1, N1, K1, 2),
                                    2.0 * (M1 * K1 + N1 * K1) + M1 * N1, 2.0 * M1 * N1 * K1),
         "attn_tc_kernel": (at_fn, at_by, at_fl),
