@@ -31,6 +31,7 @@
 // Every thread of every CTA passes both cluster barriers exactly once (no
 // early exit on any path); the pipeline waits are bounded as elsewhere.
 #include <algorithm>
+#include <climits>
 #include <mutex>
 
 #include "kernels.hpp"
@@ -83,6 +84,11 @@ __device__ __forceinline__ uint2 pack4_f16(float a, float b, float c, float d) {
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
+// marks a row whose position lies outside the rotary tables and the block
+// table (no block-table entry takes this value: entries are blocks >= 0, -1
+// for none, -2 - i for host block i)
+constexpr int kNoPos = INT_MIN;
+
 // Partial layout: row r (0 .. MT*128) of 32 float4 chunks, chunk c stored at
 // c ^ (r & 7) so that eight lanes writing one chunk of eight rows hit eight
 // different bank groups.
@@ -105,8 +111,8 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
   __shared__ float s_rs[MT * SBM];  // folded RMSNorm: rstd of rows r_begin ..
-  // EPI_QKV_ROPE: position and physical block of rows r_begin .. (-2: the
-  // position is outside the rotary tables and the block table)
+  // EPI_QKV_ROPE: position and physical block of rows r_begin .. (kNoPos:
+  // the position is outside the rotary tables and the block table)
   __shared__ int s_pos[MT * SBM], s_phys[MT * SBM];
   volatile int* abort_flag = &s_abort;
 
@@ -211,7 +217,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
       // the rows' positions and KV blocks, looked up while the main loop runs
       for (int i = threadIdx.x - 64; r_begin + i < r_end; i += 128) {
         const int p = rk.pos[r_begin + i];
-        int ph = -2;
+        int ph = kNoPos;
         if (p >= 0 && (p >> 4) < rk.n_logical) ph = rk.table[p >> 4];
         s_pos[i] = p;
         s_phys[i] = ph;
@@ -286,7 +292,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
             const int col = nt * SBN + c * 4;
             const int head = col / rk.hd, e = col - head * rk.hd, half = rk.hd >> 1;
             const int p = s_pos[r - r_begin];
-            if (head < rk.hq + rk.hkv && s_phys[r - r_begin] != -2) {
+            if (head < rk.hq + rk.hkv && s_phys[r - r_begin] != kNoPos) {
               const int64_t t = static_cast<int64_t>(p) * half + (e < half ? e : e - half);
               rc[h] = *reinterpret_cast<const float4*>(rk.cos_t + t);
               rsn[h] = *reinterpret_cast<const float4*>(rk.sin_t + t);
@@ -338,7 +344,7 @@ __global__ void __launch_bounds__(192, 1) gemm_splitk_kernel(
           const int col = nt * SBN + c * 4;
           const int head = col / rk.hd, e = col - head * rk.hd, half = rk.hd >> 1;
           const int p = s_pos[r - r_begin], phys = s_phys[r - r_begin];
-          if (phys == -2) {
+          if (phys == kNoPos) {
             set_status(status, kStatusDevice);  // outside the rotary tables and the block table
           } else {
             float y0 = acc.x, y1 = acc.y, y2 = acc.z, y3 = acc.w;
