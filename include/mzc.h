@@ -473,8 +473,9 @@ mzc_status mzc_k_gemm(const uint16_t *a, const uint16_t *w, void *out, int64_t m
                       int64_t k, int32_t epilogue, void *stream);
 
 /* RMSNorm folded into the two projections around it, as mzc_prefill runs row
- * sets of 5-256 rows (the pre-norm of the decoder layer: RMSNorm(x) W^T =
- * diag(1 / RMS(x)) ((x * g) W^T), so the norm needs no launch of its own).
+ * sets of 5-256 rows (the pre-norms of the decoder layer the paper prefills,
+ * Sec. 2.1: RMSNorm(x) W^T = diag(1 / RMS(x)) ((x * g) W^T), so the norm needs
+ * no launch of its own).
  * m: 5..256 rows (MZC_ERR_INVALID otherwise).  All pointers DEVICE.
  *   mzc_k_gemm_norm_out: the residual add x fp32 [m][n] += A W^T (epilogue 1
  *     of mzc_k_gemm, on the split-K kernel; A fp16 [m][k], W fp16 [n][k]),
