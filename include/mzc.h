@@ -249,11 +249,15 @@ mzc_status mzc_restore_async(mzc_ctx *ctx);
 /* Declares the recompute of dropped positions [p, p+n): they are re-prefilled
  * against the resident prefix in the next mzc_prefill (or mzc_sync), fused
  * with its prompt rows.  [p, p+n) must equal the dropped range (MZC_ERR_RANGE
- * otherwise). */
+ * otherwise).  (The paper names recomputing the KV cache as the alternative
+ * to slow storage reads, Sec. 1; here it is the second restore path that
+ * Sec. 4.3's balance weighs against the host-link copy, for a backward-out
+ * tail, Sec. 4.4.) */
 mzc_status mzc_recompute_tail(mzc_ctx *ctx, int64_t p, int64_t n);
 
 /* Sets the policy MZC_AUTO evictions use and the per-unit profile that sizes
- * the hybrid split (profile may be NULL to keep the current one). */
+ * the hybrid split (profile may be NULL to keep the current one): Sec. 4.3's
+ * offline profile and the choice between its restore paths. */
 mzc_status mzc_set_policy(mzc_ctx *ctx, int32_t policy, const mzc_profile *profile);
 
 /* Hybrid split (pure host arithmetic): for an evicted tail [p, n_ctx) and a
@@ -351,13 +355,17 @@ mzc_status mzc_evict_size(mzc_ctx *ctx, int64_t bytes, int64_t *freed_out, int32
  * replay the policy's decision, e.g. with mzc_plan_evict_size).  Same errors. */
 mzc_status mzc_evict_size_plan(mzc_ctx *ctx, mzc_evict_plan *out);
 
-/* Shrinks the context to n_ctx positions (frees the blocks past it). */
+/* Shrinks the context to n_ctx positions (frees the blocks past it; the
+ * context-aware request of Sec. 2.2 continues from there). */
 mzc_status mzc_truncate(mzc_ctx *ctx, int64_t n_ctx);
 /* Runs any pending recompute, waits for both streams, and surfaces device
- * status words (MZC_ERR_TIMEOUT / MZC_ERR_DEVICE). */
+ * status words (MZC_ERR_TIMEOUT / MZC_ERR_DEVICE): the point where the
+ * paper's restore completes (Sec. 4.4, Fig. 8b: restore and prefill
+ * overlapped, then joined). */
 mzc_status mzc_sync(mzc_ctx *ctx);
 
-/* Residency of (layer, logical_block) and its physical block (-1 if none). */
+/* Residency of (layer, logical_block) and its physical block (-1 if none):
+ * the per-chunk state behind Sec. 4.2's chunk-pointer array. */
 mzc_status mzc_query(mzc_ctx *ctx, int32_t layer, int64_t logical_block, int32_t *state,
                      int32_t *phys);
 /* Reads one resident block's K and V ([n_kv_heads][16][head_dim], fp16 bits
@@ -368,6 +376,8 @@ mzc_status mzc_read_kv(mzc_ctx *ctx, int32_t layer, int64_t logical_block, void 
  * into host arrays [n_layers][n][n_kv_heads][head_dim].  Every block must be
  * RESIDENT. */
 mzc_status mzc_read_kv_all(mzc_ctx *ctx, int64_t n, float *k_host, float *v_host);
+/* Counts of the context's units by residency state and of the last restore
+ * and prefill (rows, copied bytes): the memory state of Sec. 4.2's units. */
 mzc_status mzc_stats(mzc_ctx *ctx, mzc_stats_t *out);
 /* Device time in ms of the last mzc_prefill: [0] the call on the compute
  * stream, [1] restore copies on the copy stream, [2] LM head, [3] TTFT on the
