@@ -201,6 +201,8 @@ typedef struct mzc_ctx mzc_ctx;
  * options may be NULL (defaults).  On failure *out is NULL. */
 mzc_status mzc_create(const mzc_model_shape *shape, const mzc_options *options,
                       const mzc_weights *weights, mzc_ctx **out);
+/* Frees every device buffer, the pinned store and the ctx's own streams (the
+ * memory the paper's OS would reclaim, Sec. 3.1). */
 mzc_status mzc_destroy(mzc_ctx *ctx);
 
 /* Prefill: appends tokens[0..n) at positions context_tokens.. and runs, in one
@@ -381,9 +383,9 @@ mzc_status mzc_read_kv_all(mzc_ctx *ctx, int64_t n, float *k_host, float *v_host
 mzc_status mzc_stats(mzc_ctx *ctx, mzc_stats_t *out);
 /* Device time in ms of the last mzc_prefill: [0] the call on the compute
  * stream, [1] restore copies on the copy stream, [2] LM head, [3] TTFT on the
- * device: from the start of the restore copies (or of the prefill when
- * nothing was restored) to the logits' arrival in host memory.  ms must hold
- * 4 floats; -1 marks a phase that did not run. */
+ * device (the paper's metric, Sec. 6.2): from the start of the restore copies
+ * (or of the prefill when nothing was restored) to the logits' arrival in
+ * host memory.  ms must hold 4 floats; -1 marks a phase that did not run. */
 mzc_status mzc_last_times(mzc_ctx *ctx, float *ms3);
 const char *mzc_last_error(mzc_ctx *ctx);
 
