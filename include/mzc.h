@@ -124,12 +124,13 @@ typedef struct {
   void *copy_stream;        /* cudaStream_t of the restore copies, owned by the caller;
                                NULL = own.  The same stream as compute_stream is accepted
                                and serializes restore and prefill (no overlap) */
-  int32_t separate_norm;    /* 0 (default): for row sets of 5-256 rows each RMSNorm after
+  int32_t separate_norm;    /* 0 (default): for row sets of 5-256 rows, for one-row steps
+                               and for the last layer's logits row, each RMSNorm after
                                the first is folded into the projections around it (the
-                               residual-add GEMM writes x * g and the rows' partial sums
-                               of squares; the next projection scales its rows by
+                               residual-add GEMM or GEMV writes x * g and partial sums of
+                               squares of x; the next projection scales its rows by
                                1 / RMS); 1: every RMSNorm runs as its own kernel, as for
-                               larger row sets (ablation).  Results agree within the
+                               other row sets (ablation).  Results agree within the
                                fp16 rounding of the projection inputs */
   int32_t fused_rope;       /* 1: for row sets of 5-256 rows the rotary embedding and
                                KV-block write run inside the QKV projection (its split-K
