@@ -237,3 +237,27 @@ def test_row_order_does_not_matter():
     kv_b = oracle.KVState(sh, 32)
     oracle.forward(sh, w, kv_b, toks[perm], perm, logits=False)
     assert np.array_equal(kv_a.k[:, :30], kv_b.k[:, :30])
+
+
+# ---- P-6: a library routine for the same operation ---------------------------
+
+@pytest.mark.parametrize("hq,hkv,hd", [(4, 2, 64), (24, 8, 128), (8, 8, 32)])
+def test_attention_matches_torch_sdpa(hq, hkv, hd):
+    """The oracle's causal GQA attention over positions equals torch's
+    scaled_dot_product_attention (CPU, float64) with each KV head repeated
+    over its query group and a key mask of key position <= query position."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(hq + hkv + hd)
+    ctx, n = 37, 6
+    q = rng.standard_normal((n, hq, hd)).astype(np.float32)
+    k = rng.standard_normal((ctx, hkv, hd)).astype(np.float32)
+    v = rng.standard_normal((ctx, hkv, hd)).astype(np.float32)
+    pos = np.array([0, 3, 17, 18, 30, 36])
+    got = oracle.attention(q, pos, k, v)
+    g = hq // hkv
+    qt = torch.from_numpy(q.astype(np.float64)).permute(1, 0, 2)                 # [hq][n][hd]
+    kt = torch.from_numpy(k.astype(np.float64)).permute(1, 0, 2).repeat_interleave(g, 0)
+    vt = torch.from_numpy(v.astype(np.float64)).permute(1, 0, 2).repeat_interleave(g, 0)
+    mask = torch.from_numpy(np.arange(ctx)[None, :] <= pos[:, None])              # [n][ctx]
+    want = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask)
+    np.testing.assert_allclose(got, want.permute(1, 0, 2).numpy(), rtol=2e-5, atol=2e-6)
