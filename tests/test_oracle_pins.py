@@ -261,3 +261,15 @@ def test_attention_matches_torch_sdpa(hq, hkv, hd):
     mask = torch.from_numpy(np.arange(ctx)[None, :] <= pos[:, None])              # [n][ctx]
     want = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask)
     np.testing.assert_allclose(got, want.permute(1, 0, 2).numpy(), rtol=2e-5, atol=2e-6)
+
+
+def test_linear_matches_a_float64_matmul_on_a_non_square_weight():
+    """x W^T with W [n_out][n_in] in bf16 bits, against numpy's float64 matmul
+    of the decoded weights (a transposed operand or a swapped dimension
+    fails on the 48 x 80 weight; the identity pin above cannot tell)."""
+    rng = np.random.default_rng(9)
+    x = rng.standard_normal((5, 80)).astype(np.float32)
+    w_bits = synth.normal_bf16(3, 77, (48, 80), sigma=0.05)
+    w = synth.bf16_bits_to_f32(w_bits).astype(np.float64)
+    want = x.astype(np.float64) @ w.T
+    np.testing.assert_allclose(oracle.linear(x, w_bits), want, rtol=1e-5, atol=1e-6)
