@@ -273,3 +273,17 @@ def test_linear_matches_a_float64_matmul_on_a_non_square_weight():
     w = synth.bf16_bits_to_f32(w_bits).astype(np.float64)
     want = x.astype(np.float64) @ w.T
     np.testing.assert_allclose(oracle.linear(x, w_bits), want, rtol=1e-5, atol=1e-6)
+
+
+def test_rmsnorm_matches_torch_rms_norm():
+    """RMSNorm with gains against torch.nn.functional.rms_norm in float64 on
+    random rows of varied scale."""
+    torch = pytest.importorskip("torch")
+    if not hasattr(torch.nn.functional, "rms_norm"):
+        pytest.skip("torch without rms_norm")
+    rng = np.random.default_rng(12)
+    x = (rng.standard_normal((7, 96)) * rng.uniform(0.01, 30.0, (7, 1))).astype(np.float32)
+    g = (1.0 + 0.3 * rng.standard_normal(96)).astype(np.float32)
+    want = torch.nn.functional.rms_norm(torch.from_numpy(x.astype(np.float64)), (96,),
+                                        torch.from_numpy(g.astype(np.float64)), eps=1e-5).numpy()
+    np.testing.assert_allclose(oracle.rmsnorm(x, g, 1e-5), want, rtol=2e-6, atol=1e-7)
