@@ -280,3 +280,36 @@ def test_attention_rejects_an_unaligned_pool_before_any_launch():
     for fn, extra in (("mzc_k_attention", (4096, None, 0)), ("mzc_k_attention_noalloc", (4096,))):
         args = [fake, fake, 1, 32, 8, 64, fake, 4, fake + 8, 8, 1, fake, *extra, None, None]
         assert M.status_of(fn, *args) == M.MZC_ERR_INVALID, fn
+
+
+def test_hybrid_split_balances_the_two_paths():
+    """Sec. 4.3's balance: with recompute priced at a constant c per row and
+    layer (projections linear in the rows, attention free, no fixed costs) and
+    copy at the link rate per block, the split gives the recompute path as
+    much of the evicted tail as keeps its per-layer time within the 95%
+    headroom of the copy path's: the next block would break it.  So the two
+    paths finish together, up to that headroom and one block.  (c is below
+    the copy time a recomputed token saves over all layers, so moving a token
+    to recompute always shortens the layer pipeline; above it the last
+    layer's longer compute, which runs after its copy lands, outweighs the
+    saving and the split stays at copy-only, as the limits test checks.)"""
+    sh = W.THREE_B
+    L, hkv, hd = sh["n_layers"], sh["n_kv_heads"], sh["head_dim"]
+    blk = 2 * hkv * 16 * hd * 2
+    for c_us, rate, (p, n, P) in ((0.01, 200.0, (0, 32768, 128)), (0.02, 100.0, (8192, 32768, 128)),
+                                  (0.05, 211.0, (16384, 32768, 256))):
+        assert c_us < L * blk / 16 / (rate * 1e9) * 1e6
+        prof = M.mzc_profile(rate, 128 * c_us, 512 * c_us, 2048 * c_us, 1e9, 0.0, 1e9, 0.0, 0.0)
+        s = m.mzc_plan_split(sh, prof, p, n, P)
+
+        def compute(split):  # one layer's recompute + prompt rows, seconds
+            return (split - p + P) * c_us * 1e-6
+
+        def copy(split):  # one layer's copied blocks, seconds
+            return -(-(n - split) // 16) * blk / (rate * 1e9)
+
+        assert p < s < n and (s - p) % 16 == 0
+        assert compute(s) <= 0.95 * copy(s)
+        assert compute(s + 16) > 0.95 * copy(s + 16)
+        # balanced: the two paths within the headroom plus a block of each other
+        assert abs(compute(s) - 0.95 * copy(s)) <= 16 * c_us * 1e-6 + blk / (rate * 1e9)
