@@ -10,7 +10,6 @@ forgotten, the KV heads or the layers missed) fails here."""
 import math
 import os
 
-import numpy as np
 
 import oracle
 import paper_2609_01338_gb300 as m
